@@ -1,0 +1,303 @@
+/*
+ * trident_scm.h -- C ABI of the Specialization Cache Module (SCM) library.
+ *
+ * The SCM is the paper's central artifact (Trident, §3.1 and Fig. 1c): an ordered
+ * set of versions, each a guard predicate G_i paired with the computation P_i captured
+ * under it, plus a dispatcher that runs the first P_i whose G_i holds (§3.2, Algorithm 1).
+ * A cache hit stays in native code from guard evaluation through argument preparation
+ * and the kernel launch; only a miss leaves the library, through a compile hook (§3.5).
+ *
+ * In this library P_i is a hand-written sm_103a CUDA kernel for one step of an LLM
+ * decoder layer's memory-bound chain (fused residual-add + RMSNorm, per-head q/k
+ * RMSNorm, RoPE with KV-cache append, SwiGLU, or the whole chain in one launch).
+ * The layer math is not given by the paper, which runs these operators inside the
+ * Qwen3-8B / DeepSeek-V2-Lite decode loops it evaluates (§4.1); the formulas each op
+ * computes are stated below, next to the op.
+ *
+ * Conventions for every entry point:
+ *   - Tensors are described, never owned: the caller owns every buffer and the stream.
+ *   - Strides and shapes are in ELEMENTS. Pointers are device addresses for tensors
+ *     whose device field is >= 0.
+ *   - Return values are trident_status codes. Values >= 0 are not errors. A miss is
+ *     never an error code, and an error never triggers the compile hook (§3.2, §3.4,
+ *     §3.5: "miss" and "error" stay distinct).
+ *   - On an error, trident_scm_last_error() returns a thread-local message.
+ *   - All functions are thread-safe unless stated otherwise. The hit path of
+ *     trident_scm_invoke takes no lock and allocates nothing.
+ */
+#ifndef TRIDENT_SCM_H
+#define TRIDENT_SCM_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define TRIDENT_ABI_VERSION 1
+#define TRIDENT_MAX_TENSORS 20
+#define TRIDENT_MAX_FIXED 8
+/* out_selected value for a sequence element that was not run (trident_scm_invoke_seq). */
+#define TRIDENT_NOT_RUN (-2)
+
+/* ---------------------------------------------------------------- status codes */
+typedef enum trident_status {
+  TRIDENT_OK = 0,             /* hit: version *out_selected ran (Algorithm 1, return o)      */
+  TRIDENT_MISS_HANDLED = 1,   /* every guard failed; the compile hook ran and succeeded     */
+  TRIDENT_MISS = 2,           /* every guard failed and no hook ran (Algorithm 1, MISS)     */
+  TRIDENT_ERR_INVALID = -1,   /* malformed arguments, descriptor or launch precondition     */
+  TRIDENT_ERR_CUDA = -2,      /* a CUDA call failed (launch, allocation, copy)              */
+  TRIDENT_ERR_HOOK = -3,      /* the compile hook returned non-zero                         */
+  TRIDENT_ERR_CAPACITY = -4,  /* the version table is full                                  */
+  TRIDENT_ERR_STATE = -5      /* the call is not allowed in this mode (e.g. dry-run launch) */
+} trident_status;
+
+/* ---------------------------------------------------------------- dtypes */
+typedef enum trident_dtype {
+  TRIDENT_BF16 = 1,  /* 2 bytes */
+  TRIDENT_FP16 = 2,  /* 2 bytes */
+  TRIDENT_FP32 = 3,  /* 4 bytes */
+  TRIDENT_I32 = 4,   /* 4 bytes */
+  TRIDENT_I64 = 5    /* 8 bytes */
+} trident_dtype;
+
+/* ---------------------------------------------------------------- operations
+ * Each op has a fixed tensor order ("slots"). T is the token count; "act" is the
+ * activation dtype (bf16, fp16, or fp32 where noted). All float math is fp32.
+ *
+ * TRIDENT_OP_ADD_RMSNORM (5 tensors; act = bf16 | fp16 | fp32; rank 2 [T,H] or 3 [B,S,H], T = B*S)
+ *   0 x [T,H] act   1 r [T,H] act   2 gamma [H] fp32   3 y [T,H] act (out)   4 r_out [T,H] act (out)
+ *   s = x + r;  r_out = round(s);  y = round(s * rsqrt(mean(s^2) + eps) * gamma)
+ *   In place: y may be x and r_out may be r (same pointer, shape and strides).
+ *
+ * TRIDENT_OP_ROPE_KV (6 tensors; act = bf16 | fp16)
+ *   0 q [T,Hq,D] act (in/out)  1 k [T,Hkv,D] act  2 v [T,Hkv,D] act  3 pos [T] i32
+ *   4 k_cache [Hkv,S,D] act (out)  5 v_cache [Hkv,S,D] act (out)
+ *   Rotate-half RoPE with inv_freq_i = theta^(-2i/D), i < D/2, angle a = pos * inv_freq_i:
+ *     x'_i = x_i cos a - x_{i+D/2} sin a,   x'_{i+D/2} = x_{i+D/2} cos a + x_i sin a.
+ *   q is rotated in place; k_cache[h, pos[t], :] = round(rope(k[t,h,:]));
+ *   v_cache[h, pos[t], :] = v[t,h,:] (bit copy). Positions in one call must be distinct.
+ *   A position outside [0,S) is skipped for that token (q, k and v untouched) and sets
+ *   bit TRIDENT_DEVERR_POS in the device status word (trident_scm_device_status).
+ *
+ * TRIDENT_OP_QKNORM_ROPE_KV (8 tensors; act = bf16 | fp16)
+ *   slots 0-5 as ROPE_KV, 6 gamma_q [D] fp32, 7 gamma_k [D] fp32.
+ *   Before the rotation each q head and each k head is RMS-normalised over its D
+ *   elements and scaled by gamma_q / gamma_k (eps from args); the result is not rounded
+ *   between the norm and the rotation.
+ *
+ * TRIDENT_OP_SWIGLU (3 tensors; act = bf16 | fp16 | fp32; rank 2 [T,I] or 3 [B,S,I])
+ *   0 g [T,I] act  1 u [T,I] act  2 out [T,I] act (out)
+ *   out = round(g / (1 + exp(-g)) * u).  In place: out may be g or u.
+ *
+ * TRIDENT_OP_LAYER_CHAIN (18 tensors; act = bf16 | fp16): one decoder layer's non-GEMM chain
+ *   0 h [T,H]  1 r0 [T,H]  2 gamma_attn [H]  3 x1 [T,H] out  4 r1 [T,H] out
+ *   5 q [T,Hq,D] in/out  6 k [T,Hkv,D]  7 v [T,Hkv,D]  8 pos [T] i32
+ *   9 k_cache [Hkv,S,D] out  10 v_cache [Hkv,S,D] out
+ *   11 attn_out [T,H]  12 gamma_mlp [H]  13 x2 [T,H] out  14 r2 [T,H] out
+ *   15 g [T,I]  16 u [T,I]  17 o [T,I] out
+ *   = ADD_RMSNORM(h, r0, gamma_attn -> x1, r1); ROPE_KV(q, k, v, pos, caches);
+ *     ADD_RMSNORM(attn_out, r1, gamma_mlp -> x2, r2); SWIGLU(g, u -> o).
+ *   The second norm reads r1 as rounded to act. In place: x1 = h, r1 = r0, x2 = attn_out,
+ *   r2 = r1, o = g or o = u.
+ *
+ * TRIDENT_OP_LAYER_CHAIN_QKNORM (20 tensors): LAYER_CHAIN with QKNORM_ROPE_KV instead of
+ *   ROPE_KV; 18 gamma_q [D] fp32, 19 gamma_k [D] fp32.
+ */
+typedef enum trident_op {
+  TRIDENT_OP_ADD_RMSNORM = 1,
+  TRIDENT_OP_ROPE_KV = 2,
+  TRIDENT_OP_QKNORM_ROPE_KV = 3,
+  TRIDENT_OP_SWIGLU = 4,
+  TRIDENT_OP_LAYER_CHAIN = 5,
+  TRIDENT_OP_LAYER_CHAIN_QKNORM = 6
+} trident_op;
+
+/* Layout class of an argument tuple (guard field, §2.2.1 "shape-related metadata").
+ * Over the op's activation tensors (not gamma, pos or the caches):
+ *   every tensor needs unit element stride and packed inner dims, else the tuple has
+ *   no layout class and matches no version;
+ *   CONTIG      every tensor's row stride equals its row width (a tensor with one row
+ *               always counts as contiguous, as torch's is_contiguous does);
+ *   ROWSTRIDED  not CONTIG, and every row stride is >= the row width.
+ * A version's layout is CONTIG or ROWSTRIDED (exact match) or ANY (either class). */
+typedef enum trident_layout {
+  TRIDENT_LAYOUT_CONTIG = 0,
+  TRIDENT_LAYOUT_ROWSTRIDED = 1,
+  TRIDENT_LAYOUT_ANY = 2
+} trident_layout;
+
+/* Kernel family of a version. AUTO picks VECTOR when the version allows it. */
+typedef enum trident_variant {
+  TRIDENT_VARIANT_AUTO = 0,
+  TRIDENT_VARIANT_GENERIC = 1,  /* scalar element access: any alignment, any row width  */
+  TRIDENT_VARIANT_VECTOR = 2    /* 128/256-bit accesses: align_bytes 16, supported sizes */
+} trident_variant;
+
+/* Bits of the device status word. */
+#define TRIDENT_DEVERR_POS 0x1u   /* a RoPE/KV position was outside [0, S) */
+
+/* Option flags of trident_scm_create. */
+#define TRIDENT_OPT_DRY_RUN 0x1        /* no CUDA at all: invoke selects and calls the hook,
+                                          but launches nothing (host-only testing) */
+#define TRIDENT_OPT_NO_ALIAS_CHECK 0x2 /* skip the output-overlap launch precondition */
+#define TRIDENT_OPT_PDL 0x4            /* launch with programmatic stream serialisation */
+#define TRIDENT_OPT_TIMING 0x8         /* record host ns per hit (trident_scm_host_times) */
+
+/* ---------------------------------------------------------------- structs */
+/* Caller-owned tensor descriptor (DLPack-like, §3.4: tensors cross the boundary as
+ * descriptors). 88 bytes. */
+typedef struct trident_tensor {
+  void* data;            /* device address (or host address if device < 0); may be NULL
+                            only when the tensor has no elements */
+  int64_t shape[4];      /* first ndim entries used, each >= 0 */
+  int64_t stride[4];     /* elements, each >= 0 */
+  int32_t dtype;         /* trident_dtype */
+  int32_t ndim;          /* 1..4 */
+  int32_t device;        /* CUDA ordinal, or -1 for host memory (matches no version) */
+  int32_t reserved;
+} trident_tensor;
+
+/* One invocation's argument tuple: the op, its tensors in slot order, and scalars. */
+typedef struct trident_args {
+  int32_t op;            /* trident_op */
+  int32_t ntensors;      /* must equal the op's slot count */
+  double eps;            /* RMSNorm epsilon (runtime scalar, not guarded), must be >= 0 */
+  double rope_theta;     /* RoPE base; a specialised constant (guarded by equality, §3.3) */
+  int32_t flags;         /* reserved, must be 0 */
+  int32_t reserved;
+  trident_tensor t[TRIDENT_MAX_TENSORS];
+} trident_args;
+
+/* Descriptor of one version (specialisation). register_spec copies it. */
+typedef struct trident_spec_desc {
+  int32_t op;                       /* trident_op                                        */
+  int32_t dtype;                    /* activation dtype                                  */
+  int32_t rank;                     /* rank of slot 0 (2 or 3 for ADD_RMSNORM/SWIGLU,
+                                       3 for ROPE ops, 2 for the chains)                  */
+  int32_t layout;                   /* trident_layout                                    */
+  int64_t fixed[TRIDENT_MAX_FIXED]; /* fixed sizes: ADD_RMSNORM {H}; SWIGLU {I};
+                                       ROPE ops {Hq, Hkv, D, S};
+                                       chains {H, Hq, Hkv, D, S, I}; unused entries 0    */
+  int64_t tok_lo, tok_hi;           /* inclusive token-count bucket, 1 <= lo <= hi       */
+  int32_t align_bytes;              /* 16: every pointer and row stride 16-byte aligned;
+                                       or the element size (no extra requirement)        */
+  int32_t device;                   /* CUDA ordinal; must equal the SCM's device         */
+  int32_t variant;                  /* trident_variant                                   */
+  int32_t reserved;
+  double rope_theta;                /* ROPE ops and chains: guarded constant; else 0     */
+} trident_spec_desc;
+
+typedef struct trident_scm_options {
+  int32_t device;        /* CUDA ordinal the SCM launches on (ignored for DRY_RUN) */
+  int32_t max_specs;     /* capacity of the version table, 1..4096 (0 = 256)       */
+  int32_t flags;         /* TRIDENT_OPT_*                                           */
+  int32_t timing_ring;   /* samples kept by TRIDENT_OPT_TIMING (0 = 65536)          */
+} trident_scm_options;
+
+typedef struct trident_scm_stats_t {
+  uint64_t invokes;         /* calls of invoke (each element of invoke_seq counts)  */
+  uint64_t hits;            /* guard hits that launched (or would, in dry-run)       */
+  uint64_t misses;          /* calls where every guard failed                        */
+  uint64_t hook_calls;      /* misses that called the hook                           */
+  uint64_t hook_failures;   /* hook calls that returned non-zero                     */
+  uint64_t hook_registered; /* versions registered from inside a hook                */
+  uint64_t err_invalid;     /* ERR_INVALID returns (validation or precondition)      */
+  uint64_t err_cuda;        /* ERR_CUDA returns                                      */
+  uint64_t guard_evals;     /* versions whose guard was evaluated                    */
+  int32_t num_specs;        /* versions in the current table                         */
+  int32_t reserved;
+} trident_scm_stats_t;
+
+typedef struct trident_scm trident_scm_t; /* opaque; owns the table, kernels and device state */
+
+/* Compile hook, called by invoke only on a miss (§3.5: an empty SCM takes the same
+ * path on its first call). The hook must produce the result of this call (§3.5: the
+ * call that triggered compilation returns the captured result), for example by
+ * registering a version and re-invoking, or by invoking a second SCM. It may call
+ * register_spec and invoke on `scm` (a miss inside a hook does not call the hook
+ * again). It writes the index it registered, or -1, to *out_registered, and returns
+ * 0 on success or non-zero on failure (invoke then returns TRIDENT_ERR_HOOK). */
+typedef int32_t (*trident_compile_hook)(void* user, trident_scm_t* scm, const trident_args* args,
+                                        void* stream, int32_t* out_registered);
+
+/* ---------------------------------------------------------------- entry points */
+
+/* Version of this ABI (TRIDENT_ABI_VERSION). */
+int32_t trident_abi_version(void);
+
+/* Creates an empty SCM (§3.5: an empty SCM takes the miss path first).
+ * opt may be NULL (device 0, 256 versions, no flags). hook and user may be NULL.
+ * Without TRIDENT_OPT_DRY_RUN this initialises CUDA on opt->device and allocates the
+ * device status word. *out receives the handle; the caller frees it with destroy.
+ * Errors: ERR_INVALID (bad options or out == NULL), ERR_CUDA. */
+int32_t trident_scm_create(const trident_scm_options* opt, trident_compile_hook hook, void* user,
+                           trident_scm_t** out);
+
+/* Appends one version (§3.5: versions are tried in creation order). The descriptor is
+ * validated and copied; its kernel entry is resolved now, so the hit path does no
+ * lookup (§3.3: the kernel entry is resolved when the specialisation is built). RoPE
+ * versions build a cos/sin table for (theta, D, S) in fp64, rounded to fp32, shared by
+ * versions with equal (theta, D, S). Readers see the new table atomically (copy-on-write);
+ * calls already running keep the table they loaded. May be called from a hook.
+ * *out_index (may be NULL) receives the new version's index.
+ * Errors: ERR_INVALID (descriptor), ERR_CAPACITY (table full), ERR_CUDA. */
+int32_t trident_scm_register_spec(trident_scm_t* scm, const trident_spec_desc* desc,
+                                  int32_t* out_index);
+
+/* Ordered dispatch (§3.2, Algorithm 1). Validates args (ERR_INVALID, the hook is not
+ * called), then tries versions 0..n-1 in order; the first whose guard holds is
+ * selected, its launch preconditions are checked (output overlap, ERR_INVALID), its
+ * kernel parameters are packed and it is launched on `stream` (a cudaStream_t; NULL is
+ * the legacy default stream). Returns OK with *out_selected = index. If every guard
+ * fails: calls the hook (MISS_HANDLED, *out_selected = the index the hook registered
+ * or -1), or returns MISS with *out_selected = -1 when no hook ran. A failed launch
+ * returns ERR_CUDA at once; no further version is tried (Algorithm 1, raise e).
+ * out_selected may be NULL. */
+int32_t trident_scm_invoke(trident_scm_t* scm, const trident_args* args, void* stream,
+                           int32_t* out_selected);
+
+/* Invokes args[0..n-1] in order with one call (one boundary crossing per decoder step).
+ * Each element behaves as trident_scm_invoke. Stops at the first element that returns
+ * an error or MISS and returns that status; the elements after it get TRIDENT_NOT_RUN
+ * in out_selected (n entries, may be NULL). Returns OK if all hit, else MISS_HANDLED
+ * if some misses were handled. */
+int32_t trident_scm_invoke_seq(trident_scm_t* scm, const trident_args* args, int32_t n,
+                               void* stream, int32_t* out_selected);
+
+/* Selection only: validation plus Algorithm 1's guard loop, with no launch, no hook
+ * and no statistics. Returns OK (*out_selected = index), MISS (-1) or ERR_INVALID.
+ * Needs no GPU. */
+int32_t trident_scm_select(const trident_scm_t* scm, const trident_args* args,
+                           int32_t* out_selected);
+
+/* Copies the counters into *out. */
+int32_t trident_scm_stats(const trident_scm_t* scm, trident_scm_stats_t* out);
+
+/* Copies per-version hit counts into out[0..cap-1]; *n (may be NULL) gets the count. */
+int32_t trident_scm_spec_hits(const trident_scm_t* scm, uint64_t* out, int32_t cap, int32_t* n);
+
+/* With TRIDENT_OPT_TIMING: copies the host nanoseconds of the most recent hits (entry
+ * of invoke to return, launch included) into out[0..cap-1], oldest first; *n gets the
+ * count. Samples are recorded per hit, so concurrent invokers may interleave. */
+int32_t trident_scm_host_times(const trident_scm_t* scm, uint32_t* out, int32_t cap, int32_t* n);
+
+/* Reads the device status word (TRIDENT_DEVERR_* bits) after synchronising `stream`;
+ * clears it when clear != 0. Errors: ERR_STATE in dry-run mode, ERR_CUDA. */
+int32_t trident_scm_device_status(trident_scm_t* scm, void* stream, uint32_t* out_bits,
+                                  int32_t clear);
+
+/* Frees the SCM, its tables and device memory. The caller must ensure no call on it
+ * is running and its kernels have finished. NULL is ignored. */
+void trident_scm_destroy(trident_scm_t* scm);
+
+/* Thread-local message of the last error returned on this thread ("" if none). */
+const char* trident_scm_last_error(void);
+
+/* Static name of a status code. */
+const char* trident_status_name(int32_t status);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* TRIDENT_SCM_H */
