@@ -1,0 +1,725 @@
+"""Benchmark of the SCM hot path on GB300: one JSON line on stdout (rank 0).
+
+Headline ("value"): microseconds per decoder-layer step of the Llama-style non-GEMM chain
+at 64 tokens (H 4096, 32/8 heads, D 128, I 14336, theta 5e5, KV cache [8, 8192, 128]):
+one trident_scm_invoke per step from Python -- guards, argument packing and one fused
+launch -- timed with CUDA events over K back-to-back steps, inputs rotated over enough
+buffer sets that the working set exceeds twice the L2.
+
+Also reported on the same line: every token count of that workload fused and unfused,
+the 36-layer Qwen3-style step, host nanoseconds per cache hit (single add+RMSNorm call,
+1 token), the 100k-call dynamic-shape guard stress (hit/miss counts checked against the
+oracle replay), the HBM bandwidth sweep (add+RMSNorm and SwiGLU, 1..32768 tokens), the
+roofline of the dominant kernel, the end-to-end step with host copies, and the CPU
+oracle as a reported baseline.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl reference] [--quick]
+"""
+import argparse
+import ctypes
+import json
+import math
+import os
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "us per decoder-layer step (host dispatch+device) at 1-64 tok; HBM GB/s vs 8 TB/s"
+UNIT = "us/step"
+HEADLINE_T = 64
+L2_BYTES = 129 * 2 ** 20
+NOMINAL_HBM_GBS = 8000.0
+
+
+def measured_peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), "measured"
+    except Exception:
+        return 6800.0, "fallback"
+
+
+# ---------------------------------------------------------------------------- algorithmic bytes
+def chain_bytes_per_token(cfg, fused=True):
+    """Bytes one token moves through the layer chain (bf16 activations)."""
+    H, Hq, Hkv, D, I = cfg["H"], cfg["Hq"], cfg["Hkv"], cfg["D"], cfg["I"]
+    norm1 = 4 * H * 2                       # read h, r0; write x1, r1
+    norm2 = (3 if fused else 4) * H * 2     # read attn_out (+ r1 unfused); write x2, r2
+    rope = (2 * Hq * D + 2 * Hkv * D + 2 * Hkv * D) * 2 + 4 + (D // 2) * 8  # q in/out, k in/out, v in/out, pos, cos/sin
+    swiglu = 3 * I * 2
+    return norm1 + norm2 + rope + swiglu
+
+
+def chain_bytes_per_launch(cfg, T, fused=True):
+    g = 2 * cfg["H"] * 4 + (2 * cfg["D"] * 4 if cfg.get("qknorm") else 0)
+    return T * chain_bytes_per_token(cfg, fused) + g
+
+
+# ---------------------------------------------------------------------------- clocks
+class ClockSampler:
+    """nvidia-smi sampling during the measured region (stopped by the caller)."""
+
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, device_index):
+        self.proc = None
+        self.dev = device_index
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", str(device_index), "--query-gpu=" + self.Q,
+                                          "--format=csv,noheader,nounits", "-lms", "100"],
+                                         stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except Exception:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            out, _ = self.proc.communicate(timeout=5)
+        except Exception:
+            self.proc.kill()
+            out, _ = self.proc.communicate()
+        sm, mx, reasons = [], 0.0, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in out.strip().splitlines():
+            f = [x.strip() for x in line.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                sm.append(float(f[1]))
+                mx = max(mx, float(f[2]))
+            except ValueError:
+                continue
+            for n, v in zip(names, f[5:9]):
+                if v.lower() == "active":
+                    reasons.add(n)
+        if not sm:
+            return None
+        busy = [s for s in sm if s > 0.5 * mx] or sm
+        return {"sm_mhz": float(np.median(busy)), "sm_max_mhz": mx, "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+# ---------------------------------------------------------------------------- oracle (reference arm)
+def oracle_layer_step_us(cfg, T, budget_s, seed=0):
+    """The CPU oracle timed on a bounded sample of layer steps at T tokens."""
+    from oracle import layer as L
+    from paper_2609_37241_gb300 import synth
+    g = np.random.default_rng(seed)
+    inp = synth.layer_inputs(g, T, cfg)
+    L.layer_chain(inp, cfg["theta"], cfg["eps"], synth.BF16, qknorm=cfg.get("qknorm", False))  # warm
+    n, t0 = 0, time.perf_counter()
+    while True:
+        L.layer_chain(inp, cfg["theta"], cfg["eps"], synth.BF16, qknorm=cfg.get("qknorm", False))
+        n += 1
+        el = time.perf_counter() - t0
+        if el >= budget_s and n >= 2:
+            break
+    return el / n * 1e6, n
+
+
+# ---------------------------------------------------------------------------- GPU side
+class Ctx:
+    def __init__(self, device):
+        import torch
+        from paper_2609_37241_gb300 import scm as S
+        from paper_2609_37241_gb300 import synth
+        self.torch, self.S, self.synth = torch, S, synth
+        self.dev = device
+        self.stream = torch.cuda.current_stream()
+        self.sp = ctypes.c_void_p(self.stream.cuda_stream)
+        self.L = S.lib()
+        self.launches = 0
+
+    def events(self):
+        t = self.torch
+        return t.cuda.Event(enable_timing=True), t.cuda.Event(enable_timing=True)
+
+
+class ChainSets:
+    """R rotating input/output sets of one decoder layer at T tokens, carved from arenas,
+    plus per-layer norm weights and KV caches."""
+
+    def __init__(self, c, cfg, T, layers=1, min_bytes=2 * L2_BYTES, max_sets=4096, seed=0):
+        t, synth = c.torch, c.synth
+        self.cfg, self.T, self.layers = cfg, T, layers
+        H, Hq, Hkv, D, S, I = (cfg[k] for k in ("H", "Hq", "Hkv", "D", "S", "I"))
+        per_set = chain_bytes_per_token(cfg) * T
+        R = max(layers, int(math.ceil(min_bytes / per_set)))
+        R = min(max_sets, int(math.ceil(R / layers)) * layers)
+        self.R = R
+        W = (Hq + 2 * Hkv) * D
+        bf = t.bfloat16
+        dev = c.dev
+        self.h = synth.act_device((R, T, H), synth.BF16, seed + 1, dev)
+        self.r0 = synth.act_device((R, T, H), synth.BF16, seed + 2, dev)
+        self.ao = synth.act_device((R, T, H), synth.BF16, seed + 3, dev)
+        self.qkv = synth.act_device((R, T, W), synth.BF16, seed + 4, dev)
+        self.gu = synth.act_device((R, T, 2 * I), synth.BF16, seed + 5, dev)
+        self.x1 = t.empty((R, T, H), dtype=bf, device=dev)
+        self.r1 = t.empty((R, T, H), dtype=bf, device=dev)
+        self.x2 = t.empty((R, T, H), dtype=bf, device=dev)
+        self.r2 = t.empty((R, T, H), dtype=bf, device=dev)
+        self.o = t.empty((R, T, I), dtype=bf, device=dev)
+        g = np.random.default_rng(seed)
+        self.pos = t.from_numpy(np.stack([synth.positions(g, T, S) for _ in range(R)])).to(dev)
+        self.ga = [synth.gamma_device(H, seed + 10 + l, dev) for l in range(layers)]
+        self.gm = [synth.gamma_device(H, seed + 100 + l, dev) for l in range(layers)]
+        self.gq = [synth.gamma_device(D, seed + 200 + l, dev) for l in range(layers)]
+        self.gk = [synth.gamma_device(D, seed + 300 + l, dev) for l in range(layers)]
+        self.kc = [t.zeros((Hkv, S, D), dtype=bf, device=dev) for _ in range(layers)]
+        self.vc = [t.zeros((Hkv, S, D), dtype=bf, device=dev) for _ in range(layers)]
+
+    def slots(self, i, layer=0):
+        cfg = self.cfg
+        Hq, Hkv, D, I = cfg["Hq"], cfg["Hkv"], cfg["D"], cfg["I"]
+        T = self.T
+        qkv = self.qkv[i]
+        q = qkv[:, :Hq * D].view(T, Hq, D)
+        k = qkv[:, Hq * D:(Hq + Hkv) * D].view(T, Hkv, D)
+        v = qkv[:, (Hq + Hkv) * D:].view(T, Hkv, D)
+        gu = self.gu[i]
+        ts = [self.h[i], self.r0[i], self.ga[layer], self.x1[i], self.r1[i], q, k, v, self.pos[i],
+              self.kc[layer], self.vc[layer], self.ao[i], self.gm[layer], self.x2[i], self.r2[i],
+              gu[:, :I], gu[:, I:], self.o[i]]
+        if cfg.get("qknorm"):
+            ts += [self.gq[layer], self.gk[layer]]
+        return ts
+
+    def fused_args(self, c, i, layer=0):
+        S = c.S
+        op = S.OP_LAYER_CHAIN_QKNORM if self.cfg.get("qknorm") else S.OP_LAYER_CHAIN
+        return S.make_args(op, self.slots(i, layer), eps=self.cfg["eps"], rope_theta=self.cfg["theta"])
+
+    def unfused_args(self, c, i, layer=0):
+        S = c.S
+        ts = self.slots(i, layer)
+        (h, r0, ga, x1, r1, q, k, v, pos, kc, vc, ao, gm, x2, r2, g, u, o) = ts[:18]
+        if self.cfg.get("qknorm"):
+            rope = S.make_args(S.OP_QKNORM_ROPE_KV, [q, k, v, pos, kc, vc, ts[18], ts[19]],
+                               eps=self.cfg["eps"], rope_theta=self.cfg["theta"])
+        else:
+            rope = S.make_args(S.OP_ROPE_KV, [q, k, v, pos, kc, vc], rope_theta=self.cfg["theta"])
+        return [S.make_args(S.OP_ADD_RMSNORM, [h, r0, ga, x1, r1], eps=self.cfg["eps"]), rope,
+                S.make_args(S.OP_ADD_RMSNORM, [ao, r1, gm, x2, r2], eps=self.cfg["eps"]),
+                S.make_args(S.OP_SWIGLU, [g, u, o])]
+
+
+def layer_scm(c, cfg, pdl=True, timing=False):
+    """One SCM holding the layer's versions: the fused chain (index 0), then the four
+    single-step versions, all for token buckets 1..4096 and row-strided q/k/v and g/u."""
+    S = c.S
+    flags = (S.OPT_PDL if pdl else 0) | (S.OPT_TIMING if timing else 0)
+    s = S.Scm(device=c.dev.index or 0, flags=flags)
+    qk = cfg.get("qknorm", False)
+    fixed = [cfg[k] for k in ("H", "Hq", "Hkv", "D", "S", "I")]
+    op = S.OP_LAYER_CHAIN_QKNORM if qk else S.OP_LAYER_CHAIN
+    for lay in (S.LAYOUT_ROWSTRIDED, S.LAYOUT_CONTIG):
+        s.register(S.make_spec(op, S.BF16, fixed, 1, 4096, layout=lay, rope_theta=cfg["theta"]))
+    s.register(S.make_spec(S.OP_ADD_RMSNORM, S.BF16, [cfg["H"]], 1, 4096))
+    rop = S.OP_QKNORM_ROPE_KV if qk else S.OP_ROPE_KV
+    for lay in (S.LAYOUT_ROWSTRIDED, S.LAYOUT_CONTIG):
+        s.register(S.make_spec(rop, S.BF16, fixed[1:5], 1, 4096, layout=lay, rope_theta=cfg["theta"]))
+        s.register(S.make_spec(S.OP_SWIGLU, S.BF16, [cfg["I"]], 1, 4096, layout=lay))
+    return s
+
+
+def time_steps(c, fn, K, W):
+    """Runs fn(i) for W warm-up then K timed steps; returns (us per step on the device
+    clock, host us per step)."""
+    t = c.torch
+    for i in range(W):
+        fn(i)
+    t.cuda.synchronize()
+    e0, e1 = c.events()
+    h0 = time.perf_counter()
+    e0.record(c.stream)
+    for i in range(K):
+        fn(W + i)
+    e1.record(c.stream)
+    h1 = time.perf_counter()
+    t.cuda.synchronize()
+    return e0.elapsed_time(e1) * 1e3 / K, (h1 - h0) * 1e6 / K
+
+
+def bench_layer(c, cfg, T, K, W, layers=1, min_bytes=2 * L2_BYTES):
+    """Fused and unfused layer steps at T tokens (one Python call per step)."""
+    S = c.S
+    sets = ChainSets(c, cfg, T, layers=layers, min_bytes=min_bytes)
+    scm = layer_scm(c, cfg)
+    R = sets.R
+    fused = [sets.fused_args(c, i, i % layers) for i in range(R)]
+    unf = [(S.trident_args * 4)(*sets.unfused_args(c, i, i % layers)) for i in range(R)]
+    inv, seq = c.L.trident_scm_invoke, c.L.trident_scm_invoke_seq
+    h, sp = scm.h, c.sp
+    fref = [ctypes.byref(a) for a in fused]
+    if layers == 1:
+        f_fused = lambda i: inv(h, fref[i % R], sp, None)
+        f_unf = lambda i: seq(h, unf[i % R], 4, sp, None)
+        n_launch = (1, 4)
+    else:  # one step = `layers` layers through one call
+        groups = R // layers
+        farr = [(S.trident_args * layers)(*fused[g * layers:(g + 1) * layers]) for g in range(groups)]
+        uarr = [(S.trident_args * (4 * layers))(*[a for l in range(layers) for a in
+                                                   sets.unfused_args(c, g * layers + l, l)])
+                for g in range(groups)]
+        f_fused = lambda i: seq(h, farr[i % groups], layers, sp, None)
+        f_unf = lambda i: seq(h, uarr[i % groups], 4 * layers, sp, None)
+        n_launch = (layers, 4 * layers)
+    st, sel = S.trident_scm_invoke(h, fused[0], c.sp.value)
+    assert st == S.OK and sel in (0, 1), S.trident_scm_last_error()
+    fus_dev, fus_host = time_steps(c, f_fused, K, W)
+    unf_dev, unf_host = time_steps(c, f_unf, K, W)
+    c.launches += K * (n_launch[0] + n_launch[1])
+    # device throughput floor: the same launches issued from one native call
+    nat = min(K, R if layers == 1 else R)
+    if layers == 1:
+        arr = (S.trident_args * nat)(*fused[:nat])
+        nat_fn = lambda i: seq(h, arr, nat, sp, None)
+        nat_us, _ = time_steps(c, nat_fn, 4, 2)
+        nat_us /= nat
+        c.launches += 4 * nat
+    else:
+        nat_us = None
+    st, bits = S.trident_scm_device_status(h, c.sp.value)
+    assert st == S.OK and bits == 0
+    scm.close()
+    res = dict(fused_us=round(fus_dev, 3), fused_host_us=round(fus_host, 3), unfused_us=round(unf_dev, 3),
+               unfused_host_us=round(unf_host, 3), launches_per_step=list(n_launch), sets=R,
+               working_set_mb=round(R * chain_bytes_per_token(cfg) * T / 2 ** 20, 1))
+    if nat_us is not None:
+        res["fused_native_seq_us"] = round(nat_us, 3)
+    return res, sets
+
+
+def bench_e2e(c, cfg, T, K, W):
+    """End to end through the public API: per step, pinned host -> device copies of the
+    layer's inputs, one invoke, device -> host copies of its outputs."""
+    t, S = c.torch, c.S
+    sets = ChainSets(c, cfg, T, min_bytes=0, max_sets=1)
+    scm = layer_scm(c, cfg)
+    a = sets.fused_args(c, 0)
+    pin = lambda x: t.empty(x.shape, dtype=x.dtype, pin_memory=True).copy_(x)
+    ins = [(sets.h[0], pin(sets.h[0])), (sets.r0[0], pin(sets.r0[0])), (sets.ao[0], pin(sets.ao[0])),
+           (sets.qkv[0], pin(sets.qkv[0])), (sets.gu[0], pin(sets.gu[0])), (sets.pos[0], pin(sets.pos[0]))]
+    outs = [(sets.x1[0], pin(sets.x1[0])), (sets.x2[0], pin(sets.x2[0])), (sets.r2[0], pin(sets.r2[0])),
+            (sets.o[0], pin(sets.o[0]))]
+    inv = c.L.trident_scm_invoke
+    ar = ctypes.byref(a)
+
+    def step(i):
+        for d, h in ins:
+            d.copy_(h, non_blocking=True)
+        inv(scm.h, ar, c.sp, None)
+        for d, h in outs:
+            h.copy_(d, non_blocking=True)
+
+    us, host_us = time_steps(c, step, K, W)
+    c.launches += K
+    bi = sum(h.numel() * h.element_size() for _, h in ins)
+    bo = sum(h.numel() * h.element_size() for _, h in outs)
+    scm.close()
+    return dict(value=round(us, 3), unit=UNIT, h2d_bytes_per_step=int(bi), d2h_bytes_per_step=int(bo))
+
+
+def bench_host_hit(c, n=1000):
+    """Single add+RMSNorm, 1 token, H 4096; four versions (fp16 contig, fp16 strided,
+    bf16 strided, bf16 contig) so each hit evaluates four guards. Host ns per hit from
+    the library's own clock, and per call as seen from Python."""
+    t, S, synth = c.torch, c.S, c.synth
+    s = S.Scm(device=c.dev.index or 0, flags=S.OPT_TIMING)
+    for dt in (S.FP16, S.BF16):
+        for lay in ((S.LAYOUT_CONTIG, S.LAYOUT_ROWSTRIDED) if dt == S.FP16 else
+                    (S.LAYOUT_ROWSTRIDED, S.LAYOUT_CONTIG)):
+            s.register(S.make_spec(S.OP_ADD_RMSNORM, dt, [4096], 1, 1, layout=lay))
+    g = np.random.default_rng(0)
+    x = c.synth.bits_to_torch(synth.act(g, (1, 4096), synth.BF16), synth.BF16).to(c.dev)
+    r = c.synth.bits_to_torch(synth.act(g, (1, 4096), synth.BF16), synth.BF16).to(c.dev)
+    gam = t.from_numpy(synth.gamma(g, 4096)).to(c.dev)
+    y, ro = t.empty_like(x), t.empty_like(r)
+    a = S.make_args(S.OP_ADD_RMSNORM, [x, r, gam, y, ro], eps=1e-6)
+    inv, ar, sel = c.L.trident_scm_invoke, ctypes.byref(a), ctypes.c_int32(-1)
+    for _ in range(50):
+        inv(s.h, ar, c.sp, ctypes.byref(sel))
+    t.cuda.synchronize()
+    # drop the warm-up samples: restart the SCM's ring by reading the last n only
+    h0 = time.perf_counter()
+    for _ in range(n):
+        inv(s.h, ar, c.sp, ctypes.byref(sel))
+    h1 = time.perf_counter()
+    t.cuda.synchronize()
+    st, ns = S.trident_scm_host_times(s.h, n)
+    hits = S.trident_scm_spec_hits(s.h)[1]
+    ns = np.array(ns[-n:], np.float64)
+    c.launches += n
+    s.close()
+    return dict(hits_on_bf16_contig=int(hits[3]), calls=n, selected=sel.value,
+                median_ns=float(np.median(ns)), p99_ns=float(np.percentile(ns, 99)),
+                min_ns=float(ns.min()), python_call_us=round((h1 - h0) * 1e6 / n, 3))
+
+
+def bench_guard_stress(c, n_calls=None):
+    """100k add+RMSNorm calls with T ~ Zipf(1.2) on [1,512], 10% fp16, 5% row-strided.
+    Static mode: 16 pre-registered versions (buckets 1..128 x {bf16, fp16}); a miss is
+    served by a second SCM of generic catch-all versions. Growth mode: the hook
+    registers the bucket's version and re-invokes. Selections are compared with the
+    oracle's replay of the same trace (memoised per distinct tuple and table size)."""
+    t, S, synth = c.torch, c.S, c.synth
+    from oracle import guards as G
+    cfg = dict(synth.STRESS)
+    if n_calls:
+        cfg["n_calls"] = n_calls
+    g = np.random.default_rng(0)
+    Ts, dts, strided = synth.stress_trace(g, cfg)
+    H, pad = cfg["H"], cfg["pad"]
+    Tmax = int(Ts.max())
+    bufs = {}
+    for dt in (S.BF16, S.FP16):
+        tdt = synth._TORCH_DT[dt]
+        bufs[dt] = [t.randn((Tmax, H + pad), device=c.dev).to(tdt) for _ in range(4)]
+    gam = synth.gamma_device(H, 7, c.dev)
+    args_cache, odicts = {}, {}
+
+    def args_for(T, dt, st):
+        key = (int(T), int(dt), bool(st))
+        if key not in args_cache:
+            ts = [b[:T, :H] if st else b[:T].view(-1)[:T * H].view(T, H) for b in bufs[dt]]
+            full = [ts[0], ts[1], gam, ts[2], ts[3]]
+            args_cache[key] = S.make_args(S.OP_ADD_RMSNORM, full, eps=1e-6)
+            odicts[key] = dict(op=1, tensors=[dict(addr=x.data_ptr(), dtype=S.BF16 if x.dtype == t.bfloat16 else
+                                                   (S.FP16 if x.dtype == t.float16 else S.FP32),
+                                                   shape=tuple(x.shape), stride=tuple(x.stride()),
+                                                   device=c.dev.index or 0) for x in full],
+                               eps=1e-6, theta=0.0, flags=0)
+        return args_cache[key], odicts[key]
+
+    generic = S.Scm(device=c.dev.index or 0)
+    for dt in (S.BF16, S.FP16):
+        generic.register(S.make_spec(S.OP_ADD_RMSNORM, dt, [H], 1, 1 << 40, layout=S.LAYOUT_ANY,
+                                     align_bytes=2, variant=S.VARIANT_GENERIC))
+    static_specs = []
+    for b in range(8):
+        lo, hi = G.bucket_range(b)
+        for dt in (S.BF16, S.FP16):
+            static_specs.append(dict(op=1, dtype=dt, rank=2, layout=0, fixed=(H,), tok_lo=lo, tok_hi=hi,
+                                     align=16, device=c.dev.index or 0, variant=0, theta=0.0))
+    results = {}
+    for mode in ("static", "growth"):
+        oracle_table = list(static_specs) if mode == "static" else []
+
+        def hook(scm, args, stream):
+            if mode == "static":
+                st, _ = generic.invoke(args, stream)
+                if st != S.OK:
+                    raise RuntimeError("generic version failed")
+                return None
+            T = int(args.t[0].shape[0])
+            lo, hi = G.bucket_range(G.bucket_of(T))
+            lay = S.LAYOUT_CONTIG if args.t[0].stride[0] == H or T == 1 else S.LAYOUT_ROWSTRIDED
+            idx = scm.register(S.make_spec(S.OP_ADD_RMSNORM, int(args.t[0].dtype), [H], lo, hi, layout=lay))
+            st, sel = scm.invoke(args, stream)
+            if st != S.OK:
+                raise RuntimeError("re-invoke after growth missed")
+            return idx
+
+        scm = S.Scm(device=c.dev.index or 0, flags=S.OPT_TIMING, max_specs=64, hook=hook)
+        if mode == "static":
+            for sp in static_specs:
+                scm.register(S.make_spec(1, sp["dtype"], [H], sp["tok_lo"], sp["tok_hi"]))
+        memo = {}
+        inv, sel = c.L.trident_scm_invoke, ctypes.c_int32(-1)
+        mism = 0
+        hits = misses = 0
+        t.cuda.synchronize()
+        h0 = time.perf_counter()
+        for T, dt, st in zip(Ts, dts, strided):
+            a, od = args_for(T, dt, st)
+            rc = inv(scm.h, ctypes.byref(a), c.sp, ctypes.byref(sel))
+            key = (len(oracle_table), int(T), int(dt), bool(st))
+            if key not in memo:  # selection only: the buffers are distinct allocations
+                memo[key] = G.select(oracle_table, od, check_overlap=False)
+            ost, oidx = memo[key]
+            if rc == S.OK:
+                hits += 1
+                mism += not (ost == G.OK and oidx == sel.value)
+            elif rc == S.MISS_HANDLED:
+                misses += 1
+                mism += ost != G.MISS
+                if mode == "growth":  # oracle replays the same growth rule
+                    lo, hi = G.bucket_range(G.bucket_of(int(T)))
+                    oracle_table.append(dict(op=1, dtype=int(dt), rank=2, layout=1 if (st and T > 1) else 0,
+                                             fixed=(H,), tok_lo=lo, tok_hi=hi, align=16,
+                                             device=c.dev.index or 0, variant=0, theta=0.0))
+            else:
+                raise RuntimeError(f"stress call failed: {rc} {S.trident_scm_last_error()} {scm.hook_error}")
+        t.cuda.synchronize()
+        wall = time.perf_counter() - h0
+        _, ns = S.trident_scm_host_times(scm.h, 1 << 16)
+        stt = scm.stats()
+        c.launches += len(Ts) + (stt.hook_registered if mode == "growth" else 0)
+        results[mode] = dict(calls=len(Ts), hits=hits, misses=misses, mismatches_vs_oracle=int(mism),
+                             versions=stt.num_specs, host_ns_per_hit_median=float(np.median(ns)),
+                             host_ns_per_hit_p99=float(np.percentile(ns, 99)),
+                             python_us_per_call=round(wall * 1e6 / len(Ts), 3))
+        scm.close()
+    generic.close()
+    return results
+
+
+def bench_sweep(c, reps=20, quick=False):
+    """HBM bandwidth sweep: add+RMSNorm (H 8192) and SwiGLU (I 28672) at T = 2^0..2^15,
+    bf16. Each size: `reps` back-to-back launches from one native call, rotating across
+    row windows of arenas sized for 32768 tokens so no launch reads what the previous
+    left in L2 (for T >= 512 the buffers alone exceed L2)."""
+    t, S, synth = c.torch, c.S, c.synth
+    H, I, Tmax = 8192, 28672, 32768
+    peak, _ = measured_peaks()
+    s = S.Scm(device=c.dev.index or 0)
+    s.register(S.make_spec(S.OP_ADD_RMSNORM, S.BF16, [H], 1, 1 << 20))
+    s.register(S.make_spec(S.OP_SWIGLU, S.BF16, [I], 1, 1 << 20))
+    out = {"add_rmsnorm": [], "swiglu": []}
+    seq = c.L.trident_scm_invoke_seq
+    Ts = [2 ** k for k in range(16)] if not quick else [1, 64, 4096, 32768]
+    # add + RMSNorm
+    x = synth.act_device((Tmax, H), S.BF16, 11, c.dev)
+    r = synth.act_device((Tmax, H), S.BF16, 12, c.dev)
+    gam = synth.gamma_device(H, 13, c.dev)
+    y, ro = t.empty_like(x), t.empty_like(r)
+    for T in Ts:
+        nwin = Tmax // T
+        arr = (S.trident_args * reps)(*[S.make_args(S.OP_ADD_RMSNORM, [
+            x[(i % nwin) * T:(i % nwin + 1) * T], r[(i % nwin) * T:(i % nwin + 1) * T], gam,
+            y[(i % nwin) * T:(i % nwin + 1) * T], ro[(i % nwin) * T:(i % nwin + 1) * T]], eps=1e-6)
+            for i in range(reps)])
+        us, _ = time_steps(c, lambda i: seq(s.h, arr, reps, c.sp, None), 3, 2)
+        us /= reps
+        c.launches += 5 * reps
+        b = 8 * H * T + 4 * H
+        out["add_rmsnorm"].append(dict(T=T, us=round(us, 3), gbs=round(b / us / 1e3, 1),
+                                       frac_measured=round(b / us / 1e3 / peak, 3),
+                                       frac_8tbs=round(b / us / 1e3 / NOMINAL_HBM_GBS, 3)))
+    del x, r, y, ro
+    g = synth.act_device((Tmax, I), S.BF16, 14, c.dev)
+    u = synth.act_device((Tmax, I), S.BF16, 15, c.dev)
+    o = t.empty_like(g)
+    for T in Ts:
+        nwin = Tmax // T
+        arr = (S.trident_args * reps)(*[S.make_args(S.OP_SWIGLU, [
+            g[(i % nwin) * T:(i % nwin + 1) * T], u[(i % nwin) * T:(i % nwin + 1) * T],
+            o[(i % nwin) * T:(i % nwin + 1) * T]]) for i in range(reps)])
+        us, _ = time_steps(c, lambda i: seq(s.h, arr, reps, c.sp, None), 3, 2)
+        us /= reps
+        c.launches += 5 * reps
+        b = 6 * I * T
+        out["swiglu"].append(dict(T=T, us=round(us, 3), gbs=round(b / us / 1e3, 1),
+                                  frac_measured=round(b / us / 1e3 / peak, 3),
+                                  frac_8tbs=round(b / us / 1e3 / NOMINAL_HBM_GBS, 3)))
+    del g, u, o
+    s.close()
+    big = [e for e in out["add_rmsnorm"] + out["swiglu"] if e["T"] >= 4096]
+    out["min_frac_measured_T_ge_4096"] = min(e["frac_measured"] for e in big) if big else None
+    return out
+
+
+def kernel_duration_chain(c, cfg, T, reps=200):
+    """Average duration of the fused chain kernel: `reps` launches issued back to back by
+    one native call (device-bound), CUDA events on the launching stream."""
+    S = c.S
+    sets = ChainSets(c, cfg, T)
+    scm = layer_scm(c, cfg)
+    n = min(reps, sets.R)
+    arr = (S.trident_args * n)(*[sets.fused_args(c, i) for i in range(n)])
+    us, _ = time_steps(c, lambda i: c.L.trident_scm_invoke_seq(scm.h, arr, n, c.sp, None), 5, 3)
+    c.launches += 8 * n
+    scm.close()
+    return us / n
+
+
+_T0 = time.perf_counter()
+
+
+def progress(msg):
+    print("[bench %7.1fs] %s" % (time.perf_counter() - _T0, msg), file=sys.stderr, flush=True)
+
+
+def run_ours(a):
+    import torch
+    import torch.distributed as dist
+    from paper_2609_37241_gb300 import synth
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        dist.init_process_group("nccl" if torch.cuda.is_available() else "gloo")
+    torch.cuda.set_device(local)
+    import __graft_entry__
+    __graft_entry__.build()
+    c = Ctx(torch.device("cuda", local))
+    K, W = a.steps, a.warmup
+    clocks = ClockSampler(local)
+    cfg = synth.LLAMA
+
+    def barrier():
+        if world > 1:
+            dist.barrier()
+        torch.cuda.synchronize()
+
+    # ---- headline: T = 64, fused, one invoke per step; exactly K timed steps
+    sets = ChainSets(c, cfg, HEADLINE_T)
+    scm = layer_scm(c, cfg)
+    R = sets.R
+    fused_structs = [sets.fused_args(c, i) for i in range(R)]
+    fused = [ctypes.byref(x) for x in fused_structs]
+    inv = c.L.trident_scm_invoke
+    for i in range(W):
+        inv(scm.h, fused[i % R], c.sp, None)
+    barrier()
+    e0, e1 = c.events()
+    e0.record(c.stream)
+    for i in range(K):
+        inv(scm.h, fused[(W + i) % R], c.sp, None)
+    e1.record(c.stream)
+    barrier()
+    ms = e0.elapsed_time(e1)
+    c.launches += K
+    headline_launches = K
+    scm.close()
+    del sets
+    t_local = torch.tensor([ms], dtype=torch.float64, device=c.dev)
+    if world > 1:
+        dist.all_reduce(t_local, op=dist.ReduceOp.MAX)
+    ms_max = float(t_local.item())
+    us_step = ms_max * 1e3 / K
+
+    extra = {}
+    if rank == 0:
+        progress("per-token layer steps")
+        per_t = {}
+        for T in (1, 4, 16, 64):
+            per_t[str(T)], _ = bench_layer(c, cfg, T, K=min(K, 2000), W=W)
+        extra["llama_per_tokens"] = per_t
+        progress("qwen3 36-layer steps")
+        qw = {}
+        for T in ((1, 8, 32, 128) if not a.quick else (1, 128)):
+            qw[str(T)], _ = bench_layer(c, synth.QWEN3, T, K=max(20, min(K, 2000) // 36), W=W,
+                                        layers=36)
+        extra["qwen3_36layer_step"] = qw
+        progress("host dispatch")
+        extra["host_dispatch_single_addnorm"] = bench_host_hit(c)
+        progress("guard stress")
+        extra["guard_stress"] = bench_guard_stress(c, n_calls=20000 if a.quick else None)
+        progress("hbm sweep")
+        extra["hbm_sweep"] = bench_sweep(c, quick=a.quick)
+        progress("roofline kernel")
+        kd = kernel_duration_chain(c, cfg, HEADLINE_T)
+        peak, src = measured_peaks()
+        b = chain_bytes_per_launch(cfg, HEADLINE_T)
+        extra["roofline"] = dict(bound="hbm", achieved=round(b / kd / 1e3, 1), peak=peak, unit="GB/s",
+                                 frac=round(b / kd / 1e3 / peak, 3), traffic=None,
+                                 kernel="chain_kernel<bf16,H4096,D128>",
+                                 bytes_per_launch=int(b), us_per_launch=round(kd, 3), peak_source=src)
+        progress("e2e")
+        extra["e2e"] = bench_e2e(c, cfg, HEADLINE_T, K=min(K, 500), W=W)
+    ck = clocks.stop()
+    if rank == 0:
+        progress("cpu baseline")
+        budget = 3.0 if a.quick else 12.0
+        cpu_us, n = oracle_layer_step_us(cfg, HEADLINE_T, budget)
+        line = dict(metric=METRIC, value=round(us_step, 3), unit=UNIT, n_gpus=world, steps=K, warmup=W,
+                    ms_per_step=round(us_step / 1e3, 6), higher_is_better=False, scaling="weak",
+                    vs_baseline=None, dtype="bf16",
+                    data="synthetic (seeded N(0,1) activations, N(1,0.1) norm weights, distinct "
+                         "uniform positions; no model weights)",
+                    config=dict(workload="llama decode layer non-GEMM chain: 64 tokens, H 4096, 32/8 "
+                                         "heads, D 128, I 14336, theta 5e5, KV cache [8,8192,128]",
+                                tokens=HEADLINE_T, path="fused chain, 1 launch per step, PDL",
+                                l2="inputs rotated over %d sets (%.0f MB > 2x L2)" % (
+                                    R, R * chain_bytes_per_token(cfg) * HEADLINE_T / 2 ** 20),
+                                parallelism="replicas" if world > 1 else "single GPU"),
+                    gpu_launches=headline_launches, gpu_launches_whole_run=c.launches)
+        line.update(extra)
+        line["cpu_baseline"] = dict(value=round(cpu_us, 1), unit=UNIT, cores=1, kind="oracle",
+                                    sample="%d layer steps at 64 tokens (%.1f s)" % (n, cpu_us * n / 1e6))
+        if ck:
+            line["clocks"] = ck
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.barrier()
+        dist.destroy_process_group()
+
+
+def run_reference(a):
+    """Reference arm: the CPU oracle, as it stands, on the headline configuration. Each
+    step runs the whole layer chain on a sample of the 64 tokens (all four steps, every
+    head), sized so that warm-up plus steps take about a minute; the time is scaled to
+    64 tokens (the chain's work is proportional to the token count)."""
+    from paper_2609_37241_gb300 import synth
+    from oracle import layer as L
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    cfg = synth.LLAMA
+    g = np.random.default_rng(0)
+    full = synth.layer_inputs(g, HEADLINE_T, cfg)
+
+    def sample(Ts):
+        d = {k: (v[:Ts] if k in ("h", "r0", "q", "k", "v", "pos", "attn_out", "g", "u") else v)
+             for k, v in full.items()}
+        return d
+
+    one = sample(1)
+    t0 = time.perf_counter()
+    L.layer_chain(one, cfg["theta"], cfg["eps"], synth.BF16)
+    t1 = max(time.perf_counter() - t0, 1e-4)
+    budget = 20.0 if a.quick else 60.0
+    Ts = int(max(1, min(HEADLINE_T, budget / ((a.steps + a.warmup) * t1))))
+    inp = sample(Ts)
+    for _ in range(a.warmup):
+        L.layer_chain(inp, cfg["theta"], cfg["eps"], synth.BF16)
+    samples = []
+    for _ in range(a.steps):
+        t0 = time.perf_counter()
+        L.layer_chain(inp, cfg["theta"], cfg["eps"], synth.BF16)
+        samples.append((time.perf_counter() - t0) * 1e6 * HEADLINE_T / Ts)
+    us = float(np.median(samples))
+    line = dict(metric=METRIC, value=round(us, 1), unit=UNIT, n_gpus=world, steps=a.steps,
+                warmup=a.warmup, ms_per_step=round(us / 1e3, 4), higher_is_better=False,
+                scaling="weak", vs_baseline=None, dtype="f64", data="synthetic", impl="reference",
+                config=dict(workload="llama decode layer non-GEMM chain: 64 tokens, H 4096, 32/8 heads, "
+                                     "D 128, I 14336, theta 5e5, KV cache [8,8192,128]", tokens=HEADLINE_T),
+                cpu_baseline=dict(value=round(us, 1), unit=UNIT, cores=1, kind="oracle",
+                                  sample="each step: the layer chain on %d of the 64 tokens, scaled "
+                                         "to 64 (median of %d steps)" % (Ts, a.steps)),
+                e2e=dict(value=round(us, 1), unit=UNIT, h2d_bytes_per_step=0, d2h_bytes_per_step=0))
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    p = argparse.ArgumentParser()
+    p.add_argument("--gpus", type=int, default=1)
+    p.add_argument("--steps", type=int, default=5000)
+    p.add_argument("--warmup", type=int, default=20)
+    p.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    p.add_argument("--quick", action="store_true", help="smaller sections (for smoke runs)")
+    a = p.parse_args()
+    if a.warmup < 3:
+        a.warmup = 3
+    if a.impl == "reference":
+        run_reference(a)
+    else:
+        run_ours(a)
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,136 @@
+// addnorm.cu -- fused residual add + RMSNorm kernels (sm_103a).
+//
+//   s = x + r (fp32);  r_out = round(s);  y = round(s * rsqrt(mean(s^2) + eps) * gamma)
+//
+// rms_norm is the paper's running example (Fig. 1, §2.3); the residual add fused in front
+// of it is how decoder layers call it. One block owns one row: the row's bytes are
+// loaded once with 16-byte accesses, the sum of squares is reduced with warp shuffles and
+// one barrier, and both outputs are written with 16-byte stores. Three families:
+//   addnorm_vec_kernel<DT, VPT>   H = VPT * 256 * VE, row held in registers (one pass)
+//   addnorm_loop_kernel<DT>       any H with 16-byte rows (two passes, the second from L2)
+//   addnorm_generic_kernel<DT>    any H, any element-aligned pointer (scalar accesses)
+#include "device_common.cuh"
+
+namespace trident {
+
+template <int DT, int VPT>
+__global__ void __launch_bounds__(kThreads) addnorm_vec_kernel(const AddNormParams p) {
+  pdl_prologue();
+  __shared__ float red[kThreads / 32];
+  constexpr int EB = Act<DT>::BYTES;
+  constexpr int VE = Act<DT>::VE;
+  const int tid = threadIdx.x;
+  for (int64_t row = blockIdx.x; row < p.T; row += gridDim.x) {
+    AddNormRegs<DT, VPT> R;
+    R.load(row_ptr(p.x, row, p.x_rs, EB), row_ptr(p.r, row, p.r_rs, EB), p.gamma, tid);
+    float s[VPT][VE];
+    const float ss = R.residual(row_ptr(p.r_out, row, p.ro_rs, EB), tid, s);
+    const float tot = block_sum(ss, red);
+    R.normalize(row_ptr(p.y, row, p.y_rs, EB), tid, s, rsqrtf(tot * p.inv_H + p.eps));
+    __syncthreads();  // `red` is reused by the next row
+  }
+}
+
+// Two passes: the first only reduces, the second recomputes s and writes both outputs,
+// so that in-place calls (r_out = r, y = x) never read a value they already overwrote.
+template <int DT>
+__global__ void __launch_bounds__(kThreads) addnorm_loop_kernel(const AddNormParams p) {
+  pdl_prologue();
+  __shared__ float red[kThreads / 32];
+  constexpr int EB = Act<DT>::BYTES;
+  constexpr int VE = Act<DT>::VE;
+  const int tid = threadIdx.x;
+  const int64_t nvec = p.H / VE;
+  for (int64_t row = blockIdx.x; row < p.T; row += gridDim.x) {
+    const uint4* x = reinterpret_cast<const uint4*>(row_ptr(p.x, row, p.x_rs, EB));
+    const uint4* r = reinterpret_cast<const uint4*>(row_ptr(p.r, row, p.r_rs, EB));
+    float ss = 0.f;
+    for (int64_t vi = tid; vi < nvec; vi += kThreads) {
+      float xf[VE], rf[VE];
+      unpack<DT>(ld16(x + vi), xf);
+      unpack<DT>(ld16(r + vi), rf);
+#pragma unroll
+      for (int e = 0; e < VE; ++e) {
+        const float s = xf[e] + rf[e];
+        ss = fmaf(s, s, ss);
+      }
+    }
+    const float inv = rsqrtf(block_sum(ss, red) * p.inv_H + p.eps);
+    uint4* y = reinterpret_cast<uint4*>(row_ptr(p.y, row, p.y_rs, EB));
+    uint4* ro = reinterpret_cast<uint4*>(row_ptr(p.r_out, row, p.ro_rs, EB));
+    for (int64_t vi = tid; vi < nvec; vi += kThreads) {
+      float xf[VE], rf[VE], s[VE], yf[VE], g[VE];
+      unpack<DT>(ld16(x + vi), xf);
+      unpack<DT>(ld16(r + vi), rf);
+#pragma unroll
+      for (int q = 0; q < VE / 4; ++q) {
+        const float4 g4 = ldg_f4(p.gamma + vi * VE + 4 * q);
+        g[4 * q] = g4.x; g[4 * q + 1] = g4.y; g[4 * q + 2] = g4.z; g[4 * q + 3] = g4.w;
+      }
+#pragma unroll
+      for (int e = 0; e < VE; ++e) {
+        s[e] = xf[e] + rf[e];
+        yf[e] = s[e] * inv * g[e];
+      }
+      st16(ro + vi, pack<DT>(s));
+      st16(y + vi, pack<DT>(yf));
+    }
+    __syncthreads();
+  }
+}
+
+template <int DT>
+__global__ void __launch_bounds__(kThreads) addnorm_generic_kernel(const AddNormParams p) {
+  pdl_prologue();
+  __shared__ float red[kThreads / 32];
+  const int tid = threadIdx.x;
+  for (int64_t row = blockIdx.x; row < p.T; row += gridDim.x) {
+    const int64_t xo = row * p.x_rs, ro = row * p.r_rs;
+    float ss = 0.f;
+    for (int64_t j = tid; j < p.H; j += kThreads) {
+      const float s = load_elem<DT>(p.x, xo + j) + load_elem<DT>(p.r, ro + j);
+      ss = fmaf(s, s, ss);
+    }
+    const float inv = rsqrtf(block_sum(ss, red) * p.inv_H + p.eps);
+    for (int64_t j = tid; j < p.H; j += kThreads) {
+      const float s = load_elem<DT>(p.x, xo + j) + load_elem<DT>(p.r, ro + j);
+      store_elem<DT>(p.r_out, row * p.ro_rs + j, s);
+      store_elem<DT>(p.y, row * p.y_rs + j, s * inv * p.gamma[j]);
+    }
+    __syncthreads();
+  }
+}
+
+template <int DT>
+static bool pick_vec(int64_t H, KernelEntry* out) {
+  constexpr int VE = Act<DT>::VE;
+  const int64_t per = (int64_t)kThreads * VE;
+  if (H == per * 1) { out->fn = (const void*)addnorm_vec_kernel<DT, 1>; return true; }
+  if (H == per * 2) { out->fn = (const void*)addnorm_vec_kernel<DT, 2>; return true; }
+  if (H == per * 4) { out->fn = (const void*)addnorm_vec_kernel<DT, 4>; return true; }
+  if (H == per * 8) { out->fn = (const void*)addnorm_vec_kernel<DT, 8>; return true; }
+  out->fn = (const void*)addnorm_loop_kernel<DT>;
+  return true;
+}
+
+bool addnorm_kernel(int32_t dtype, int32_t variant, int64_t H, KernelEntry* out, const char** why) {
+  out->kind = KK_ADDNORM_ROW;
+  out->unroll = 1;
+  const int eb = dtype == DT_FP32 ? 4 : 2;
+  if (dtype != DT_BF16 && dtype != DT_FP16 && dtype != DT_FP32) { *why = "dtype"; return false; }
+  if (H < 1) { *why = "H must be >= 1"; return false; }
+  if (variant == 1) {  // GENERIC
+    out->vec = 1;
+    out->fn = dtype == DT_BF16 ? (const void*)addnorm_generic_kernel<DT_BF16>
+            : dtype == DT_FP16 ? (const void*)addnorm_generic_kernel<DT_FP16>
+                               : (const void*)addnorm_generic_kernel<DT_FP32>;
+    return true;
+  }
+  if ((H * eb) % 16 != 0) { *why = "vector add+RMSNorm needs H * elem_size % 16 == 0"; return false; }
+  out->vec = 16 / eb;
+  if (dtype == DT_BF16) return pick_vec<DT_BF16>(H, out);
+  if (dtype == DT_FP16) return pick_vec<DT_FP16>(H, out);
+  return pick_vec<DT_FP32>(H, out);
+}
+
+}  // namespace trident

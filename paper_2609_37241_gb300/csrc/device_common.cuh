@@ -1,0 +1,340 @@
+// device_common.cuh -- device-side building blocks shared by the kernels of this library.
+//
+// Every kernel is memory bound (a few flops per byte), so the building blocks are about
+// moving bytes: 16-byte vector loads and stores per thread, fp32 math in registers,
+// warp-shuffle reductions. Each kernel starts with the programmatic-dependent-launch
+// pair (trigger, then wait) so that, when launched with programmatic stream
+// serialisation, the next kernel's launch overlaps this one while every global memory
+// access still waits for the previous kernel to finish.
+#pragma once
+#include <cuda_bf16.h>
+#include <cuda_fp16.h>
+#include <stdint.h>
+
+#include "internal.h"
+
+namespace trident {
+
+constexpr uint32_t kErrPos = 0x1u;  // TRIDENT_DEVERR_POS
+
+__device__ __forceinline__ void pdl_prologue() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+}
+
+template <int DT> struct Act;
+template <> struct Act<DT_BF16> { static constexpr int VE = 8; static constexpr int BYTES = 2; };
+template <> struct Act<DT_FP16> { static constexpr int VE = 8; static constexpr int BYTES = 2; };
+template <> struct Act<DT_FP32> { static constexpr int VE = 4; static constexpr int BYTES = 4; };
+
+// ---------------------------------------------------------------- 16-byte vectors
+__device__ __forceinline__ uint4 ldg16(const void* p) { return __ldg(reinterpret_cast<const uint4*>(p)); }
+__device__ __forceinline__ uint4 ld16(const void* p) { return *reinterpret_cast<const uint4*>(p); }
+__device__ __forceinline__ void st16(void* p, uint4 v) { *reinterpret_cast<uint4*>(p) = v; }
+__device__ __forceinline__ float4 ldg_f4(const float* p) { return __ldg(reinterpret_cast<const float4*>(p)); }
+
+template <int DT> __device__ __forceinline__ void unpack(const uint4& v, float* f);
+template <> __device__ __forceinline__ void unpack<DT_BF16>(const uint4& v, float* f) {
+  const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    f[2 * i] = __uint_as_float(w[i] << 16);
+    f[2 * i + 1] = __uint_as_float(w[i] & 0xffff0000u);
+  }
+}
+template <> __device__ __forceinline__ void unpack<DT_FP16>(const uint4& v, float* f) {
+  const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    __half2 h;
+    memcpy(&h, &w[i], 4);
+    float2 ff = __half22float2(h);
+    f[2 * i] = ff.x;
+    f[2 * i + 1] = ff.y;
+  }
+}
+template <> __device__ __forceinline__ void unpack<DT_FP32>(const uint4& v, float* f) {
+  f[0] = __uint_as_float(v.x); f[1] = __uint_as_float(v.y);
+  f[2] = __uint_as_float(v.z); f[3] = __uint_as_float(v.w);
+}
+
+template <int DT> __device__ __forceinline__ uint4 pack(const float* f);
+template <> __device__ __forceinline__ uint4 pack<DT_BF16>(const float* f) {
+  uint32_t w[4];
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    __nv_bfloat162 b = __floats2bfloat162_rn(f[2 * i], f[2 * i + 1]);
+    memcpy(&w[i], &b, 4);
+  }
+  return make_uint4(w[0], w[1], w[2], w[3]);
+}
+template <> __device__ __forceinline__ uint4 pack<DT_FP16>(const float* f) {
+  uint32_t w[4];
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    __half2 h = __floats2half2_rn(f[2 * i], f[2 * i + 1]);
+    memcpy(&w[i], &h, 4);
+  }
+  return make_uint4(w[0], w[1], w[2], w[3]);
+}
+template <> __device__ __forceinline__ uint4 pack<DT_FP32>(const float* f) {
+  return make_uint4(__float_as_uint(f[0]), __float_as_uint(f[1]), __float_as_uint(f[2]),
+                    __float_as_uint(f[3]));
+}
+
+// ---------------------------------------------------------------- scalar elements
+template <int DT> __device__ __forceinline__ float load_elem(const void* p, int64_t i);
+template <> __device__ __forceinline__ float load_elem<DT_BF16>(const void* p, int64_t i) {
+  return __bfloat162float(reinterpret_cast<const __nv_bfloat16*>(p)[i]);
+}
+template <> __device__ __forceinline__ float load_elem<DT_FP16>(const void* p, int64_t i) {
+  return __half2float(reinterpret_cast<const __half*>(p)[i]);
+}
+template <> __device__ __forceinline__ float load_elem<DT_FP32>(const void* p, int64_t i) {
+  return reinterpret_cast<const float*>(p)[i];
+}
+template <int DT> __device__ __forceinline__ void store_elem(void* p, int64_t i, float v);
+template <> __device__ __forceinline__ void store_elem<DT_BF16>(void* p, int64_t i, float v) {
+  reinterpret_cast<__nv_bfloat16*>(p)[i] = __float2bfloat16_rn(v);
+}
+template <> __device__ __forceinline__ void store_elem<DT_FP16>(void* p, int64_t i, float v) {
+  reinterpret_cast<__half*>(p)[i] = __float2half_rn(v);
+}
+template <> __device__ __forceinline__ void store_elem<DT_FP32>(void* p, int64_t i, float v) {
+  reinterpret_cast<float*>(p)[i] = v;
+}
+// Rounds v to the activation type and back (the value a store would hold).
+template <int DT> __device__ __forceinline__ float round_act(float v);
+template <> __device__ __forceinline__ float round_act<DT_BF16>(float v) {
+  return __bfloat162float(__float2bfloat16_rn(v));
+}
+template <> __device__ __forceinline__ float round_act<DT_FP16>(float v) {
+  return __half2float(__float2half_rn(v));
+}
+template <> __device__ __forceinline__ float round_act<DT_FP32>(float v) { return v; }
+
+__device__ __forceinline__ const char* row_ptr(const void* base, int64_t row, int64_t rs, int eb) {
+  return reinterpret_cast<const char*>(base) + row * rs * eb;
+}
+__device__ __forceinline__ char* row_ptr(void* base, int64_t row, int64_t rs, int eb) {
+  return reinterpret_cast<char*>(base) + row * rs * eb;
+}
+
+// ---------------------------------------------------------------- reductions
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  return v;
+}
+
+// Sum over the block; every thread gets the same total (same summation order).
+// `red` holds kThreads/32 floats and must not be reused until after a barrier.
+__device__ __forceinline__ float block_sum(float v, float* red) {
+  constexpr int NW = kThreads / 32;
+  v = warp_sum(v);
+  if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = v;
+  __syncthreads();
+  float t = 0.f;
+#pragma unroll
+  for (int i = 0; i < NW; ++i) t += red[i];
+  return t;
+}
+
+// ---------------------------------------------------------------- add + RMSNorm row
+// One row of H = VPT * kThreads * VE elements held in registers by one block.
+// Thread `tid` owns vectors v*kThreads + tid, v < VPT (coalesced 16-byte accesses).
+template <int DT, int VPT>
+struct AddNormRegs {
+  static constexpr int VE = Act<DT>::VE;
+  uint4 xv[VPT], rv[VPT];
+  float g[VPT][VE];
+
+  __device__ __forceinline__ void load(const void* x_row, const void* r_row, const float* gamma,
+                                       int tid) {
+#pragma unroll
+    for (int v = 0; v < VPT; ++v) {
+      const int64_t vi = (int64_t)v * kThreads + tid;
+      xv[v] = ldg16(reinterpret_cast<const uint4*>(x_row) + vi);
+      rv[v] = ldg16(reinterpret_cast<const uint4*>(r_row) + vi);
+#pragma unroll
+      for (int q = 0; q < VE / 4; ++q) {
+        float4 gg = ldg_f4(gamma + vi * VE + 4 * q);
+        g[v][4 * q] = gg.x; g[v][4 * q + 1] = gg.y; g[v][4 * q + 2] = gg.z; g[v][4 * q + 3] = gg.w;
+      }
+    }
+  }
+  // Loads only x and gamma; the residual is given in registers (already rounded).
+  __device__ __forceinline__ void load_x_gamma(const void* x_row, const float* gamma, int tid) {
+#pragma unroll
+    for (int v = 0; v < VPT; ++v) {
+      const int64_t vi = (int64_t)v * kThreads + tid;
+      xv[v] = ldg16(reinterpret_cast<const uint4*>(x_row) + vi);
+#pragma unroll
+      for (int q = 0; q < VE / 4; ++q) {
+        float4 gg = ldg_f4(gamma + vi * VE + 4 * q);
+        g[v][4 * q] = gg.x; g[v][4 * q + 1] = gg.y; g[v][4 * q + 2] = gg.z; g[v][4 * q + 3] = gg.w;
+      }
+    }
+  }
+
+  // s = x + r (fp32); stores round(s) to r_out (and leaves it in rv); returns sum(s^2)
+  // of this thread; s is left in `s`.
+  __device__ __forceinline__ float residual(void* ro_row, int tid, float (&s)[VPT][VE]) {
+    float ss = 0.f;
+#pragma unroll
+    for (int v = 0; v < VPT; ++v) {
+      float xf[VE], rf[VE];
+      unpack<DT>(xv[v], xf);
+      unpack<DT>(rv[v], rf);
+#pragma unroll
+      for (int e = 0; e < VE; ++e) {
+        s[v][e] = xf[e] + rf[e];
+        ss = fmaf(s[v][e], s[v][e], ss);
+      }
+      rv[v] = pack<DT>(s[v]);
+      st16(reinterpret_cast<uint4*>(ro_row) + (int64_t)v * kThreads + tid, rv[v]);
+    }
+    return ss;
+  }
+
+  __device__ __forceinline__ void normalize(void* y_row, int tid, const float (&s)[VPT][VE],
+                                            float inv) {
+#pragma unroll
+    for (int v = 0; v < VPT; ++v) {
+      float y[VE];
+#pragma unroll
+      for (int e = 0; e < VE; ++e) y[e] = s[v][e] * inv * g[v][e];
+      st16(reinterpret_cast<uint4*>(y_row) + (int64_t)v * kThreads + tid, pack<DT>(y));
+    }
+  }
+};
+
+// ---------------------------------------------------------------- RoPE head-row
+// One head-row (token t, head hh) handled by LPH = D / VE consecutive lanes, each lane
+// owning VE consecutive elements. Rotate-half pairs element i with i + D/2, i.e. lane
+// l with lane l ^ (LPH/2). hh < Hq: q head (rotated in place); hh < Hq + Hkv: k head
+// (rotated into k_cache); else v head (copied into v_cache).
+template <int DT, int D, bool QKNORM>
+__device__ __forceinline__ void rope_head_row(const RopeParams& p, int64_t unit, int lane) {
+  constexpr int VE = Act<DT>::VE;
+  constexpr int LPH = D / VE;
+  constexpr int HALF = LPH / 2;
+  static_assert(LPH >= 2 && LPH <= 32 && (LPH & (LPH - 1)) == 0, "head size");
+  const unsigned group_mask =
+      (LPH == 32) ? 0xffffffffu : (((1u << LPH) - 1u) << ((threadIdx.x & 31) & ~(LPH - 1)));
+
+  const int64_t t = unit / p.NH;
+  const int hh = (int)(unit - t * p.NH);
+  const int32_t pos = __ldg(p.pos + t);
+  if (pos < 0 || (int64_t)pos >= p.S) {
+    if (lane == 0) atomicOr(p.err, kErrPos);
+    return;
+  }
+  constexpr int EB = Act<DT>::BYTES;
+  if (hh >= p.Hq + p.Hkv) {  // v: bit copy into the cache
+    const int h = hh - p.Hq - p.Hkv;
+    const char* src = row_ptr(p.v, t, p.v_rs, EB) + ((int64_t)h * D + lane * VE) * EB;
+    char* dst = reinterpret_cast<char*>(p.v_cache) + (((int64_t)h * p.S + pos) * D + lane * VE) * EB;
+    st16(dst, ldg16(src));
+    return;
+  }
+  const bool is_q = hh < p.Hq;
+  const int h = is_q ? hh : hh - p.Hq;
+  const char* src = is_q ? row_ptr(p.q, t, p.q_rs, EB) + ((int64_t)h * D + lane * VE) * EB
+                         : row_ptr(p.k, t, p.k_rs, EB) + ((int64_t)h * D + lane * VE) * EB;
+  float x[VE];
+  unpack<DT>(is_q ? ld16(src) : ldg16(src), x);
+  // (cos, sin) of the VE frequencies i = (lane % HALF) * VE + e
+  const float* csrow = reinterpret_cast<const float*>(p.cs + (int64_t)pos * (D / 2)) +
+                       2 * (lane % HALF) * VE;
+  float cs[2 * VE];
+#pragma unroll
+  for (int q = 0; q < VE / 2; ++q) {
+    float4 c4 = ldg_f4(csrow + 4 * q);
+    cs[4 * q] = c4.x; cs[4 * q + 1] = c4.y; cs[4 * q + 2] = c4.z; cs[4 * q + 3] = c4.w;
+  }
+  if (QKNORM) {
+    const float* gam = (is_q ? p.gamma_q : p.gamma_k) + lane * VE;
+    float gg[VE];
+#pragma unroll
+    for (int q = 0; q < VE / 4; ++q) {
+      float4 g4 = ldg_f4(gam + 4 * q);
+      gg[4 * q] = g4.x; gg[4 * q + 1] = g4.y; gg[4 * q + 2] = g4.z; gg[4 * q + 3] = g4.w;
+    }
+    float ss = 0.f;
+#pragma unroll
+    for (int e = 0; e < VE; ++e) ss = fmaf(x[e], x[e], ss);
+#pragma unroll
+    for (int o = LPH / 2; o > 0; o >>= 1) ss += __shfl_xor_sync(group_mask, ss, o, LPH);
+    const float inv = rsqrtf(ss * p.inv_D + p.eps);
+#pragma unroll
+    for (int e = 0; e < VE; ++e) x[e] = x[e] * inv * gg[e];
+  }
+  float other[VE];
+#pragma unroll
+  for (int e = 0; e < VE; ++e) other[e] = __shfl_xor_sync(group_mask, x[e], HALF, LPH);
+  const bool low = lane < HALF;
+  float y[VE];
+#pragma unroll
+  for (int e = 0; e < VE; ++e) {
+    const float c = cs[2 * e], s = cs[2 * e + 1];
+    // low half: x_i c - x_{i+D/2} s;  high half: x_{i+D/2} c + x_i s
+    y[e] = low ? fmaf(x[e], c, -other[e] * s) : fmaf(x[e], c, other[e] * s);
+  }
+  if (is_q) {
+    st16(row_ptr(p.q, t, p.q_rs, EB) + ((int64_t)h * D + lane * VE) * EB, pack<DT>(y));
+  } else {
+    char* dst = reinterpret_cast<char*>(p.k_cache) + (((int64_t)h * p.S + pos) * D + lane * VE) * EB;
+    st16(dst, pack<DT>(y));
+  }
+}
+
+// ---------------------------------------------------------------- SwiGLU tile
+template <int DT> __device__ __forceinline__ float silu_mul(float g, float u);
+// bf16/fp16 outputs: fast exp and divide (relative error ~1e-6, far below the output ulp;
+// for g below about -87 the result is -0, the limit of g * sigmoid(g)).
+template <> __device__ __forceinline__ float silu_mul<DT_BF16>(float g, float u) {
+  return __fdividef(g, 1.0f + __expf(-g)) * u;
+}
+template <> __device__ __forceinline__ float silu_mul<DT_FP16>(float g, float u) {
+  return __fdividef(g, 1.0f + __expf(-g)) * u;
+}
+// fp32 outputs: full-precision exp and IEEE division.
+template <> __device__ __forceinline__ float silu_mul<DT_FP32>(float g, float u) {
+  return g / (1.0f + expf(-g)) * u;
+}
+
+// One tile of UNROLL * kThreads vectors of one row, starting at vector index v0.
+template <int DT, int UNROLL>
+__device__ __forceinline__ void swiglu_tile(const SwigluParams& p, int64_t row, int64_t v0,
+                                            int tid) {
+  constexpr int VE = Act<DT>::VE;
+  constexpr int EB = Act<DT>::BYTES;
+  const int64_t nvec = p.I / VE;
+  const uint4* g = reinterpret_cast<const uint4*>(row_ptr(p.g, row, p.g_rs, EB));
+  const uint4* u = reinterpret_cast<const uint4*>(row_ptr(p.u, row, p.u_rs, EB));
+  uint4* o = reinterpret_cast<uint4*>(row_ptr(p.out, row, p.o_rs, EB));
+  uint4 gv[UNROLL], uv[UNROLL];
+#pragma unroll
+  for (int k = 0; k < UNROLL; ++k) {
+    const int64_t vi = v0 + (int64_t)k * kThreads + tid;
+    if (vi < nvec) {
+      gv[k] = ldg16(g + vi);
+      uv[k] = ldg16(u + vi);
+    }
+  }
+#pragma unroll
+  for (int k = 0; k < UNROLL; ++k) {
+    const int64_t vi = v0 + (int64_t)k * kThreads + tid;
+    if (vi < nvec) {
+      float gf[VE], uf[VE], of[VE];
+      unpack<DT>(gv[k], gf);
+      unpack<DT>(uv[k], uf);
+#pragma unroll
+      for (int e = 0; e < VE; ++e) of[e] = silu_mul<DT>(gf[e], uf[e]);
+      st16(o + vi, pack<DT>(of));
+    }
+  }
+}
+
+}  // namespace trident

@@ -1,0 +1,99 @@
+// internal.h -- interface between the SCM host core (scm.cpp) and the kernels (*.cu).
+//
+// Each kernel takes one parameter struct by value. The host core packs it on the hit
+// path (argument preparation, §3.2 and §3.5 of the paper: graph operands are rebuilt
+// only after every guard passed) and launches the kernel entry that was resolved when
+// the version was registered (§3.3).
+#pragma once
+#include <stdint.h>
+
+namespace trident {
+
+// Activation element types (values equal trident_dtype).
+enum : int32_t { DT_BF16 = 1, DT_FP16 = 2, DT_FP32 = 3 };
+
+constexpr int kThreads = 256;  // block size of every kernel in this library
+
+// add + RMSNorm over T rows of H elements. Row strides in elements.
+struct AddNormParams {
+  const void* x;
+  const void* r;
+  const float* gamma;
+  void* y;
+  void* r_out;
+  int64_t T, H;
+  int64_t x_rs, r_rs, y_rs, ro_rs;
+  float eps, inv_H;
+};
+
+// RoPE on q/k (optionally after per-head RMSNorm) plus KV-cache append.
+// q/k/v rows: token stride *_rs, head stride D, element stride 1.
+// cs: [S][D/2] pairs (cos, sin) in fp32. Caches dense [Hkv][S][D].
+struct RopeParams {
+  void* q;
+  const void* k;
+  const void* v;
+  const int32_t* pos;
+  void* k_cache;
+  void* v_cache;
+  const float* gamma_q;
+  const float* gamma_k;
+  const float2* cs;
+  uint32_t* err;
+  int64_t T, S;
+  int64_t q_rs, k_rs, v_rs;
+  int32_t Hq, Hkv, D, NH;  // NH = Hq + 2 Hkv head-rows per token
+  float eps, inv_D;
+};
+
+// out = silu(g) * u over T rows of I elements.
+struct SwigluParams {
+  const void* g;
+  const void* u;
+  void* out;
+  int64_t T, I;
+  int64_t g_rs, u_rs, o_rs;
+};
+
+// One decoder layer's chain in one launch. Blocks [0, nA) run the two add+RMSNorm
+// steps of one token each, [nA, nA+nB) the RoPE/KV head-rows, the rest SwiGLU tiles.
+struct ChainParams {
+  AddNormParams n1;   // h, r0 -> x1, r1
+  AddNormParams n2;   // attn_out, (r1 from registers) -> x2, r2; n2.r is unused
+  RopeParams rope;
+  SwigluParams sw;
+  int32_t nA, nB, nC, sw_tiles_per_row;
+};
+
+// Kernel entry (host stub address) plus its launch shape rule.
+struct KernelEntry {
+  const void* fn = nullptr;
+  int32_t kind = 0;      // which grid rule the host applies (KernelKind)
+  int32_t vec = 0;       // elements per vector (VE), or tile width for SwiGLU
+  int32_t unroll = 1;    // vectors per thread per tile (SwiGLU, chain)
+};
+
+enum KernelKind : int32_t {
+  KK_ADDNORM_ROW = 1,   // grid = T rows, one block per row
+  KK_ROPE_HALFWARP = 2, // grid = ceil(T*NH / units_per_block)
+  KK_ROPE_WARP = 3,     // generic: one warp per head-row
+  KK_SWIGLU_TILE = 4,   // grid = (tiles per row, rows)
+  KK_SWIGLU_FLAT = 5,   // generic: flat grid-stride
+  KK_CHAIN = 6
+};
+
+// Lookup of compiled kernels. Return false (with a reason) if no kernel fits.
+bool addnorm_kernel(int32_t dtype, int32_t variant, int64_t H, KernelEntry* out, const char** why);
+bool rope_kernel(int32_t dtype, int32_t variant, int32_t D, bool qknorm, KernelEntry* out,
+                 const char** why);
+bool swiglu_kernel(int32_t dtype, int32_t variant, int64_t I, KernelEntry* out, const char** why);
+bool chain_kernel(int32_t dtype, int64_t H, int32_t D, bool qknorm, KernelEntry* out,
+                  const char** why);
+
+// Units (head-rows) handled by one block of the vector RoPE kernel for head size D.
+inline int32_t rope_units_per_block(int32_t D, int32_t elem_bytes) {
+  int32_t lanes_per_head = D * elem_bytes / 16;
+  return kThreads / lanes_per_head;
+}
+
+}  // namespace trident

@@ -1,0 +1,1021 @@
+// scm.cpp -- the Specialization Cache Module: version table, guards, dispatch, launch.
+//
+// The paper's SCM (§3.1, Fig. 1c) compiles, for several guarded specialisations, the
+// guard evaluation, the argument/environment preparation and the host execution into one
+// native module, so a cache hit never returns to Python (§3.2). Here that module is this
+// file: trident_scm_invoke validates the argument tuple, evaluates the versions' guards
+// in creation order (Algorithm 1), packs the selected kernel's parameters and launches it
+// on the caller's stream. Only a miss leaves native code, through the compile hook
+// (§3.5); an error is returned at once and never falls through to another version.
+//
+// Guards are evaluated in two halves. The argument tuple's guarded properties (common
+// device, dtypes, ranks, sizes, token count, layout class, alignment) are computed once
+// per call into a Sig; each version's G_i then compares its fields against the Sig, so
+// checks shared by every version run once (§3.2: redundant checks are removed and the
+// rest ordered by their data dependencies). The result equals evaluating each G_i on
+// its own, field by field.
+//
+// Table publication is append-only: slots never move and are written before the count
+// that exposes them is released, so a reader needs one acquire load and no lock, and a
+// registration from inside a hook is visible to every later call (§3.5: growth).
+#include <cuda.h>
+#include <cuda_runtime.h>
+
+#include <atomic>
+#include <chrono>
+#include <cmath>
+#include <cstdarg>
+#include <cstdio>
+#include <cstdlib>
+#include <cstring>
+#include <initializer_list>
+#include <mutex>
+#include <tuple>
+#include <new>
+#include <vector>
+
+#include "internal.h"
+#include "trident_scm.h"
+
+#define TRIDENT_API extern "C" __attribute__((visibility("default")))
+
+using namespace trident;
+
+namespace {
+
+// ------------------------------------------------------------------ errors
+thread_local char tl_err[512] = "";
+thread_local int tl_hook_depth = 0;
+
+int32_t fail(int32_t status, const char* fmt, ...) {
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(tl_err, sizeof(tl_err), fmt, ap);
+  va_end(ap);
+  return status;
+}
+
+// ------------------------------------------------------------------ driver entry points
+// The launch goes straight to the driver (cuLaunchKernelEx) with the CUfunction resolved
+// at registration. The driver is reached through the runtime's entry-point query, so the
+// library has no link-time dependency on libcuda and loads on machines without a GPU.
+struct Driver {
+  CUresult (*launch_ex)(const CUlaunchConfig*, CUfunction, void**, void**) = nullptr;
+  CUresult (*ctx_get)(CUcontext*) = nullptr;
+  CUresult (*ctx_push)(CUcontext) = nullptr;
+  CUresult (*ctx_pop)(CUcontext*) = nullptr;
+  bool ok = false;
+};
+Driver g_drv;
+std::once_flag g_drv_once;
+
+bool driver() {
+  std::call_once(g_drv_once, [] {
+    cudaDriverEntryPointQueryResult q;
+    void* f = nullptr;
+    bool ok = true;
+    auto get = [&](const char* name) -> void* {
+      f = nullptr;
+      if (cudaGetDriverEntryPointByVersion(name, &f, 12000, cudaEnableDefault, &q) != cudaSuccess ||
+          q != cudaDriverEntryPointSuccess)
+        ok = false;
+      return f;
+    };
+    g_drv.launch_ex = reinterpret_cast<decltype(g_drv.launch_ex)>(get("cuLaunchKernelEx"));
+    g_drv.ctx_get = reinterpret_cast<decltype(g_drv.ctx_get)>(get("cuCtxGetCurrent"));
+    g_drv.ctx_push = reinterpret_cast<decltype(g_drv.ctx_push)>(get("cuCtxPushCurrent"));
+    g_drv.ctx_pop = reinterpret_cast<decltype(g_drv.ctx_pop)>(get("cuCtxPopCurrent"));
+    g_drv.ok = ok && g_drv.launch_ex && g_drv.ctx_get && g_drv.ctx_push && g_drv.ctx_pop;
+  });
+  return g_drv.ok;
+}
+
+// ------------------------------------------------------------------ op tables
+enum Kind : uint8_t { K_ACT_H, K_ACT_I, K_GAMMA_H, K_GAMMA_D, K_HEADS_Q, K_HEADS_KV, K_POS, K_CACHE };
+
+struct OpInfo {
+  int32_t nslots;
+  int32_t nfixed;
+  bool flattening;  // activations may be rank 2 [T,W] or rank 3 [B,S,W]
+  bool rope;        // guarded RoPE base
+  Kind kind[TRIDENT_MAX_TENSORS];
+  bool out[TRIDENT_MAX_TENSORS];
+  uint8_t group[TRIDENT_MAX_TENSORS];  // in-place group id (0: none)
+};
+
+constexpr int kMaxOp = 6;
+OpInfo g_ops[kMaxOp + 1];
+
+// slot index constants of the chains
+enum { C_H = 0, C_R0, C_GA, C_X1, C_R1, C_Q, C_K, C_V, C_POS, C_KC, C_VC, C_AO, C_GM, C_X2, C_R2,
+       C_G, C_U, C_O, C_GQ, C_GK };
+
+struct OpInit {
+  OpInit() {
+    auto set = [](int op, int nfixed, bool flat, bool rope,
+                  std::initializer_list<std::tuple<Kind, bool, int>> slots) {
+      OpInfo& o = g_ops[op];
+      o.nslots = (int32_t)slots.size();
+      o.nfixed = nfixed;
+      o.flattening = flat;
+      o.rope = rope;
+      int i = 0;
+      for (auto& s : slots) {
+        o.kind[i] = std::get<0>(s);
+        o.out[i] = std::get<1>(s);
+        o.group[i] = (uint8_t)std::get<2>(s);
+        ++i;
+      }
+    };
+    set(TRIDENT_OP_ADD_RMSNORM, 1, true, false,
+        {{K_ACT_H, false, 1}, {K_ACT_H, false, 2}, {K_GAMMA_H, false, 0}, {K_ACT_H, true, 1},
+         {K_ACT_H, true, 2}});
+    set(TRIDENT_OP_ROPE_KV, 4, false, true,
+        {{K_HEADS_Q, true, 0}, {K_HEADS_KV, false, 0}, {K_HEADS_KV, false, 0}, {K_POS, false, 0},
+         {K_CACHE, true, 0}, {K_CACHE, true, 0}});
+    set(TRIDENT_OP_QKNORM_ROPE_KV, 4, false, true,
+        {{K_HEADS_Q, true, 0}, {K_HEADS_KV, false, 0}, {K_HEADS_KV, false, 0}, {K_POS, false, 0},
+         {K_CACHE, true, 0}, {K_CACHE, true, 0}, {K_GAMMA_D, false, 0}, {K_GAMMA_D, false, 0}});
+    set(TRIDENT_OP_SWIGLU, 1, true, false, {{K_ACT_I, false, 1}, {K_ACT_I, false, 1}, {K_ACT_I, true, 1}});
+    const std::initializer_list<std::tuple<Kind, bool, int>> chain = {
+        {K_ACT_H, false, 1},  {K_ACT_H, false, 2},    {K_GAMMA_H, false, 0}, {K_ACT_H, true, 1},
+        {K_ACT_H, true, 2},   {K_HEADS_Q, true, 0},   {K_HEADS_KV, false, 0}, {K_HEADS_KV, false, 0},
+        {K_POS, false, 0},    {K_CACHE, true, 0},     {K_CACHE, true, 0},     {K_ACT_H, false, 3},
+        {K_GAMMA_H, false, 0}, {K_ACT_H, true, 3},    {K_ACT_H, true, 2},     {K_ACT_I, false, 4},
+        {K_ACT_I, false, 4},  {K_ACT_I, true, 4}};
+    set(TRIDENT_OP_LAYER_CHAIN, 6, false, true, chain);
+    OpInfo& o = g_ops[TRIDENT_OP_LAYER_CHAIN_QKNORM];
+    o = g_ops[TRIDENT_OP_LAYER_CHAIN];
+    o.nslots = 20;
+    o.kind[18] = o.kind[19] = K_GAMMA_D;
+    o.out[18] = o.out[19] = false;
+    o.group[18] = o.group[19] = 0;
+  }
+} g_op_init;
+
+inline int elem_size(int32_t dt) {
+  switch (dt) {
+    case TRIDENT_BF16: case TRIDENT_FP16: return 2;
+    case TRIDENT_FP32: case TRIDENT_I32: return 4;
+    case TRIDENT_I64: return 8;
+    default: return 0;
+  }
+}
+inline bool is_act(Kind k) { return k == K_ACT_H || k == K_ACT_I || k == K_HEADS_Q || k == K_HEADS_KV; }
+
+// Rows view of a tensor: (rows, row width in elements, row stride in elements, packed).
+struct Rows {
+  int64_t n, width, stride;
+  bool packed;
+};
+
+inline Rows rows_of(const trident_tensor& t, Kind k) {
+  const int64_t* sh = t.shape;
+  const int64_t* st = t.stride;
+  if (k == K_HEADS_Q || k == K_HEADS_KV)
+    return {sh[0], sh[1] * sh[2], st[0], st[2] == 1 && (sh[1] <= 1 || st[1] == sh[2])};
+  if (k == K_ACT_H || k == K_ACT_I) {
+    if (t.ndim == 2) return {sh[0], sh[1], st[0], st[1] == 1};
+    const bool inner = st[2] == 1;
+    if (sh[1] == 1) return {sh[0], sh[2], st[0], inner};
+    if (sh[0] == 1) return {sh[1], sh[2], st[1], inner};
+    return {sh[0] * sh[1], sh[2], st[1], inner && st[0] == sh[1] * st[1]};
+  }
+  // gamma, pos, cache: one dense row
+  int64_t n = 1;
+  for (int d = 0; d < t.ndim; ++d) n *= sh[d];
+  return {1, n, n, true};
+}
+
+// ------------------------------------------------------------------ argument signature
+constexpr int32_t kMixed = INT32_MIN;
+
+struct Sig {
+  int32_t device;
+  int32_t act_dtype;
+  int32_t rank;
+  int32_t layout;  // trident_layout class, or -1
+  bool aux_dtype_ok, ranks_ok, shapes_ok, aux_layout_ok, aligned16;
+  int64_t T;
+  int64_t lead[2];
+  int32_t nlead;
+  int64_t fixed[TRIDENT_MAX_FIXED];
+};
+
+// Structural validation: everything that makes a call malformed rather than a miss.
+int32_t validate(const trident_args* a, const OpInfo** info) {
+  if (!a) return fail(TRIDENT_ERR_INVALID, "args is NULL");
+  if (a->op < 1 || a->op > kMaxOp) return fail(TRIDENT_ERR_INVALID, "unknown op %d", a->op);
+  const OpInfo& oi = g_ops[a->op];
+  if (a->ntensors != oi.nslots)
+    return fail(TRIDENT_ERR_INVALID, "op %d takes %d tensors, got %d", a->op, oi.nslots, a->ntensors);
+  if (a->flags != 0) return fail(TRIDENT_ERR_INVALID, "args.flags must be 0");
+  if (!(a->eps >= 0.0)) return fail(TRIDENT_ERR_INVALID, "eps must be >= 0");
+  for (int i = 0; i < oi.nslots; ++i) {
+    const trident_tensor& t = a->t[i];
+    const int es = elem_size(t.dtype);
+    if (es == 0) return fail(TRIDENT_ERR_INVALID, "tensor %d: unknown dtype %d", i, t.dtype);
+    if (t.ndim < 1 || t.ndim > 4) return fail(TRIDENT_ERR_INVALID, "tensor %d: ndim %d", i, t.ndim);
+    if (t.device < -1) return fail(TRIDENT_ERR_INVALID, "tensor %d: device %d", i, t.device);
+    bool empty = false;
+    for (int d = 0; d < t.ndim; ++d) {
+      if (t.shape[d] < 0 || t.stride[d] < 0)
+        return fail(TRIDENT_ERR_INVALID, "tensor %d: negative shape or stride", i);
+      if (t.shape[d] == 0) empty = true;
+    }
+    const uintptr_t p = reinterpret_cast<uintptr_t>(t.data);
+    if (!p && !empty) return fail(TRIDENT_ERR_INVALID, "tensor %d: NULL data", i);
+    if (p % (uintptr_t)es != 0) return fail(TRIDENT_ERR_INVALID, "tensor %d: not element-aligned", i);
+  }
+  *info = &oi;
+  return TRIDENT_OK;
+}
+
+inline bool shape_is(const trident_tensor& t, std::initializer_list<int64_t> want) {
+  int d = 0;
+  for (int64_t w : want) {
+    if (t.shape[d] != w) return false;
+    ++d;
+  }
+  return true;
+}
+
+void compute_sig(const trident_args* a, const OpInfo& oi, Sig* s) {
+  const trident_tensor* t = a->t;
+  const int n = oi.nslots;
+  // device
+  s->device = t[0].device;
+  for (int i = 1; i < n; ++i)
+    if (t[i].device != s->device) { s->device = kMixed; break; }
+  // dtypes
+  s->act_dtype = -1;
+  s->aux_dtype_ok = true;
+  for (int i = 0; i < n; ++i) {
+    const Kind k = oi.kind[i];
+    if (is_act(k) || k == K_CACHE) {
+      if (s->act_dtype == -1) s->act_dtype = t[i].dtype;
+      else if (s->act_dtype != t[i].dtype) s->act_dtype = kMixed;
+    } else if (k == K_POS) {
+      s->aux_dtype_ok &= t[i].dtype == TRIDENT_I32;
+    } else {
+      s->aux_dtype_ok &= t[i].dtype == TRIDENT_FP32;
+    }
+  }
+  // ranks
+  s->rank = t[0].ndim;
+  const int act_rank = oi.flattening ? s->rank : 2;
+  s->ranks_ok = !oi.flattening || s->rank == 2 || s->rank == 3;
+  for (int i = 0; i < n && s->ranks_ok; ++i) {
+    const Kind k = oi.kind[i];
+    const int want = (k == K_ACT_H || k == K_ACT_I) ? act_rank
+                   : (k == K_HEADS_Q || k == K_HEADS_KV || k == K_CACHE) ? 3 : 1;
+    s->ranks_ok = t[i].ndim == want;
+  }
+  s->shapes_ok = false;
+  s->layout = -1;
+  s->aux_layout_ok = false;
+  for (int i = 0; i < TRIDENT_MAX_FIXED; ++i) s->fixed[i] = -1;
+  s->T = -1;
+  if (!s->ranks_ok) return;
+  // leading dims, T and the fixed sizes read off the arguments
+  if (oi.flattening && s->rank == 3) {
+    s->nlead = 2;
+    s->lead[0] = t[0].shape[0];
+    s->lead[1] = t[0].shape[1];
+    s->T = s->lead[0] * s->lead[1];
+  } else {
+    s->nlead = 1;
+    s->lead[0] = t[0].shape[0];
+    s->T = s->lead[0];
+  }
+  int64_t H = -1, I = -1, Hq = -1, Hkv = -1, D = -1, S = -1;
+  const int op = a->op;
+  if (op == TRIDENT_OP_ADD_RMSNORM) {
+    H = t[0].shape[s->rank - 1];
+    s->fixed[0] = H;
+  } else if (op == TRIDENT_OP_SWIGLU) {
+    I = t[0].shape[s->rank - 1];
+    s->fixed[0] = I;
+  } else {
+    const int qs = (op == TRIDENT_OP_ROPE_KV || op == TRIDENT_OP_QKNORM_ROPE_KV) ? 0 : C_Q;
+    Hq = t[qs].shape[1];
+    D = t[qs].shape[2];
+    Hkv = t[qs + 1].shape[1];
+    S = t[qs + 4].shape[1];
+    if (qs == 0) {
+      s->fixed[0] = Hq; s->fixed[1] = Hkv; s->fixed[2] = D; s->fixed[3] = S;
+    } else {
+      H = t[C_H].shape[1];
+      I = t[C_G].shape[1];
+      s->fixed[0] = H; s->fixed[1] = Hq; s->fixed[2] = Hkv; s->fixed[3] = D; s->fixed[4] = S;
+      s->fixed[5] = I;
+    }
+  }
+  const int64_t T0 = s->lead[0];
+  bool ok = true;
+  for (int i = 0; i < n && ok; ++i) {
+    const trident_tensor& x = t[i];
+    switch (oi.kind[i]) {
+      case K_ACT_H: case K_ACT_I: {
+        const int64_t w = oi.kind[i] == K_ACT_H ? H : I;
+        ok = s->nlead == 2 ? shape_is(x, {s->lead[0], s->lead[1], w}) : shape_is(x, {T0, w});
+        break;
+      }
+      case K_GAMMA_H: ok = shape_is(x, {H}); break;
+      case K_GAMMA_D: ok = shape_is(x, {D}); break;
+      case K_HEADS_Q: ok = shape_is(x, {T0, Hq, D}); break;
+      case K_HEADS_KV: ok = shape_is(x, {T0, Hkv, D}); break;
+      case K_POS: ok = shape_is(x, {T0}); break;
+      case K_CACHE: ok = shape_is(x, {Hkv, S, D}); break;
+    }
+  }
+  s->shapes_ok = ok;
+  // layout class over the activations
+  bool all_contig = true, none = false;
+  for (int i = 0; i < n; ++i) {
+    if (!is_act(oi.kind[i])) continue;
+    const Rows r = rows_of(t[i], oi.kind[i]);
+    if (!r.packed) { none = true; break; }
+    if (r.n <= 1) continue;
+    if (r.stride < r.width) { none = true; break; }
+    if (r.stride != r.width) all_contig = false;
+  }
+  s->layout = none ? -1 : (all_contig ? TRIDENT_LAYOUT_CONTIG : TRIDENT_LAYOUT_ROWSTRIDED);
+  // gamma and pos dense, caches dense [Hkv, S, D]
+  bool aux = true;
+  for (int i = 0; i < n && aux; ++i) {
+    const Kind k = oi.kind[i];
+    if (k == K_GAMMA_H || k == K_GAMMA_D || k == K_POS) aux = t[i].shape[0] <= 1 || t[i].stride[0] == 1;
+    else if (k == K_CACHE)
+      aux = t[i].stride[0] == S * D && t[i].stride[1] == D && t[i].stride[2] == 1;
+  }
+  s->aux_layout_ok = aux;
+}
+
+bool aligned16(const trident_args* a, int n) {
+  for (int i = 0; i < n; ++i) {
+    const trident_tensor& t = a->t[i];
+    if (reinterpret_cast<uintptr_t>(t.data) % 16 != 0) return false;
+    const int es = elem_size(t.dtype);
+    for (int d = 0; d + 1 < t.ndim; ++d)
+      if (t.shape[d] > 1 && (t.stride[d] * es) % 16 != 0) return false;
+  }
+  return true;
+}
+
+// ------------------------------------------------------------------ versions
+struct RopeTable {
+  double theta;
+  int32_t D;
+  int64_t S;
+  float2* dev;
+};
+
+struct Version {
+  trident_spec_desc d;
+  int32_t nfixed;
+  bool rope;
+  KernelEntry ke;
+  CUfunction fn;
+  const float2* cs;
+};
+
+}  // namespace
+
+struct trident_scm {
+  trident_scm_options opt{};
+  trident_compile_hook hook = nullptr;
+  void* user = nullptr;
+  bool dry = false;
+  Version* versions = nullptr;
+  std::atomic<int32_t> count{0};
+  std::mutex reg_mu;
+  std::atomic<uint64_t>* hits_per = nullptr;
+  std::atomic<uint64_t> invokes{0}, hits{0}, misses{0}, hook_calls{0}, hook_failures{0},
+      hook_registered{0}, err_invalid{0}, err_cuda{0}, guard_evals{0};
+  // device state
+  int32_t device = 0;
+  CUcontext ctx = nullptr;
+  uint32_t* d_err = nullptr;
+  std::vector<RopeTable> tables;
+  // host timing of hits
+  uint32_t* ring = nullptr;
+  int32_t ring_cap = 0;
+  std::atomic<uint64_t> ring_n{0};
+};
+
+namespace {
+
+bool guard_holds(const Version& v, const Sig& s, const trident_args* a, int nslots,
+                 int* aligned_cache) {
+  const trident_spec_desc& d = v.d;
+  if (d.device != s.device || d.dtype != s.act_dtype || !s.aux_dtype_ok) return false;
+  if (d.rank != s.rank || !s.ranks_ok || !s.shapes_ok) return false;
+  for (int i = 0; i < v.nfixed; ++i)
+    if (d.fixed[i] != s.fixed[i]) return false;
+  if (v.rope && !(d.rope_theta == a->rope_theta)) return false;
+  if (s.T < d.tok_lo || s.T > d.tok_hi) return false;
+  if (s.layout < 0 || (d.layout != TRIDENT_LAYOUT_ANY && d.layout != s.layout)) return false;
+  if (!s.aux_layout_ok) return false;
+  if (d.align_bytes == 16) {
+    if (*aligned_cache < 0) *aligned_cache = aligned16(a, nslots) ? 1 : 0;
+    if (!*aligned_cache) return false;
+  }
+  return true;
+}
+
+// floor division for int64 with positive divisor
+inline int64_t fdiv(int64_t a, int64_t b) { return a >= 0 ? a / b : -((-a + b - 1) / b); }
+
+// Do two row sets share a byte? Rows are byte intervals [base + i*rs, base + i*rs + w).
+// Exact when one set has one row or both have the same row stride; otherwise the
+// answer is "yes" (conservative) once their overall extents intersect.
+bool rows_overlap(int64_t a, int64_t na, int64_t wa, int64_t rsa, int64_t b, int64_t nb,
+                  int64_t wb, int64_t rsb) {
+  if (na <= 0 || nb <= 0 || wa <= 0 || wb <= 0) return false;
+  const int64_t ea = a + (na - 1) * rsa + wa, eb = b + (nb - 1) * rsb + wb;
+  if (ea <= b || eb <= a) return false;
+  if (na == 1 && nb == 1) return true;  // extents are the rows
+  if (na == 1 || nb == 1) {
+    // single interval [p, p+w) against rows q + j*rs, j in [0, n)
+    const bool a1 = na == 1;
+    const int64_t p = a1 ? a : b, w = a1 ? wa : wb;
+    const int64_t q = a1 ? b : a, wq = a1 ? wb : wa, rs = a1 ? rsb : rsa, n = a1 ? nb : na;
+    // need q + j rs < p + w and p < q + j rs + wq  <=>  (p - wq - q) < j rs < (p + w - q)
+    const int64_t jmin = fdiv(p - wq - q, rs) + 1;
+    const int64_t jmax = -fdiv(-(p + w - q), rs) - 1;  // ceil(x/rs) - 1
+    const int64_t lo = jmin > 0 ? jmin : 0, hi = jmax < n - 1 ? jmax : n - 1;
+    return lo <= hi;
+  }
+  if (rsa != rsb) return true;
+  const int64_t rs = rsa, d = a - b;
+  // rows i of A and j of B overlap iff -wa < d + k rs < wb with k = i - j
+  const int64_t kmin = fdiv(-wa - d, rs) + 1;
+  const int64_t kmax = -fdiv(-(wb - d), rs) - 1;
+  const int64_t lo = kmin > -(nb - 1) ? kmin : -(nb - 1);
+  const int64_t hi = kmax < na - 1 ? kmax : na - 1;
+  return lo <= hi;
+}
+
+bool same_desc(const trident_tensor& x, const trident_tensor& y) {
+  if (x.data != y.data || x.dtype != y.dtype || x.ndim != y.ndim) return false;
+  for (int d = 0; d < x.ndim; ++d)
+    if (x.shape[d] != y.shape[d] || x.stride[d] != y.stride[d]) return false;
+  return true;
+}
+
+// Launch precondition (checked after a hit, before the launch): no output shares a byte
+// with another slot unless the two are the same tensor in one of the op's in-place groups.
+int32_t check_overlap(const trident_args* a, const OpInfo& oi) {
+  const int n = oi.nslots;
+  int64_t base[TRIDENT_MAX_TENSORS], nr[TRIDENT_MAX_TENSORS], w[TRIDENT_MAX_TENSORS],
+      rs[TRIDENT_MAX_TENSORS];
+  for (int i = 0; i < n; ++i) {
+    const Rows r = rows_of(a->t[i], oi.kind[i]);
+    const int es = elem_size(a->t[i].dtype);
+    base[i] = (int64_t)reinterpret_cast<uintptr_t>(a->t[i].data);
+    nr[i] = r.n;
+    w[i] = r.width * es;
+    rs[i] = r.stride * es;
+  }
+  for (int i = 0; i < n; ++i) {
+    if (!oi.out[i]) continue;
+    for (int j = 0; j < n; ++j) {
+      if (j == i) continue;
+      if (!rows_overlap(base[i], nr[i], w[i], rs[i], base[j], nr[j], w[j], rs[j])) continue;
+      if (oi.group[i] != 0 && oi.group[i] == oi.group[j] && same_desc(a->t[i], a->t[j])) continue;
+      return fail(TRIDENT_ERR_INVALID, "output tensor %d overlaps tensor %d", i, j);
+    }
+  }
+  return TRIDENT_OK;
+}
+
+// ------------------------------------------------------------------ parameter packing
+inline int64_t row_stride(const trident_tensor& t, Kind k) { return rows_of(t, k).stride; }
+
+void pack_addnorm(const trident_args* a, int x, int r, int g, int y, int ro, const Sig& s,
+                  Kind kind, AddNormParams* p) {
+  const trident_tensor* t = a->t;
+  p->x = t[x].data; p->r = t[r].data; p->gamma = (const float*)t[g].data;
+  p->y = t[y].data; p->r_out = t[ro].data;
+  p->T = s.T;
+  p->H = t[g].shape[0];
+  p->x_rs = row_stride(t[x], kind); p->r_rs = row_stride(t[r], kind);
+  p->y_rs = row_stride(t[y], kind); p->ro_rs = row_stride(t[ro], kind);
+  p->eps = (float)a->eps;
+  p->inv_H = (float)(1.0 / (double)p->H);
+}
+
+void pack_rope(const trident_args* a, int base, int gq, const Version& v, uint32_t* err,
+               RopeParams* p) {
+  const trident_tensor* t = a->t;
+  p->q = t[base].data; p->k = t[base + 1].data; p->v = t[base + 2].data;
+  p->pos = (const int32_t*)t[base + 3].data;
+  p->k_cache = t[base + 4].data; p->v_cache = t[base + 5].data;
+  p->gamma_q = gq >= 0 ? (const float*)t[gq].data : nullptr;
+  p->gamma_k = gq >= 0 ? (const float*)t[gq + 1].data : nullptr;
+  p->cs = v.cs;
+  p->err = err;
+  p->T = t[base].shape[0];
+  p->S = t[base + 4].shape[1];
+  p->q_rs = t[base].stride[0]; p->k_rs = t[base + 1].stride[0]; p->v_rs = t[base + 2].stride[0];
+  p->Hq = (int32_t)t[base].shape[1];
+  p->Hkv = (int32_t)t[base + 1].shape[1];
+  p->D = (int32_t)t[base].shape[2];
+  p->NH = p->Hq + 2 * p->Hkv;
+  p->eps = (float)a->eps;
+  p->inv_D = (float)(1.0 / (double)p->D);
+}
+
+void pack_swiglu(const trident_args* a, int g, int u, int o, int64_t T, SwigluParams* p) {
+  const trident_tensor* t = a->t;
+  p->g = t[g].data; p->u = t[u].data; p->out = t[o].data;
+  p->T = T;
+  p->I = t[g].shape[t[g].ndim - 1];
+  p->g_rs = row_stride(t[g], K_ACT_I); p->u_rs = row_stride(t[u], K_ACT_I);
+  p->o_rs = row_stride(t[o], K_ACT_I);
+}
+
+inline unsigned cap_grid(int64_t n) { return (unsigned)(n < 1 ? 1 : (n > 0x7fffffff ? 0x7fffffff : n)); }
+
+int32_t do_launch(trident_scm* scm, const Version& v, const trident_args* a, const Sig& s,
+                  void* stream) {
+  const int op = a->op;
+  CUlaunchConfig cfg;
+  std::memset(&cfg, 0, sizeof(cfg));
+  cfg.blockDimX = kThreads; cfg.blockDimY = 1; cfg.blockDimZ = 1;
+  cfg.gridDimY = 1; cfg.gridDimZ = 1;
+  cfg.hStream = (CUstream)stream;
+  CUlaunchAttribute attr[1];
+  std::memset(attr, 0, sizeof(attr));
+  if (scm->opt.flags & TRIDENT_OPT_PDL) {
+    attr[0].id = CU_LAUNCH_ATTRIBUTE_PROGRAMMATIC_STREAM_SERIALIZATION;
+    attr[0].value.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+  }
+  union {
+    AddNormParams an;
+    RopeParams rp;
+    SwigluParams sw;
+    ChainParams ch;
+  } P;
+  void* kp[1] = {&P};
+  switch (op) {
+    case TRIDENT_OP_ADD_RMSNORM:
+      pack_addnorm(a, 0, 1, 2, 3, 4, s, K_ACT_H, &P.an);
+      cfg.gridDimX = cap_grid(s.T);
+      break;
+    case TRIDENT_OP_ROPE_KV:
+    case TRIDENT_OP_QKNORM_ROPE_KV: {
+      pack_rope(a, 0, op == TRIDENT_OP_QKNORM_ROPE_KV ? 6 : -1, v, scm->d_err, &P.rp);
+      const int64_t units = P.rp.T * P.rp.NH;
+      const int64_t upb = v.ke.kind == KK_ROPE_HALFWARP ? rope_units_per_block(P.rp.D, 2) : kThreads / 32;
+      cfg.gridDimX = cap_grid((units + upb - 1) / upb);
+      break;
+    }
+    case TRIDENT_OP_SWIGLU:
+      pack_swiglu(a, 0, 1, 2, s.T, &P.sw);
+      if (v.ke.kind == KK_SWIGLU_TILE) {
+        const int64_t per = (int64_t)v.ke.unroll * kThreads * v.ke.vec;
+        cfg.gridDimX = cap_grid((P.sw.I + per - 1) / per);
+        cfg.gridDimY = (unsigned)(s.T < 65535 ? (s.T < 1 ? 1 : s.T) : 65535);
+      } else {
+        const int64_t total = s.T * P.sw.I;
+        cfg.gridDimX = cap_grid((total + kThreads - 1) / kThreads < 152 * 64 ? (total + kThreads - 1) / kThreads : 152 * 64);
+      }
+      break;
+    case TRIDENT_OP_LAYER_CHAIN:
+    case TRIDENT_OP_LAYER_CHAIN_QKNORM: {
+      ChainParams& c = P.ch;
+      pack_addnorm(a, C_H, C_R0, C_GA, C_X1, C_R1, s, K_ACT_H, &c.n1);
+      pack_addnorm(a, C_AO, C_R1, C_GM, C_X2, C_R2, s, K_ACT_H, &c.n2);
+      pack_rope(a, C_Q, op == TRIDENT_OP_LAYER_CHAIN_QKNORM ? C_GQ : -1, v, scm->d_err, &c.rope);
+      pack_swiglu(a, C_G, C_U, C_O, s.T, &c.sw);
+      const int64_t per = (int64_t)v.ke.unroll * kThreads * v.ke.vec;
+      const int64_t tiles = (c.sw.I + per - 1) / per;
+      const int64_t upb = rope_units_per_block(c.rope.D, 2);
+      const int64_t nA = s.T, nB = (s.T * c.rope.NH + upb - 1) / upb, nC = s.T * tiles;
+      if (nA + nB + nC > 0x7fffffff) return fail(TRIDENT_ERR_INVALID, "layer chain too large for one launch");
+      c.nA = (int32_t)nA; c.nB = (int32_t)nB; c.nC = (int32_t)nC;
+      c.sw_tiles_per_row = (int32_t)tiles;
+      cfg.gridDimX = (unsigned)(nA + nB + nC);
+      break;
+    }
+    default:
+      return fail(TRIDENT_ERR_INVALID, "op");
+  }
+  CUcontext cur = nullptr;
+  g_drv.ctx_get(&cur);
+  const bool swap = cur != scm->ctx;
+  if (swap && g_drv.ctx_push(scm->ctx) != CUDA_SUCCESS)
+    return fail(TRIDENT_ERR_CUDA, "cannot make the SCM's context current");
+  const CUresult rc = g_drv.launch_ex(&cfg, v.fn, kp, nullptr);
+  if (swap) {
+    CUcontext dummy;
+    g_drv.ctx_pop(&dummy);
+  }
+  if (rc != CUDA_SUCCESS) return fail(TRIDENT_ERR_CUDA, "cuLaunchKernelEx failed (%d)", (int)rc);
+  return TRIDENT_OK;
+}
+
+// Algorithm 1 over the current table snapshot. Returns OK with *sel, MISS, or an error.
+int32_t dispatch(const trident_scm* scm, const trident_args* a, const OpInfo** oi_out, Sig* s,
+                 int32_t* sel, bool check_alias) {
+  const OpInfo* oi = nullptr;
+  int32_t st = validate(a, &oi);
+  if (st != TRIDENT_OK) return st;
+  *oi_out = oi;
+  compute_sig(a, *oi, s);
+  const int32_t n = scm->count.load(std::memory_order_acquire);
+  int aligned = -1;
+  for (int32_t i = 0; i < n; ++i) {
+    const Version& v = scm->versions[i];
+    if (v.d.op != a->op) continue;
+    if (!guard_holds(v, *s, a, oi->nslots, &aligned)) continue;
+    if (check_alias) {
+      st = check_overlap(a, *oi);
+      if (st != TRIDENT_OK) return st;
+    }
+    *sel = i;
+    return TRIDENT_OK;
+  }
+  *sel = -1;
+  return TRIDENT_MISS;
+}
+
+inline uint64_t now_ns() {
+  return (uint64_t)std::chrono::duration_cast<std::chrono::nanoseconds>(
+             std::chrono::steady_clock::now().time_since_epoch()).count();
+}
+
+int32_t count_error(trident_scm* scm, int32_t st) {
+  if (st == TRIDENT_ERR_INVALID) scm->err_invalid.fetch_add(1, std::memory_order_relaxed);
+  else if (st == TRIDENT_ERR_CUDA) scm->err_cuda.fetch_add(1, std::memory_order_relaxed);
+  return st;
+}
+
+// Runs `fn` with the SCM's device current on this thread, restoring the previous one.
+template <class F>
+int32_t on_device(trident_scm* scm, F fn) {
+  int prev = -1;
+  if (cudaGetDevice(&prev) != cudaSuccess) prev = -1;
+  if (prev != scm->device && cudaSetDevice(scm->device) != cudaSuccess)
+    return fail(TRIDENT_ERR_CUDA, "cudaSetDevice(%d) failed", scm->device);
+  const int32_t st = fn();
+  if (prev >= 0 && prev != scm->device) cudaSetDevice(prev);
+  return st;
+}
+
+// cos/sin table [S][D/2] for RoPE base theta: angles in fp64, rounded once to fp32.
+int32_t get_rope_table(trident_scm* scm, double theta, int32_t D, int64_t S, const float2** out) {
+  for (const RopeTable& rt : scm->tables)
+    if (rt.theta == theta && rt.D == D && rt.S == S) { *out = rt.dev; return TRIDENT_OK; }
+  const int64_t half = D / 2;
+  std::vector<float2> host((size_t)(S * half));
+  std::vector<double> inv_freq((size_t)half);
+  for (int64_t i = 0; i < half; ++i) inv_freq[i] = std::pow(theta, -2.0 * (double)i / (double)D);
+  for (int64_t p = 0; p < S; ++p)
+    for (int64_t i = 0; i < half; ++i) {
+      const double ang = (double)p * inv_freq[i];
+      host[(size_t)(p * half + i)] = make_float2((float)std::cos(ang), (float)std::sin(ang));
+    }
+  float2* dev = nullptr;
+  if (cudaMalloc(&dev, host.size() * sizeof(float2)) != cudaSuccess)
+    return fail(TRIDENT_ERR_CUDA, "cudaMalloc of the RoPE table failed");
+  if (cudaMemcpy(dev, host.data(), host.size() * sizeof(float2), cudaMemcpyHostToDevice) != cudaSuccess) {
+    cudaFree(dev);
+    return fail(TRIDENT_ERR_CUDA, "upload of the RoPE table failed");
+  }
+  scm->tables.push_back({theta, D, S, dev});
+  *out = dev;
+  return TRIDENT_OK;
+}
+
+int32_t validate_desc(const trident_scm* scm, const trident_spec_desc* d, int32_t* nfixed) {
+  if (!d) return fail(TRIDENT_ERR_INVALID, "descriptor is NULL");
+  if (d->op < 1 || d->op > kMaxOp) return fail(TRIDENT_ERR_INVALID, "unknown op %d", d->op);
+  const OpInfo& oi = g_ops[d->op];
+  const bool chain = d->op == TRIDENT_OP_LAYER_CHAIN || d->op == TRIDENT_OP_LAYER_CHAIN_QKNORM;
+  if (d->dtype != TRIDENT_BF16 && d->dtype != TRIDENT_FP16 && d->dtype != TRIDENT_FP32)
+    return fail(TRIDENT_ERR_INVALID, "activation dtype %d", d->dtype);
+  if (d->dtype == TRIDENT_FP32 && (oi.rope))
+    return fail(TRIDENT_ERR_INVALID, "RoPE ops and chains take bf16 or fp16");
+  if (oi.flattening ? (d->rank != 2 && d->rank != 3) : (d->rank != (chain ? 2 : 3)))
+    return fail(TRIDENT_ERR_INVALID, "rank %d is not valid for op %d", d->rank, d->op);
+  if (d->layout < TRIDENT_LAYOUT_CONTIG || d->layout > TRIDENT_LAYOUT_ANY)
+    return fail(TRIDENT_ERR_INVALID, "layout %d", d->layout);
+  for (int i = 0; i < oi.nfixed; ++i)
+    if (d->fixed[i] < 1) return fail(TRIDENT_ERR_INVALID, "fixed[%d] must be >= 1", i);
+  for (int i = oi.nfixed; i < TRIDENT_MAX_FIXED; ++i)
+    if (d->fixed[i] != 0) return fail(TRIDENT_ERR_INVALID, "fixed[%d] must be 0 for op %d", i, d->op);
+  if (d->tok_lo < 1 || d->tok_hi < d->tok_lo) return fail(TRIDENT_ERR_INVALID, "token bucket");
+  const int es = elem_size(d->dtype);
+  if (d->align_bytes != 16 && d->align_bytes != es)
+    return fail(TRIDENT_ERR_INVALID, "align_bytes must be 16 or the element size");
+  if (!scm->dry && d->device != scm->device)
+    return fail(TRIDENT_ERR_INVALID, "version device %d differs from the SCM's %d", d->device, scm->device);
+  if (d->device < 0) return fail(TRIDENT_ERR_INVALID, "device");
+  if (d->variant < TRIDENT_VARIANT_AUTO || d->variant > TRIDENT_VARIANT_VECTOR)
+    return fail(TRIDENT_ERR_INVALID, "variant %d", d->variant);
+  if (d->variant == TRIDENT_VARIANT_VECTOR && d->align_bytes != 16)
+    return fail(TRIDENT_ERR_INVALID, "the vector variant needs align_bytes 16");
+  if (oi.rope && !(d->rope_theta > 0.0 && std::isfinite(d->rope_theta)))
+    return fail(TRIDENT_ERR_INVALID, "rope_theta must be positive");
+  if (!oi.rope && d->rope_theta != 0.0) return fail(TRIDENT_ERR_INVALID, "rope_theta must be 0");
+  if (d->reserved != 0) return fail(TRIDENT_ERR_INVALID, "reserved must be 0");
+  if (oi.rope) {
+    const int64_t D = chain ? d->fixed[3] : d->fixed[2];
+    if (D % 2 != 0 || D > 1024) return fail(TRIDENT_ERR_INVALID, "head size D must be even and <= 1024");
+  }
+  *nfixed = oi.nfixed;
+  return TRIDENT_OK;
+}
+
+// Chooses the kernel of a version (AUTO -> VECTOR when the version guarantees 16-byte
+// alignment and the sizes have a vector kernel, else GENERIC).
+int32_t resolve_kernel(const trident_spec_desc& d, KernelEntry* ke) {
+  const char* why = "";
+  const bool chain = d.op == TRIDENT_OP_LAYER_CHAIN || d.op == TRIDENT_OP_LAYER_CHAIN_QKNORM;
+  auto try_variant = [&](int32_t var) -> bool {
+    switch (d.op) {
+      case TRIDENT_OP_ADD_RMSNORM: return addnorm_kernel(d.dtype, var, d.fixed[0], ke, &why);
+      case TRIDENT_OP_SWIGLU: return swiglu_kernel(d.dtype, var, d.fixed[0], ke, &why);
+      case TRIDENT_OP_ROPE_KV:
+      case TRIDENT_OP_QKNORM_ROPE_KV:
+        return rope_kernel(d.dtype, var, (int32_t)d.fixed[2], d.op == TRIDENT_OP_QKNORM_ROPE_KV, ke, &why);
+      default:
+        if (var == TRIDENT_VARIANT_GENERIC) { why = "the layer chain has no generic variant"; return false; }
+        return chain_kernel(d.dtype, d.fixed[0], (int32_t)d.fixed[3], d.op == TRIDENT_OP_LAYER_CHAIN_QKNORM, ke, &why);
+    }
+  };
+  if (d.variant == TRIDENT_VARIANT_AUTO) {
+    if (d.align_bytes == 16 && try_variant(TRIDENT_VARIANT_VECTOR)) return TRIDENT_OK;
+    if (!chain && try_variant(TRIDENT_VARIANT_GENERIC)) return TRIDENT_OK;
+    return fail(TRIDENT_ERR_INVALID, "no kernel for this version: %s", why);
+  }
+  if (!try_variant(d.variant)) return fail(TRIDENT_ERR_INVALID, "no kernel for this version: %s", why);
+  return TRIDENT_OK;
+}
+
+}  // namespace
+
+// ====================================================================== C ABI
+TRIDENT_API int32_t trident_abi_version(void) { return TRIDENT_ABI_VERSION; }
+
+TRIDENT_API const char* trident_scm_last_error(void) { return tl_err; }
+
+TRIDENT_API const char* trident_status_name(int32_t s) {
+  switch (s) {
+    case TRIDENT_OK: return "OK";
+    case TRIDENT_MISS_HANDLED: return "MISS_HANDLED";
+    case TRIDENT_MISS: return "MISS";
+    case TRIDENT_ERR_INVALID: return "ERR_INVALID";
+    case TRIDENT_ERR_CUDA: return "ERR_CUDA";
+    case TRIDENT_ERR_HOOK: return "ERR_HOOK";
+    case TRIDENT_ERR_CAPACITY: return "ERR_CAPACITY";
+    case TRIDENT_ERR_STATE: return "ERR_STATE";
+    default: return "UNKNOWN";
+  }
+}
+
+TRIDENT_API int32_t trident_scm_create(const trident_scm_options* opt, trident_compile_hook hook,
+                                       void* user, trident_scm_t** out) {
+  if (!out) return fail(TRIDENT_ERR_INVALID, "out is NULL");
+  *out = nullptr;
+  trident_scm_options o{};
+  if (opt) o = *opt;
+  if (o.max_specs == 0) o.max_specs = 256;
+  if (o.max_specs < 1 || o.max_specs > 4096) return fail(TRIDENT_ERR_INVALID, "max_specs must be 1..4096");
+  if (o.timing_ring == 0) o.timing_ring = 65536;
+  if (o.timing_ring < 1 || o.timing_ring > (1 << 24)) return fail(TRIDENT_ERR_INVALID, "timing_ring");
+  if (o.flags & ~(TRIDENT_OPT_DRY_RUN | TRIDENT_OPT_NO_ALIAS_CHECK | TRIDENT_OPT_PDL | TRIDENT_OPT_TIMING))
+    return fail(TRIDENT_ERR_INVALID, "unknown option flags");
+  if (o.device < 0) return fail(TRIDENT_ERR_INVALID, "device");
+  trident_scm* s = new (std::nothrow) trident_scm();
+  if (!s) return fail(TRIDENT_ERR_INVALID, "out of host memory");
+  s->opt = o;
+  s->hook = hook;
+  s->user = user;
+  s->dry = (o.flags & TRIDENT_OPT_DRY_RUN) != 0;
+  s->device = o.device;
+  s->versions = static_cast<Version*>(std::calloc((size_t)o.max_specs, sizeof(Version)));
+  s->hits_per = new (std::nothrow) std::atomic<uint64_t>[(size_t)o.max_specs];
+  if (o.flags & TRIDENT_OPT_TIMING) {
+    s->ring_cap = o.timing_ring;
+    s->ring = static_cast<uint32_t*>(std::calloc((size_t)o.timing_ring, sizeof(uint32_t)));
+  }
+  if (!s->versions || !s->hits_per || ((o.flags & TRIDENT_OPT_TIMING) && !s->ring)) {
+    trident_scm_destroy(s);
+    return fail(TRIDENT_ERR_INVALID, "out of host memory");
+  }
+  for (int i = 0; i < o.max_specs; ++i) s->hits_per[i].store(0);
+  if (!s->dry) {
+    if (!driver()) {
+      trident_scm_destroy(s);
+      return fail(TRIDENT_ERR_CUDA, "CUDA driver entry points unavailable");
+    }
+    const int32_t st = on_device(s, [&]() -> int32_t {
+      if (cudaFree(nullptr) != cudaSuccess) return fail(TRIDENT_ERR_CUDA, "CUDA init failed");
+      if (g_drv.ctx_get(&s->ctx) != CUDA_SUCCESS || !s->ctx)
+        return fail(TRIDENT_ERR_CUDA, "no current CUDA context");
+      if (cudaMalloc(&s->d_err, sizeof(uint32_t)) != cudaSuccess)
+        return fail(TRIDENT_ERR_CUDA, "cudaMalloc of the status word failed");
+      if (cudaMemset(s->d_err, 0, sizeof(uint32_t)) != cudaSuccess)
+        return fail(TRIDENT_ERR_CUDA, "cudaMemset failed");
+      return TRIDENT_OK;
+    });
+    if (st != TRIDENT_OK) {
+      trident_scm_destroy(s);
+      return st;
+    }
+  }
+  *out = s;
+  return TRIDENT_OK;
+}
+
+TRIDENT_API int32_t trident_scm_register_spec(trident_scm_t* scm, const trident_spec_desc* desc,
+                                              int32_t* out_index) {
+  if (!scm) return fail(TRIDENT_ERR_INVALID, "scm is NULL");
+  int32_t nfixed = 0;
+  int32_t st = validate_desc(scm, desc, &nfixed);
+  if (st != TRIDENT_OK) return st;
+  Version v;
+  std::memset(&v, 0, sizeof(v));
+  v.d = *desc;
+  v.nfixed = nfixed;
+  v.rope = g_ops[desc->op].rope;
+  st = resolve_kernel(v.d, &v.ke);
+  if (st != TRIDENT_OK) return st;
+  std::lock_guard<std::mutex> lk(scm->reg_mu);
+  const int32_t n = scm->count.load(std::memory_order_relaxed);
+  if (n >= scm->opt.max_specs) return fail(TRIDENT_ERR_CAPACITY, "version table full (%d)", n);
+  if (!scm->dry) {
+    st = on_device(scm, [&]() -> int32_t {
+      cudaFunction_t f = nullptr;
+      if (cudaGetFuncBySymbol(&f, v.ke.fn) != cudaSuccess || !f)
+        return fail(TRIDENT_ERR_CUDA, "cannot resolve the kernel entry");
+      v.fn = reinterpret_cast<CUfunction>(f);
+      if (v.rope) {
+        const bool chain = desc->op == TRIDENT_OP_LAYER_CHAIN || desc->op == TRIDENT_OP_LAYER_CHAIN_QKNORM;
+        const int32_t D = (int32_t)(chain ? desc->fixed[3] : desc->fixed[2]);
+        const int64_t S = chain ? desc->fixed[4] : desc->fixed[3];
+        return get_rope_table(scm, desc->rope_theta, D, S, &v.cs);
+      }
+      return TRIDENT_OK;
+    });
+    if (st != TRIDENT_OK) return st;
+  }
+  scm->versions[n] = v;
+  scm->hits_per[n].store(0, std::memory_order_relaxed);
+  scm->count.store(n + 1, std::memory_order_release);
+  if (tl_hook_depth > 0) scm->hook_registered.fetch_add(1, std::memory_order_relaxed);
+  if (out_index) *out_index = n;
+  return TRIDENT_OK;
+}
+
+TRIDENT_API int32_t trident_scm_select(const trident_scm_t* scm, const trident_args* args,
+                                       int32_t* out_selected) {
+  if (out_selected) *out_selected = -1;
+  if (!scm) return fail(TRIDENT_ERR_INVALID, "scm is NULL");
+  const OpInfo* oi = nullptr;
+  Sig s;
+  int32_t sel = -1;
+  const int32_t st = dispatch(scm, args, &oi, &s, &sel, !(scm->opt.flags & TRIDENT_OPT_NO_ALIAS_CHECK));
+  if (out_selected) *out_selected = sel;
+  return st;
+}
+
+TRIDENT_API int32_t trident_scm_invoke(trident_scm_t* scm, const trident_args* args, void* stream,
+                                       int32_t* out_selected) {
+  if (out_selected) *out_selected = -1;
+  if (!scm) return fail(TRIDENT_ERR_INVALID, "scm is NULL");
+  const bool timing = scm->ring != nullptr;
+  const uint64_t t0 = timing ? now_ns() : 0;
+  scm->invokes.fetch_add(1, std::memory_order_relaxed);
+  const OpInfo* oi = nullptr;
+  Sig s;
+  int32_t sel = -1;
+  int32_t st = dispatch(scm, args, &oi, &s, &sel, !(scm->opt.flags & TRIDENT_OPT_NO_ALIAS_CHECK));
+  if (st == TRIDENT_OK) {
+    const Version& v = scm->versions[sel];
+    if (!scm->dry) {
+      st = do_launch(scm, v, args, s, stream);
+      if (st != TRIDENT_OK) return count_error(scm, st);  // Algorithm 1: raise, no next version
+    }
+    scm->hits.fetch_add(1, std::memory_order_relaxed);
+    scm->hits_per[sel].fetch_add(1, std::memory_order_relaxed);
+    scm->guard_evals.fetch_add((uint64_t)sel + 1, std::memory_order_relaxed);
+    if (timing) {
+      const uint64_t k = scm->ring_n.fetch_add(1, std::memory_order_relaxed);
+      const uint64_t dt = now_ns() - t0;
+      scm->ring[k % (uint64_t)scm->ring_cap] = dt > 0xffffffffull ? 0xffffffffu : (uint32_t)dt;
+    }
+    if (out_selected) *out_selected = sel;
+    return TRIDENT_OK;
+  }
+  if (st != TRIDENT_MISS) return count_error(scm, st);
+  // every guard failed: a specialisation miss (§3.5)
+  scm->misses.fetch_add(1, std::memory_order_relaxed);
+  scm->guard_evals.fetch_add((uint64_t)scm->count.load(std::memory_order_relaxed),
+                             std::memory_order_relaxed);
+  if (!scm->hook || tl_hook_depth > 0) return TRIDENT_MISS;
+  scm->hook_calls.fetch_add(1, std::memory_order_relaxed);
+  int32_t reg = -1;
+  ++tl_hook_depth;
+  const int32_t hr = scm->hook(scm->user, scm, args, stream, &reg);
+  --tl_hook_depth;
+  if (hr != 0) {
+    scm->hook_failures.fetch_add(1, std::memory_order_relaxed);
+    return fail(TRIDENT_ERR_HOOK, "compile hook returned %d", hr);
+  }
+  if (out_selected) *out_selected = reg;
+  return TRIDENT_MISS_HANDLED;
+}
+
+TRIDENT_API int32_t trident_scm_invoke_seq(trident_scm_t* scm, const trident_args* args, int32_t n,
+                                           void* stream, int32_t* out_selected) {
+  if (!scm || (!args && n > 0) || n < 0) return fail(TRIDENT_ERR_INVALID, "bad sequence");
+  int32_t result = TRIDENT_OK;
+  for (int32_t i = 0; i < n; ++i) {
+    int32_t sel = -1;
+    const int32_t st = trident_scm_invoke(scm, args + i, stream, &sel);
+    if (out_selected) out_selected[i] = sel;
+    if (st < 0 || st == TRIDENT_MISS) {
+      if (out_selected)
+        for (int32_t j = i + 1; j < n; ++j) out_selected[j] = TRIDENT_NOT_RUN;
+      return st;
+    }
+    if (st == TRIDENT_MISS_HANDLED) result = TRIDENT_MISS_HANDLED;
+  }
+  return result;
+}
+
+TRIDENT_API int32_t trident_scm_stats(const trident_scm_t* scm, trident_scm_stats_t* out) {
+  if (!scm || !out) return fail(TRIDENT_ERR_INVALID, "NULL argument");
+  std::memset(out, 0, sizeof(*out));
+  out->invokes = scm->invokes.load();
+  out->hits = scm->hits.load();
+  out->misses = scm->misses.load();
+  out->hook_calls = scm->hook_calls.load();
+  out->hook_failures = scm->hook_failures.load();
+  out->hook_registered = scm->hook_registered.load();
+  out->err_invalid = scm->err_invalid.load();
+  out->err_cuda = scm->err_cuda.load();
+  out->guard_evals = scm->guard_evals.load();
+  out->num_specs = scm->count.load();
+  return TRIDENT_OK;
+}
+
+TRIDENT_API int32_t trident_scm_spec_hits(const trident_scm_t* scm, uint64_t* out, int32_t cap,
+                                          int32_t* n) {
+  if (!scm || (cap > 0 && !out) || cap < 0) return fail(TRIDENT_ERR_INVALID, "bad arguments");
+  const int32_t cnt = scm->count.load(std::memory_order_acquire);
+  const int32_t m = cnt < cap ? cnt : cap;
+  for (int32_t i = 0; i < m; ++i) out[i] = scm->hits_per[i].load(std::memory_order_relaxed);
+  if (n) *n = cnt;
+  return TRIDENT_OK;
+}
+
+TRIDENT_API int32_t trident_scm_host_times(const trident_scm_t* scm, uint32_t* out, int32_t cap,
+                                           int32_t* n) {
+  if (!scm || (cap > 0 && !out) || cap < 0) return fail(TRIDENT_ERR_INVALID, "bad arguments");
+  if (!scm->ring) return fail(TRIDENT_ERR_STATE, "TRIDENT_OPT_TIMING is off");
+  const uint64_t total = scm->ring_n.load(std::memory_order_relaxed);
+  const uint64_t have = total < (uint64_t)scm->ring_cap ? total : (uint64_t)scm->ring_cap;
+  const uint64_t m = have < (uint64_t)cap ? have : (uint64_t)cap;
+  const uint64_t first = total - m;
+  for (uint64_t i = 0; i < m; ++i) out[i] = scm->ring[(first + i) % (uint64_t)scm->ring_cap];
+  if (n) *n = (int32_t)m;
+  return TRIDENT_OK;
+}
+
+TRIDENT_API int32_t trident_scm_device_status(trident_scm_t* scm, void* stream, uint32_t* out_bits,
+                                              int32_t clear) {
+  if (!scm || !out_bits) return fail(TRIDENT_ERR_INVALID, "NULL argument");
+  if (scm->dry) return fail(TRIDENT_ERR_STATE, "dry-run SCM has no device state");
+  return on_device(scm, [&]() -> int32_t {
+    if (cudaStreamSynchronize((cudaStream_t)stream) != cudaSuccess)
+      return fail(TRIDENT_ERR_CUDA, "stream synchronize failed: %s", cudaGetErrorString(cudaGetLastError()));
+    if (cudaMemcpy(out_bits, scm->d_err, sizeof(uint32_t), cudaMemcpyDeviceToHost) != cudaSuccess)
+      return fail(TRIDENT_ERR_CUDA, "status read failed");
+    if (clear && cudaMemset(scm->d_err, 0, sizeof(uint32_t)) != cudaSuccess)
+      return fail(TRIDENT_ERR_CUDA, "status clear failed");
+    return TRIDENT_OK;
+  });
+}
+
+TRIDENT_API void trident_scm_destroy(trident_scm_t* scm) {
+  if (!scm) return;
+  if (!scm->dry && (scm->d_err || !scm->tables.empty())) {
+    on_device(scm, [&]() -> int32_t {
+      for (RopeTable& rt : scm->tables) cudaFree(rt.dev);
+      if (scm->d_err) cudaFree(scm->d_err);
+      return TRIDENT_OK;
+    });
+  }
+  std::free(scm->versions);
+  delete[] scm->hits_per;
+  std::free(scm->ring);
+  delete scm;
+}

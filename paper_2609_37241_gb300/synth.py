@@ -112,3 +112,20 @@ def stress_trace(g, cfg=STRESS):
     dt = np.where(g.random(n) < cfg["p_fp16"], FP16, BF16).astype(np.int32)
     strided = (g.random(n) < cfg["p_strided"])
     return T, dt, strided
+
+
+def act_device(shape, dtype, seed, device="cuda", mean=0.0, std=1.0):
+    """Large activation drawn on the device by torch's seeded generator (N(mean, std) in
+    fp32, then cast): for full-size workloads where host generation would dominate."""
+    gen = torch.Generator(device=device)
+    gen.manual_seed(seed)
+    t = torch.randn(shape, generator=gen, device=device, dtype=torch.float32)
+    if std != 1.0 or mean != 0.0:
+        t = t * std + mean
+    return t.to(_TORCH_DT[dtype])
+
+
+def gamma_device(n, seed, device="cuda"):
+    gen = torch.Generator(device=device)
+    gen.manual_seed(seed)
+    return torch.randn(n, generator=gen, device=device, dtype=torch.float32) * 0.1 + 1.0

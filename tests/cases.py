@@ -109,3 +109,54 @@ def make_args(d):
         ts = ts + [tensor(alloc(), 3, (1,), device=dev)] * delta
     return dict(op=op, tensors=ts, eps=float(d.get("eps", 1e-6)),
                 theta=float(d.get("theta", 0.0)), flags=0)
+
+
+def make_chain_args(d):
+    """Argument tuple for ops 5/6 (layer chains). layout 'contig': separate dense
+    buffers; 'strided': q/k/v views of one qkv buffer and g/u halves of one [T, 2I]."""
+    op = d["op"]
+    dt = DT[d.get("dtype", "bf16")]
+    dev = d.get("device", 0)
+    alloc = _Alloc()
+    T, H, Hq, Hkv, D, S, I = (d[k] for k in ("T", "H", "Hq", "Hkv", "D", "S", "I"))
+    es = ES[dt]
+    act = lambda w: tensor(alloc(), dt, (T, w), device=dev)
+    ts = [act(H), act(H), tensor(alloc(), 3, (H,), device=dev), act(H), act(H)]
+    if d.get("layout", "contig") == "contig":
+        q = tensor(alloc(), dt, (T, Hq, D), device=dev)
+        k = tensor(alloc(), dt, (T, Hkv, D), device=dev)
+        v = tensor(alloc(), dt, (T, Hkv, D), device=dev)
+        g, u = act(I), act(I)
+    else:
+        W = (Hq + 2 * Hkv) * D
+        base = alloc()
+        q = tensor(base, dt, (T, Hq, D), (W, D, 1), dev)
+        k = tensor(base + Hq * D * es, dt, (T, Hkv, D), (W, D, 1), dev)
+        v = tensor(base + (Hq + Hkv) * D * es, dt, (T, Hkv, D), (W, D, 1), dev)
+        gu = alloc()
+        g = tensor(gu, dt, (T, I), (2 * I, 1), dev)
+        u = tensor(gu + I * es, dt, (T, I), (2 * I, 1), dev)
+    ts += [q, k, v, tensor(alloc(), 4, (T,), device=dev),
+           tensor(alloc(), dt, (Hkv, S, D), device=dev), tensor(alloc(), dt, (Hkv, S, D), device=dev),
+           act(H), tensor(alloc(), 3, (H,), device=dev), act(H), act(H), g, u, act(I)]
+    if op == 6:
+        ts += [tensor(alloc(), 3, (D,), device=dev), tensor(alloc(), 3, (D,), device=dev)]
+    return dict(op=op, tensors=ts, eps=float(d.get("eps", 1e-6)), theta=float(d.get("theta", 0.0)),
+                flags=0)
+
+
+def lib_spec(spec):
+    """Library descriptor (ctypes) from an oracle-style spec dict."""
+    from paper_2609_37241_gb300 import scm
+    return scm.make_spec(spec["op"], spec["dtype"], spec["fixed"], spec["tok_lo"], spec["tok_hi"],
+                         rank=spec["rank"], layout=spec["layout"], align_bytes=spec["align"],
+                         device=spec["device"], variant=spec["variant"], rope_theta=spec["theta"])
+
+
+def lib_args(args):
+    """Library argument tuple (ctypes) from an oracle-style args dict."""
+    from paper_2609_37241_gb300 import scm
+    return scm.make_args(args["op"], args["tensors"], eps=args["eps"], rope_theta=args["theta"])
+
+
+STATUS = {0: "OK", 2: "MISS", -1: "INVALID"}

@@ -25,3 +25,12 @@ def pytest_collection_modifyitems(config, items):
     for item in items:
         if "gpu" in item.keywords:
             item.add_marker(skip)
+
+
+@pytest.fixture(scope="session")
+def built_lib():
+    """The C-ABI library, built in-tree first if it is missing or stale."""
+    from paper_2609_37241_gb300 import build
+    build.build()
+    from paper_2609_37241_gb300 import scm
+    return scm.lib()
