@@ -233,6 +233,15 @@ def layer_scm(c, cfg, pdl=True, timing=False):
     return s
 
 
+def assert_all_hit(scm, what):
+    """Every timed call must have been a cache hit that launched (no silent misses)."""
+    st = scm.stats()
+    if st.misses or st.err_invalid or st.err_cuda or st.hits != st.invokes:
+        raise RuntimeError(f"{what}: {st.invokes} invokes, {st.hits} hits, {st.misses} misses, "
+                           f"{st.err_invalid} invalid, {st.err_cuda} cuda errors")
+    return st.hits
+
+
 def time_steps(c, fn, K, W):
     """Runs fn(i) for W warm-up then K timed steps; returns (us per step on the device
     clock, host us per step)."""
@@ -292,6 +301,7 @@ def bench_layer(c, cfg, T, K, W, layers=1, min_bytes=2 * L2_BYTES):
         nat_us = None
     st, bits = S.trident_scm_device_status(h, c.sp.value)
     assert st == S.OK and bits == 0
+    assert_all_hit(scm, "layer T=%d" % T)
     scm.close()
     res = dict(fused_us=round(fus_dev, 3), fused_host_us=round(fus_host, 3), unfused_us=round(unf_dev, 3),
                unfused_host_us=round(unf_host, 3), launches_per_step=list(n_launch), sets=R,
@@ -324,6 +334,7 @@ def bench_e2e(c, cfg, T, K, W):
             h.copy_(d, non_blocking=True)
 
     us, host_us = time_steps(c, step, K, W)
+    assert_all_hit(scm, "e2e")
     c.launches += K
     bi = sum(h.numel() * h.element_size() for _, h in ins)
     bo = sum(h.numel() * h.element_size() for _, h in outs)
@@ -359,6 +370,7 @@ def bench_host_hit(c, n=1000):
     t.cuda.synchronize()
     st, ns = S.trident_scm_host_times(s.h, n)
     hits = S.trident_scm_spec_hits(s.h)[1]
+    assert_all_hit(s, "host dispatch")
     ns = np.array(ns[-n:], np.float64)
     c.launches += n
     s.close()
@@ -524,6 +536,7 @@ def bench_sweep(c, reps=20, quick=False):
                                   frac_measured=round(b / us / 1e3 / peak, 3),
                                   frac_8tbs=round(b / us / 1e3 / NOMINAL_HBM_GBS, 3)))
     del g, u, o
+    assert_all_hit(s, "sweep")
     s.close()
     big = [e for e in out["add_rmsnorm"] + out["swiglu"] if e["T"] >= 4096]
     out["min_frac_measured_T_ge_4096"] = min(e["frac_measured"] for e in big) if big else None
@@ -539,6 +552,7 @@ def kernel_duration_chain(c, cfg, T, reps=200):
     n = min(reps, sets.R)
     arr = (S.trident_args * n)(*[sets.fused_args(c, i) for i in range(n)])
     us, _ = time_steps(c, lambda i: c.L.trident_scm_invoke_seq(scm.h, arr, n, c.sp, None), 5, 3)
+    assert_all_hit(scm, "roofline kernel")
     c.launches += 8 * n
     scm.close()
     return us / n
@@ -591,8 +605,8 @@ def run_ours(a):
     e1.record(c.stream)
     barrier()
     ms = e0.elapsed_time(e1)
+    headline_launches = assert_all_hit(scm, "headline") - W
     c.launches += K
-    headline_launches = K
     scm.close()
     del sets
     t_local = torch.tensor([ms], dtype=torch.float64, device=c.dev)
@@ -602,24 +616,30 @@ def run_ours(a):
     us_step = ms_max * 1e3 / K
 
     extra = {}
-    if rank == 0:
+    want = (lambda name: True) if a.sections == "all" else (lambda name: name in a.sections.split(","))
+    if rank == 0 and want("layers"):
         progress("per-token layer steps")
         per_t = {}
         for T in (1, 4, 16, 64):
             per_t[str(T)], _ = bench_layer(c, cfg, T, K=min(K, 2000), W=W)
         extra["llama_per_tokens"] = per_t
+    if rank == 0 and want("qwen3"):
         progress("qwen3 36-layer steps")
         qw = {}
         for T in ((1, 8, 32, 128) if not a.quick else (1, 128)):
             qw[str(T)], _ = bench_layer(c, synth.QWEN3, T, K=max(20, min(K, 2000) // 36), W=W,
                                         layers=36)
         extra["qwen3_36layer_step"] = qw
+    if rank == 0 and want("host"):
         progress("host dispatch")
         extra["host_dispatch_single_addnorm"] = bench_host_hit(c)
+    if rank == 0 and want("stress"):
         progress("guard stress")
         extra["guard_stress"] = bench_guard_stress(c, n_calls=20000 if a.quick else None)
+    if rank == 0 and want("sweep"):
         progress("hbm sweep")
         extra["hbm_sweep"] = bench_sweep(c, quick=a.quick)
+    if rank == 0 and want("roofline"):
         progress("roofline kernel")
         kd = kernel_duration_chain(c, cfg, HEADLINE_T)
         peak, src = measured_peaks()
@@ -628,13 +648,16 @@ def run_ours(a):
                                  frac=round(b / kd / 1e3 / peak, 3), traffic=None,
                                  kernel="chain_kernel<bf16,H4096,D128>",
                                  bytes_per_launch=int(b), us_per_launch=round(kd, 3), peak_source=src)
+    if rank == 0 and want("e2e"):
         progress("e2e")
         extra["e2e"] = bench_e2e(c, cfg, HEADLINE_T, K=min(K, 500), W=W)
     ck = clocks.stop()
     if rank == 0:
-        progress("cpu baseline")
-        budget = 3.0 if a.quick else 12.0
-        cpu_us, n = oracle_layer_step_us(cfg, HEADLINE_T, budget)
+        cpu_us = n = None
+        if want("cpu"):
+            progress("cpu baseline")
+            budget = 3.0 if a.quick else 12.0
+            cpu_us, n = oracle_layer_step_us(cfg, HEADLINE_T, budget)
         line = dict(metric=METRIC, value=round(us_step, 3), unit=UNIT, n_gpus=world, steps=K, warmup=W,
                     ms_per_step=round(us_step / 1e3, 6), higher_is_better=False, scaling="weak",
                     vs_baseline=None, dtype="bf16",
@@ -648,8 +671,9 @@ def run_ours(a):
                                 parallelism="replicas" if world > 1 else "single GPU"),
                     gpu_launches=headline_launches, gpu_launches_whole_run=c.launches)
         line.update(extra)
-        line["cpu_baseline"] = dict(value=round(cpu_us, 1), unit=UNIT, cores=1, kind="oracle",
-                                    sample="%d layer steps at 64 tokens (%.1f s)" % (n, cpu_us * n / 1e6))
+        if cpu_us is not None:
+            line["cpu_baseline"] = dict(value=round(cpu_us, 1), unit=UNIT, cores=1, kind="oracle",
+                                        sample="%d layer steps at 64 tokens (%.1f s)" % (n, cpu_us * n / 1e6))
         if ck:
             line["clocks"] = ck
         print(json.dumps(line), flush=True)
@@ -712,6 +736,9 @@ def main():
     p.add_argument("--warmup", type=int, default=20)
     p.add_argument("--impl", default="ours", choices=["ours", "reference"])
     p.add_argument("--quick", action="store_true", help="smaller sections (for smoke runs)")
+    p.add_argument("--sections", default="all",
+                   help="comma list of: layers,qwen3,host,stress,sweep,roofline,e2e,cpu (default all;"
+                        " the headline always runs)")
     a = p.parse_args()
     if a.warmup < 3:
         a.warmup = 3

@@ -180,7 +180,8 @@ typedef struct trident_spec_desc {
                                        ROPE ops {Hq, Hkv, D, S};
                                        chains {H, Hq, Hkv, D, S, I}; unused entries 0    */
   int64_t tok_lo, tok_hi;           /* inclusive token-count bucket, 1 <= lo <= hi       */
-  int32_t align_bytes;              /* 16: every pointer and row stride 16-byte aligned;
+  int32_t align_bytes;              /* 16: every pointer and every outer stride 16-byte
+                                       aligned (positions excepted: read per element);
                                        or the element size (no extra requirement)        */
   int32_t device;                   /* CUDA ordinal; must equal the SCM's device         */
   int32_t variant;                  /* trident_variant                                   */

@@ -210,9 +210,13 @@ def aux_layout_ok(args, fx):
 
 
 def aligned16(args):
-    """Every pointer is a multiple of 16 bytes, and so is every stride (in bytes) of every
-    dimension except the innermost, among dimensions of size > 1."""
-    for t in args["tensors"]:
+    """Every tensor the kernels move in 16-byte units -- all but the positions, which are
+    read one element at a time -- starts on a multiple of 16 bytes, and so does every
+    stride (in bytes) of every dimension except the innermost, among dimensions of
+    size > 1."""
+    for (name, kind, _), t in zip(SLOTS[args["op"]], args["tensors"]):
+        if kind == "pos":
+            continue
         es = ELEM_SIZE[t["dtype"]]
         if t["addr"] % 16 != 0:
             return False

@@ -352,8 +352,11 @@ void compute_sig(const trident_args* a, const OpInfo& oi, Sig* s) {
   s->aux_layout_ok = aux;
 }
 
-bool aligned16(const trident_args* a, int n) {
-  for (int i = 0; i < n; ++i) {
+// 16-byte alignment of every tensor the kernels move in 16-byte units (positions are
+// read one element at a time and only need their natural alignment).
+bool aligned16(const trident_args* a, const OpInfo& oi) {
+  for (int i = 0; i < oi.nslots; ++i) {
+    if (oi.kind[i] == K_POS) continue;
     const trident_tensor& t = a->t[i];
     if (reinterpret_cast<uintptr_t>(t.data) % 16 != 0) return false;
     const int es = elem_size(t.dtype);
@@ -406,7 +409,7 @@ struct trident_scm {
 
 namespace {
 
-bool guard_holds(const Version& v, const Sig& s, const trident_args* a, int nslots,
+bool guard_holds(const Version& v, const Sig& s, const trident_args* a, const OpInfo& oi,
                  int* aligned_cache) {
   const trident_spec_desc& d = v.d;
   if (d.device != s.device || d.dtype != s.act_dtype || !s.aux_dtype_ok) return false;
@@ -418,7 +421,7 @@ bool guard_holds(const Version& v, const Sig& s, const trident_args* a, int nslo
   if (s.layout < 0 || (d.layout != TRIDENT_LAYOUT_ANY && d.layout != s.layout)) return false;
   if (!s.aux_layout_ok) return false;
   if (d.align_bytes == 16) {
-    if (*aligned_cache < 0) *aligned_cache = aligned16(a, nslots) ? 1 : 0;
+    if (*aligned_cache < 0) *aligned_cache = aligned16(a, oi) ? 1 : 0;
     if (!*aligned_cache) return false;
   }
   return true;
@@ -632,7 +635,7 @@ int32_t dispatch(const trident_scm* scm, const trident_args* a, const OpInfo** o
   for (int32_t i = 0; i < n; ++i) {
     const Version& v = scm->versions[i];
     if (v.d.op != a->op) continue;
-    if (!guard_holds(v, *s, a, oi->nslots, &aligned)) continue;
+    if (!guard_holds(v, *s, a, *oi, &aligned)) continue;
     if (check_alias) {
       st = check_overlap(a, *oi);
       if (st != TRIDENT_OK) return st;
