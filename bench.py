@@ -36,6 +36,30 @@ L2_BYTES = 129 * 2 ** 20
 NOMINAL_HBM_GBS = 8000.0
 
 
+CHAIN_SOURCES = ["paper_2609_37241_gb300/csrc/chain.cu", "paper_2609_37241_gb300/csrc/device_common.cuh",
+                 "paper_2609_37241_gb300/csrc/internal.h"]
+CHAIN_PROFILE = "profiles/chain_kernel_llama_t64.md"
+
+
+def chain_traffic():
+    """DRAM bytes per launch of the chain kernel from the committed ncu summary, or None
+    when the kernel sources changed since those counters were taken."""
+    import hashlib
+    import re
+    try:
+        h = hashlib.sha256()
+        for f in CHAIN_SOURCES:
+            with open(os.path.join(ROOT, f), "rb") as fh:
+                h.update(fh.read())
+        with open(os.path.join(ROOT, CHAIN_PROFILE)) as fh:
+            txt = fh.read()
+        sha = re.search(r"source_sha256: ([0-9a-f]{64})", txt).group(1)
+        traffic = int(re.search(r"traffic_bytes_per_launch: (\d+)", txt).group(1))
+        return traffic if sha == h.hexdigest() else None
+    except Exception:
+        return None
+
+
 def measured_peaks():
     try:
         with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
@@ -645,7 +669,7 @@ def run_ours(a):
         peak, src = measured_peaks()
         b = chain_bytes_per_launch(cfg, HEADLINE_T)
         extra["roofline"] = dict(bound="hbm", achieved=round(b / kd / 1e3, 1), peak=peak, unit="GB/s",
-                                 frac=round(b / kd / 1e3 / peak, 3), traffic=None,
+                                 frac=round(b / kd / 1e3 / peak, 3), traffic=chain_traffic(),
                                  kernel="chain_kernel<bf16,H4096,D128>",
                                  bytes_per_launch=int(b), us_per_launch=round(kd, 3), peak_source=src)
     if rank == 0 and want("e2e"):
