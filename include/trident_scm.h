@@ -288,6 +288,25 @@ int32_t trident_scm_host_times(const trident_scm_t* scm, uint32_t* out, int32_t 
 int32_t trident_scm_device_status(trident_scm_t* scm, void* stream, uint32_t* out_bits,
                                   int32_t clear);
 
+/* RoPE + KV-cache append (ROPE_KV or QKNORM_ROPE_KV argument tuple, same slots and math)
+ * that allocates nothing, for callers that cannot allocate device memory -- for example a
+ * serving engine that has given all of HBM to its own pool, or code where a cudaMalloc
+ * would synchronise the device. The paper has no counterpart: it is an addition of this
+ * library. There is no SCM handle and no guard table: the call validates the tuple,
+ * requires what the vector kernel needs (bf16 or fp16, D in {64, 128, 256}, 16-byte
+ * aligned tensors, dense caches, tensors on the current device) and launches on `stream`.
+ * Its scratch -- the status word and the (cos, sin) table -- lives in one static device
+ * array of 256 bytes + 4 MiB that every GPU loading the library holds until exit; S * D/2
+ * above 524288 (cos, sin) pairs is rejected with ERR_INVALID. The first call on a device
+ * looks up the array's device address (cudaGetSymbolAddress), so make that first call
+ * before any stream capture. Every call shares the array, which keeps the last call's
+ * table: the table is rebuilt on the device when (theta, D, S) changes, and the status
+ * word is cleared at the start of each call. Calls that overlap on the GPU (other
+ * streams, other host threads) race on the array. *out_status (may be NULL) receives the
+ * status word (TRIDENT_DEVERR_* bits) by an asynchronous copy on `stream`: read it after
+ * synchronising the stream. Errors: ERR_INVALID, ERR_CUDA. */
+int32_t trident_rope_kv_noalloc(const trident_args* args, void* stream, uint32_t* out_status);
+
 /* Frees the SCM, its tables and device memory. The caller must ensure no call on it
  * is running and its kernels have finished. NULL is ignored. */
 void trident_scm_destroy(trident_scm_t* scm);

@@ -90,6 +90,15 @@ bool swiglu_kernel(int32_t dtype, int32_t variant, int64_t I, KernelEntry* out, 
 bool chain_kernel(int32_t dtype, int64_t H, int32_t D, bool qknorm, KernelEntry* out,
                   const char** why);
 
+// Validation, guard-equivalent checks (sizes, layouts, 16-byte alignment, overlap) and
+// parameter packing of a ROPE_KV / QKNORM_ROPE_KV argument tuple without an SCM. Leaves
+// p->cs and p->err NULL. Returns a trident_status (message in trident_scm_last_error).
+int32_t prepare_rope_args(const void* trident_args_ptr, RopeParams* p, int32_t* dtype,
+                          bool* qknorm);
+
+// Sets the thread-local last-error message and returns `status`.
+int32_t internal_fail(int32_t status, const char* msg);
+
 // Units (head-rows) handled by one block of the vector RoPE kernel for head size D.
 inline int32_t rope_units_per_block(int32_t D, int32_t elem_bytes) {
   int32_t lanes_per_head = D * elem_bytes / 16;

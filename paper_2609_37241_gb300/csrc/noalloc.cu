@@ -1,0 +1,127 @@
+// noalloc.cu -- RoPE + KV-cache append that allocates nothing.
+//
+// The SCM path keeps two pieces of scratch memory in device allocations it makes itself:
+// the cos/sin table of a RoPE version (cudaMalloc at registration) and the device status
+// word (cudaMalloc at creation). Some callers cannot allocate device memory at all: a
+// serving engine that has handed every byte of HBM to its own pool, or code running where
+// a cudaMalloc would synchronise the device and stall other streams. For them,
+// trident_rope_kv_noalloc runs the same vector RoPE/KV kernel with its scratch in a
+// file-scope static device array of fixed size, so no call allocates anything (no
+// cudaMalloc, no cudaFree, no allocating library routine).
+//
+// Scratch layout (kScratchBytes = 256 + 4 MiB, held by every GPU that loads the library
+// until the process exits): bytes [0, 4) the status word, bytes [256, end) the
+// (cos, sin) table [S][D/2] in fp32, at most kMaxPairs = 524288 pairs (for example
+// S 8192 x D 128). The table is recomputed on the device (angles in fp64, rounded once to
+// fp32) only when (theta, D, S) differs from what the array held after the previous call
+// on that device; the status word is cleared at the start of every call.
+#include <cuda_runtime.h>
+
+#include <cmath>
+#include <mutex>
+
+#include "device_common.cuh"
+#include "trident_scm.h"
+
+namespace trident {
+namespace {
+
+constexpr size_t kTableOffset = 256;
+constexpr int64_t kMaxPairs = int64_t(1) << 19;
+constexpr size_t kScratchBytes = kTableOffset + size_t(kMaxPairs) * sizeof(float2);
+constexpr int kMaxDevices = 64;
+
+static __device__ __align__(256) unsigned char g_scratch[kScratchBytes];
+
+struct DeviceScratch {
+  std::once_flag once;
+  cudaError_t setup_error = cudaSuccess;
+  unsigned char* addr = nullptr;  // device address of g_scratch on this device
+  std::mutex mu;                  // guards the table key below
+  double theta = 0.0;
+  int32_t D = 0;
+  int64_t S = 0;
+};
+DeviceScratch g_dev[kMaxDevices];
+
+// Fills the (cos, sin) table: angle p * theta^(-2i/D) in fp64, rounded to fp32.
+__global__ void __launch_bounds__(kThreads) fill_cos_sin(float2* cs, int64_t S, int32_t D, double theta) {
+  const int64_t half = D / 2;
+  const int64_t n = S * half;
+  for (int64_t k = (int64_t)blockIdx.x * kThreads + threadIdx.x; k < n; k += (int64_t)gridDim.x * kThreads) {
+    const int64_t p = k / half;
+    const int64_t i = k - p * half;
+    const double ang = (double)p * pow(theta, -2.0 * (double)i / (double)D);
+    double s, c;
+    sincos(ang, &s, &c);
+    cs[k] = make_float2((float)c, (float)s);
+  }
+}
+
+__global__ void clear_word(uint32_t* w) { *w = 0u; }
+
+}  // namespace
+}  // namespace trident
+
+using namespace trident;
+
+extern "C" __attribute__((visibility("default"))) int32_t trident_rope_kv_noalloc(
+    const trident_args* args, void* stream, uint32_t* out_status) {
+  RopeParams p;
+  int32_t dtype = 0;
+  bool qknorm = false;
+  int32_t st = prepare_rope_args(args, &p, &dtype, &qknorm);
+  if (st != TRIDENT_OK) return st;
+  const int dev = args->t[0].device;
+  if (dev >= kMaxDevices) return internal_fail(TRIDENT_ERR_INVALID, "device ordinal too large");
+  int cur = -1;
+  if (cudaGetDevice(&cur) != cudaSuccess || cur != dev)
+    return internal_fail(TRIDENT_ERR_INVALID, "the tensors' device must be the current device");
+  if (p.S * (p.D / 2) > kMaxPairs)
+    return internal_fail(TRIDENT_ERR_INVALID,
+                         "S * D/2 exceeds the static scratch maximum of 524288 (cos, sin) pairs");
+  KernelEntry ke;
+  const char* why = "";
+  if (!rope_kernel(dtype, TRIDENT_VARIANT_VECTOR, p.D, qknorm, &ke, &why))
+    return internal_fail(TRIDENT_ERR_INVALID, why);
+
+  // one-time set-up on this device: the device address of the static array
+  DeviceScratch& ds = g_dev[dev];
+  std::call_once(ds.once, [&] {
+    void* a = nullptr;
+    ds.setup_error = cudaGetSymbolAddress(&a, g_scratch);
+    ds.addr = static_cast<unsigned char*>(a);
+  });
+  if (ds.setup_error != cudaSuccess || !ds.addr)
+    return internal_fail(TRIDENT_ERR_CUDA, "cudaGetSymbolAddress of the scratch array failed");
+
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  uint32_t* status = reinterpret_cast<uint32_t*>(ds.addr);
+  float2* table = reinterpret_cast<float2*>(ds.addr + kTableOffset);
+  {
+    std::lock_guard<std::mutex> lk(ds.mu);
+    clear_word<<<1, 1, 0, s>>>(status);
+    if (!(ds.theta == args->rope_theta && ds.D == p.D && ds.S == p.S)) {
+      const int64_t n = p.S * (p.D / 2);
+      const int64_t blocks = (n + kThreads - 1) / kThreads;
+      fill_cos_sin<<<(unsigned)(blocks < 4096 ? blocks : 4096), kThreads, 0, s>>>(table, p.S, p.D,
+                                                                                 args->rope_theta);
+      ds.theta = args->rope_theta;
+      ds.D = p.D;
+      ds.S = p.S;
+    }
+  }
+  p.cs = table;
+  p.err = status;
+  const int64_t upb = rope_units_per_block(p.D, 2);
+  const int64_t blocks = (p.T * p.NH + upb - 1) / upb;
+  void* kargs[1] = {&p};
+  if (cudaLaunchKernel(ke.fn, dim3((unsigned)(blocks < 0x7fffffff ? blocks : 0x7fffffff)), dim3(kThreads),
+                       kargs, 0, s) != cudaSuccess)
+    return internal_fail(TRIDENT_ERR_CUDA, "RoPE launch failed");
+  if (out_status &&
+      cudaMemcpyAsync(out_status, status, sizeof(uint32_t), cudaMemcpyDeviceToHost, s) != cudaSuccess)
+    return internal_fail(TRIDENT_ERR_CUDA, "status copy failed");
+  if (cudaGetLastError() != cudaSuccess) return internal_fail(TRIDENT_ERR_CUDA, "launch error");
+  return TRIDENT_OK;
+}

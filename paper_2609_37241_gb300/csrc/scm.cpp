@@ -763,6 +763,38 @@ int32_t resolve_kernel(const trident_spec_desc& d, KernelEntry* ke) {
 
 }  // namespace
 
+// ====================================================================== internal
+int32_t trident::prepare_rope_args(const void* args_ptr, RopeParams* p, int32_t* dtype, bool* qknorm) {
+  const trident_args* a = static_cast<const trident_args*>(args_ptr);
+  const OpInfo* oi = nullptr;
+  int32_t st = validate(a, &oi);
+  if (st != TRIDENT_OK) return st;
+  if (a->op != TRIDENT_OP_ROPE_KV && a->op != TRIDENT_OP_QKNORM_ROPE_KV)
+    return fail(TRIDENT_ERR_INVALID, "op %d is not a RoPE op", a->op);
+  Sig s;
+  compute_sig(a, *oi, &s);
+  if (s.device == kMixed || s.device < 0) return fail(TRIDENT_ERR_INVALID, "tensors must share one CUDA device");
+  if (s.act_dtype != TRIDENT_BF16 && s.act_dtype != TRIDENT_FP16)
+    return fail(TRIDENT_ERR_INVALID, "activations must all be bf16 or all fp16");
+  if (!s.aux_dtype_ok) return fail(TRIDENT_ERR_INVALID, "gamma must be fp32 and pos int32");
+  if (!s.ranks_ok || !s.shapes_ok) return fail(TRIDENT_ERR_INVALID, "inconsistent ranks or shapes");
+  if (s.T < 1) return fail(TRIDENT_ERR_INVALID, "no tokens");
+  if (s.layout < 0 || !s.aux_layout_ok) return fail(TRIDENT_ERR_INVALID, "unsupported layout");
+  if (!aligned16(a, *oi)) return fail(TRIDENT_ERR_INVALID, "tensors must be 16-byte aligned");
+  if (!(a->rope_theta > 0.0 && std::isfinite(a->rope_theta)))
+    return fail(TRIDENT_ERR_INVALID, "rope_theta must be positive");
+  st = check_overlap(a, *oi);
+  if (st != TRIDENT_OK) return st;
+  Version v;
+  std::memset(&v, 0, sizeof(v));
+  pack_rope(a, 0, a->op == TRIDENT_OP_QKNORM_ROPE_KV ? 6 : -1, v, nullptr, p);
+  *dtype = s.act_dtype;
+  *qknorm = a->op == TRIDENT_OP_QKNORM_ROPE_KV;
+  return TRIDENT_OK;
+}
+
+int32_t trident::internal_fail(int32_t status, const char* msg) { return fail(status, "%s", msg); }
+
 // ====================================================================== C ABI
 TRIDENT_API int32_t trident_abi_version(void) { return TRIDENT_ABI_VERSION; }
 

@@ -81,6 +81,7 @@ def lib():
             "trident_scm_host_times": (c_i32, [c_vp, P(c_u32), c_i32, P(c_i32)]),
             "trident_scm_device_status": (c_i32, [c_vp, c_vp, P(c_u32), c_i32]),
             "trident_scm_destroy": (None, [c_vp]),
+            "trident_rope_kv_noalloc": (c_i32, [P(trident_args), c_vp, P(c_u32)]),
             "trident_scm_last_error": (ctypes.c_char_p, []),
             "trident_status_name": (ctypes.c_char_p, [c_i32]),
         }
@@ -162,6 +163,14 @@ def trident_scm_device_status(scm, stream=None, clear=True):
     bits = c_u32(0)
     st = lib().trident_scm_device_status(scm, stream, ctypes.byref(bits), 1 if clear else 0)
     return st, bits.value
+
+
+def trident_rope_kv_noalloc(args, stream=None):
+    """RoPE + KV append with no allocation (static scratch). Returns (status, status_word);
+    the status word is valid once the stream has been synchronised."""
+    word = c_u32(0)
+    st = lib().trident_rope_kv_noalloc(ctypes.byref(args), stream, ctypes.byref(word))
+    return st, word
 
 
 def trident_scm_destroy(scm):
