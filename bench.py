@@ -75,13 +75,14 @@ def chain_bytes_per_token(cfg, fused=True):
     H, Hq, Hkv, D, I = cfg["H"], cfg["Hq"], cfg["Hkv"], cfg["D"], cfg["I"]
     norm1 = 4 * H * 2                       # read h, r0; write x1, r1
     norm2 = (3 if fused else 4) * H * 2     # read attn_out (+ r1 unfused); write x2, r2
-    rope = (2 * Hq * D + 2 * Hkv * D + 2 * Hkv * D) * 2 + 4 + (D // 2) * 8  # q in/out, k in/out, v in/out, pos, cos/sin
+    rope = (2 * Hq * D + 2 * Hkv * D + 2 * Hkv * D) * 2 + 4  # q in/out, k in/out, v in/out, pos
     swiglu = 3 * I * 2
     return norm1 + norm2 + rope + swiglu
 
 
 def chain_bytes_per_launch(cfg, T, fused=True):
-    g = 2 * cfg["H"] * 4 + (2 * cfg["D"] * 4 if cfg.get("qknorm") else 0)
+    # norm weights (+ q/k norm weights) and the RoPE frequency table, once per launch
+    g = 2 * cfg["H"] * 4 + (2 * cfg["D"] * 4 if cfg.get("qknorm") else 0) + cfg["D"] * 4
     return T * chain_bytes_per_token(cfg, fused) + g
 
 

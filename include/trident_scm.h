@@ -238,8 +238,9 @@ int32_t trident_scm_create(const trident_scm_options* opt, trident_compile_hook 
 /* Appends one version (§3.5: versions are tried in creation order). The descriptor is
  * validated and copied; its kernel entry is resolved now, so the hit path does no
  * lookup (§3.3: the kernel entry is resolved when the specialisation is built). RoPE
- * versions build a cos/sin table for (theta, D, S) in fp64, rounded to fp32, shared by
- * versions with equal (theta, D, S). Readers see the new table atomically (copy-on-write);
+ * versions build a frequency table for (theta, D) -- theta^(-2i/D) in fp64, split into two
+ * fp32 -- shared by versions with equal (theta, D); the kernels form cos and sin of the
+ * angle from it. Readers see the new table atomically (copy-on-write);
  * calls already running keep the table they loaded. May be called from a hook.
  * *out_index (may be NULL) receives the new version's index.
  * Errors: ERR_INVALID (descriptor), ERR_CAPACITY (table full), ERR_CUDA. */
@@ -295,13 +296,13 @@ int32_t trident_scm_device_status(trident_scm_t* scm, void* stream, uint32_t* ou
  * library. There is no SCM handle and no guard table: the call validates the tuple,
  * requires what the vector kernel needs (bf16 or fp16, D in {64, 128, 256}, 16-byte
  * aligned tensors, dense caches, tensors on the current device) and launches on `stream`.
- * Its scratch -- the status word and the (cos, sin) table -- lives in one static device
- * array of 256 bytes + 4 MiB that every GPU loading the library holds until exit; S * D/2
- * above 524288 (cos, sin) pairs is rejected with ERR_INVALID. The first call on a device
- * looks up the array's device address (cudaGetSymbolAddress), so make that first call
- * before any stream capture. Every call shares the array, which keeps the last call's
- * table: the table is rebuilt on the device when (theta, D, S) changes, and the status
- * word is cleared at the start of each call. Calls that overlap on the GPU (other
+ * Its scratch -- the status word and the RoPE frequency table -- lives in one static
+ * device array of 256 + 1024 bytes that every GPU loading the library holds until exit;
+ * a head size above 256 (more than 128 frequency pairs) is rejected with ERR_INVALID.
+ * The first call on a device looks up the array's device address (cudaGetSymbolAddress),
+ * so make that first call before any stream capture. Every call shares the array, which
+ * keeps the last call's table: the table is rebuilt on the device when (theta, D)
+ * changes, and the status word is cleared at the start of each call. Calls that overlap on the GPU (other
  * streams, other host threads) race on the array. *out_status (may be NULL) receives the
  * status word (TRIDENT_DEVERR_* bits) by an asynchronous copy on `stream`: read it after
  * synchronising the stream. Errors: ERR_INVALID, ERR_CUDA. */

@@ -27,31 +27,104 @@ __global__ void __launch_bounds__(kThreads) chain_kernel(const ChainParams c) {
   const int tid = threadIdx.x;
   const int b = blockIdx.x;
   if (b < c.nA) {
-    __shared__ float red[2][kThreads / 32];
+    // Both norms of token b. The second residual sum s2 = attn_out + round(s1) is
+    // elementwise, so both sums of squares are formed before any reduction and reduced
+    // together: one barrier. s1 and s2 are recomputed from the packed inputs afterwards
+    // rather than kept, which keeps the register count (and occupancy) of the kernel.
+    __shared__ float2 red[kThreads / 32];
     const int64_t row = b;
     const AddNormParams& n1 = c.n1;
     const AddNormParams& n2 = c.n2;
-    AddNormRegs<DT, VPT> A, B;
-    // every load of both norms is issued before the first reduction
-    A.load(row_ptr(n1.x, row, n1.x_rs, EB), row_ptr(n1.r, row, n1.r_rs, EB), n1.gamma, tid);
-    B.load_x_gamma(row_ptr(n2.x, row, n2.x_rs, EB), n2.gamma, tid);
-    float s[VPT][VE];
-    float ss = A.residual(row_ptr(n1.r_out, row, n1.ro_rs, EB), tid, s);
-    float tot = block_sum(ss, red[0]);
-    A.normalize(row_ptr(n1.y, row, n1.y_rs, EB), tid, s, rsqrtf(tot * n1.inv_H + n1.eps));
-    // the second residual input is r1 as stored (rounded), taken from registers
+    uint4 hv[VPT], rv[VPT], av[VPT];
+    float ga[VPT][VE], gm[VPT][VE];
+    const uint4* hp = reinterpret_cast<const uint4*>(row_ptr(n1.x, row, n1.x_rs, EB));
+    const uint4* rp = reinterpret_cast<const uint4*>(row_ptr(n1.r, row, n1.r_rs, EB));
+    const uint4* ap = reinterpret_cast<const uint4*>(row_ptr(n2.x, row, n2.x_rs, EB));
 #pragma unroll
-    for (int v = 0; v < VPT; ++v) B.rv[v] = A.rv[v];
-    ss = B.residual(row_ptr(n2.r_out, row, n2.ro_rs, EB), tid, s);
-    tot = block_sum(ss, red[1]);
-    B.normalize(row_ptr(n2.y, row, n2.y_rs, EB), tid, s, rsqrtf(tot * n2.inv_H + n2.eps));
+    for (int v = 0; v < VPT; ++v) {
+      const int64_t vi = (int64_t)v * kThreads + tid;
+      hv[v] = ldg16(hp + vi);
+      rv[v] = ldg16(rp + vi);
+      av[v] = ldg16(ap + vi);
+#pragma unroll
+      for (int q = 0; q < VE / 4; ++q) {
+        const float4 g1 = ldg_f4(n1.gamma + vi * VE + 4 * q);
+        const float4 g2 = ldg_f4(n2.gamma + vi * VE + 4 * q);
+        ga[v][4 * q] = g1.x; ga[v][4 * q + 1] = g1.y; ga[v][4 * q + 2] = g1.z; ga[v][4 * q + 3] = g1.w;
+        gm[v][4 * q] = g2.x; gm[v][4 * q + 1] = g2.y; gm[v][4 * q + 2] = g2.z; gm[v][4 * q + 3] = g2.w;
+      }
+    }
+    uint4* r1p = reinterpret_cast<uint4*>(row_ptr(n1.r_out, row, n1.ro_rs, EB));
+    uint4* r2p = reinterpret_cast<uint4*>(row_ptr(n2.r_out, row, n2.ro_rs, EB));
+    float ss1 = 0.f, ss2 = 0.f;
+#pragma unroll
+    for (int v = 0; v < VPT; ++v) {
+      const int64_t vi = (int64_t)v * kThreads + tid;
+      float hf[VE], rf[VE], af[VE], s1[VE], s2[VE];
+      unpack<DT>(hv[v], hf);
+      unpack<DT>(rv[v], rf);
+      unpack<DT>(av[v], af);
+#pragma unroll
+      for (int e = 0; e < VE; ++e) {
+        s1[e] = hf[e] + rf[e];
+        ss1 = fmaf(s1[e], s1[e], ss1);
+      }
+      const uint4 r1 = pack<DT>(s1);
+      float r1f[VE];
+      unpack<DT>(r1, r1f);
+#pragma unroll
+      for (int e = 0; e < VE; ++e) {
+        s2[e] = af[e] + r1f[e];
+        ss2 = fmaf(s2[e], s2[e], ss2);
+      }
+      st16(r1p + vi, r1);              // r1, then r2: in place (r2 = r1) keeps r2
+      st16(r2p + vi, pack<DT>(s2));
+    }
+    float2 part = make_float2(ss1, ss2);
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      part.x += __shfl_xor_sync(0xffffffffu, part.x, o);
+      part.y += __shfl_xor_sync(0xffffffffu, part.y, o);
+    }
+    if ((tid & 31) == 0) red[tid >> 5] = part;
+    __syncthreads();
+    float2 tot = make_float2(0.f, 0.f);
+#pragma unroll
+    for (int i = 0; i < kThreads / 32; ++i) {
+      tot.x += red[i].x;
+      tot.y += red[i].y;
+    }
+    const float inv1 = rsqrtf(tot.x * n1.inv_H + n1.eps);
+    const float inv2 = rsqrtf(tot.y * n2.inv_H + n2.eps);
+    uint4* x1p = reinterpret_cast<uint4*>(row_ptr(n1.y, row, n1.y_rs, EB));
+    uint4* x2p = reinterpret_cast<uint4*>(row_ptr(n2.y, row, n2.y_rs, EB));
+#pragma unroll
+    for (int v = 0; v < VPT; ++v) {
+      const int64_t vi = (int64_t)v * kThreads + tid;
+      float hf[VE], rf[VE], af[VE], s1[VE], y1[VE], y2[VE];
+      unpack<DT>(hv[v], hf);
+      unpack<DT>(rv[v], rf);
+      unpack<DT>(av[v], af);
+#pragma unroll
+      for (int e = 0; e < VE; ++e) s1[e] = hf[e] + rf[e];
+      float r1f[VE];
+      unpack<DT>(pack<DT>(s1), r1f);
+#pragma unroll
+      for (int e = 0; e < VE; ++e) {
+        y1[e] = s1[e] * inv1 * ga[v][e];
+        y2[e] = (af[e] + r1f[e]) * inv2 * gm[v][e];
+      }
+      st16(x1p + vi, pack<DT>(y1));
+      st16(x2p + vi, pack<DT>(y2));
+    }
   } else if (b < c.nA + c.nB) {
     constexpr int LPH = D / VE;
     constexpr int UPB = kThreads / LPH;
     const int64_t unit = (int64_t)(b - c.nA) * UPB + tid / LPH;
     if (unit < c.rope.T * c.rope.NH) rope_head_row<DT, D, QKNORM>(c.rope, unit, tid % LPH);
   } else {
-    const int tile = b - c.nA - c.nB;
+    const int64_t tile = b - c.nA - c.nB;
+    if (tile >= c.sw_tiles) return;
     const int64_t row = tile / c.sw_tiles_per_row;
     const int64_t col_tile = tile - row * c.sw_tiles_per_row;
     swiglu_tile<DT, kChainSwigluUnroll>(c.sw, row, col_tile * kChainSwigluUnroll * kThreads, tid);

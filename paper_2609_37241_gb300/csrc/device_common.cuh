@@ -163,20 +163,6 @@ struct AddNormRegs {
       }
     }
   }
-  // Loads only x and gamma; the residual is given in registers (already rounded).
-  __device__ __forceinline__ void load_x_gamma(const void* x_row, const float* gamma, int tid) {
-#pragma unroll
-    for (int v = 0; v < VPT; ++v) {
-      const int64_t vi = (int64_t)v * kThreads + tid;
-      xv[v] = ldg16(reinterpret_cast<const uint4*>(x_row) + vi);
-#pragma unroll
-      for (int q = 0; q < VE / 4; ++q) {
-        float4 gg = ldg_f4(gamma + vi * VE + 4 * q);
-        g[v][4 * q] = gg.x; g[v][4 * q + 1] = gg.y; g[v][4 * q + 2] = gg.z; g[v][4 * q + 3] = gg.w;
-      }
-    }
-  }
-
   // s = x + r (fp32); stores round(s) to r_out (and leaves it in rv); returns sum(s^2)
   // of this thread; s is left in `s`.
   __device__ __forceinline__ float residual(void* ro_row, int tid, float (&s)[VPT][VE]) {
@@ -209,58 +195,85 @@ struct AddNormRegs {
   }
 };
 
+// ---------------------------------------------------------------- RoPE angles
+// sin and cos of the angle pos * f, with f = fhi + flo (a double-float split of
+// theta^(-2i/D) made in fp64 on the host). The product is kept as ah + al (al holds the
+// exact rounding error of pos * fhi, from one fma, plus pos * flo); ah is reduced modulo
+// 2 pi with the Cody-Waite method (Cody and Waite, "Software Manual for the Elementary
+// Functions", 1980) using 2 pi = A + B + C, A with 12 significant bits so that k * A is
+// exact for k < 4096, i.e. angles up to about 25700 rad; the reduced angle, within about
+// [-pi, pi], goes to the hardware sine/cosine (absolute error about 2^-21).
+constexpr float kInv2Pi = 0.159154936671257019f;     // 1 / (2 pi), rounded to fp32
+constexpr float k2PiA = 6.283203125f;                // 2 pi to 12 significant bits (3217/512)
+constexpr float k2PiB = -1.78178197529632598e-05f;   // fp32(2 pi - A)
+constexpr float k2PiC = -6.60559822986128669e-13f;   // fp32(2 pi - A - B)
+
+__device__ __forceinline__ void rope_sincos(float pos, float fhi, float flo, float* s, float* c) {
+  const float ah = pos * fhi;
+  const float al = fmaf(pos, fhi, -ah) + pos * flo;
+  const float k = rintf(ah * kInv2Pi);
+  float r = fmaf(-k, k2PiA, ah);
+  r = fmaf(-k, k2PiB, r);
+  r = fmaf(-k, k2PiC, r);
+  __sincosf(r + al, s, c);
+}
+
 // ---------------------------------------------------------------- RoPE head-row
 // One head-row (token t, head hh) handled by LPH = D / VE consecutive lanes, each lane
 // owning VE consecutive elements. Rotate-half pairs element i with i + D/2, i.e. lane
 // l with lane l ^ (LPH/2). hh < Hq: q head (rotated in place); hh < Hq + Hkv: k head
-// (rotated into k_cache); else v head (copied into v_cache).
+// (rotated into k_cache); else v head (copied into v_cache). Every load -- the row, the
+// position, the lane's frequencies and norm weights -- is issued before any of them is
+// used, so a head-row costs one memory round trip.
 template <int DT, int D, bool QKNORM>
 __device__ __forceinline__ void rope_head_row(const RopeParams& p, int64_t unit, int lane) {
   constexpr int VE = Act<DT>::VE;
   constexpr int LPH = D / VE;
   constexpr int HALF = LPH / 2;
+  constexpr int EB = Act<DT>::BYTES;
   static_assert(LPH >= 2 && LPH <= 32 && (LPH & (LPH - 1)) == 0, "head size");
   const unsigned group_mask =
       (LPH == 32) ? 0xffffffffu : (((1u << LPH) - 1u) << ((threadIdx.x & 31) & ~(LPH - 1)));
 
   const int64_t t = unit / p.NH;
   const int hh = (int)(unit - t * p.NH);
+  const bool is_v = hh >= p.Hq + p.Hkv;
+  const bool is_q = hh < p.Hq;
+  const int h = is_q ? hh : (is_v ? hh - p.Hq - p.Hkv : hh - p.Hq);
+  const char* src = is_q ? row_ptr(p.q, t, p.q_rs, EB) : is_v ? row_ptr(p.v, t, p.v_rs, EB)
+                                                             : row_ptr(p.k, t, p.k_rs, EB);
+  src += ((int64_t)h * D + lane * VE) * EB;
+  const uint4 raw = is_q ? ld16(src) : ldg16(src);
   const int32_t pos = __ldg(p.pos + t);
+  float fq[2 * VE];  // (hi, lo) of the lane's VE frequencies i = (lane % HALF) * VE + e
+  float gg[VE];
+  if (!is_v) {
+    const float* fr = reinterpret_cast<const float*>(p.inv_freq) + 2 * (lane % HALF) * VE;
+#pragma unroll
+    for (int q = 0; q < VE / 2; ++q) {
+      const float4 f4 = ldg_f4(fr + 4 * q);
+      fq[4 * q] = f4.x; fq[4 * q + 1] = f4.y; fq[4 * q + 2] = f4.z; fq[4 * q + 3] = f4.w;
+    }
+    if (QKNORM) {
+      const float* gam = (is_q ? p.gamma_q : p.gamma_k) + lane * VE;
+#pragma unroll
+      for (int q = 0; q < VE / 4; ++q) {
+        const float4 g4 = ldg_f4(gam + 4 * q);
+        gg[4 * q] = g4.x; gg[4 * q + 1] = g4.y; gg[4 * q + 2] = g4.z; gg[4 * q + 3] = g4.w;
+      }
+    }
+  }
   if (pos < 0 || (int64_t)pos >= p.S) {
     if (lane == 0) atomicOr(p.err, kErrPos);
     return;
   }
-  constexpr int EB = Act<DT>::BYTES;
-  if (hh >= p.Hq + p.Hkv) {  // v: bit copy into the cache
-    const int h = hh - p.Hq - p.Hkv;
-    const char* src = row_ptr(p.v, t, p.v_rs, EB) + ((int64_t)h * D + lane * VE) * EB;
-    char* dst = reinterpret_cast<char*>(p.v_cache) + (((int64_t)h * p.S + pos) * D + lane * VE) * EB;
-    st16(dst, ldg16(src));
+  if (is_v) {  // bit copy into the cache
+    st16(reinterpret_cast<char*>(p.v_cache) + (((int64_t)h * p.S + pos) * D + lane * VE) * EB, raw);
     return;
   }
-  const bool is_q = hh < p.Hq;
-  const int h = is_q ? hh : hh - p.Hq;
-  const char* src = is_q ? row_ptr(p.q, t, p.q_rs, EB) + ((int64_t)h * D + lane * VE) * EB
-                         : row_ptr(p.k, t, p.k_rs, EB) + ((int64_t)h * D + lane * VE) * EB;
   float x[VE];
-  unpack<DT>(is_q ? ld16(src) : ldg16(src), x);
-  // (cos, sin) of the VE frequencies i = (lane % HALF) * VE + e
-  const float* csrow = reinterpret_cast<const float*>(p.cs + (int64_t)pos * (D / 2)) +
-                       2 * (lane % HALF) * VE;
-  float cs[2 * VE];
-#pragma unroll
-  for (int q = 0; q < VE / 2; ++q) {
-    float4 c4 = ldg_f4(csrow + 4 * q);
-    cs[4 * q] = c4.x; cs[4 * q + 1] = c4.y; cs[4 * q + 2] = c4.z; cs[4 * q + 3] = c4.w;
-  }
+  unpack<DT>(raw, x);
   if (QKNORM) {
-    const float* gam = (is_q ? p.gamma_q : p.gamma_k) + lane * VE;
-    float gg[VE];
-#pragma unroll
-    for (int q = 0; q < VE / 4; ++q) {
-      float4 g4 = ldg_f4(gam + 4 * q);
-      gg[4 * q] = g4.x; gg[4 * q + 1] = g4.y; gg[4 * q + 2] = g4.z; gg[4 * q + 3] = g4.w;
-    }
     float ss = 0.f;
 #pragma unroll
     for (int e = 0; e < VE; ++e) ss = fmaf(x[e], x[e], ss);
@@ -274,12 +287,14 @@ __device__ __forceinline__ void rope_head_row(const RopeParams& p, int64_t unit,
 #pragma unroll
   for (int e = 0; e < VE; ++e) other[e] = __shfl_xor_sync(group_mask, x[e], HALF, LPH);
   const bool low = lane < HALF;
+  const float fpos = (float)pos;
   float y[VE];
 #pragma unroll
   for (int e = 0; e < VE; ++e) {
-    const float c = cs[2 * e], s = cs[2 * e + 1];
+    float sn, cs;
+    rope_sincos(fpos, fq[2 * e], fq[2 * e + 1], &sn, &cs);
     // low half: x_i c - x_{i+D/2} s;  high half: x_{i+D/2} c + x_i s
-    y[e] = low ? fmaf(x[e], c, -other[e] * s) : fmaf(x[e], c, other[e] * s);
+    y[e] = low ? fmaf(x[e], cs, -other[e] * sn) : fmaf(x[e], cs, other[e] * sn);
   }
   if (is_q) {
     st16(row_ptr(p.q, t, p.q_rs, EB) + ((int64_t)h * D + lane * VE) * EB, pack<DT>(y));

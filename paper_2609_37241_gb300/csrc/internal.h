@@ -27,8 +27,8 @@ struct AddNormParams {
 };
 
 // RoPE on q/k (optionally after per-head RMSNorm) plus KV-cache append.
-// q/k/v rows: token stride *_rs, head stride D, element stride 1.
-// cs: [S][D/2] pairs (cos, sin) in fp32. Caches dense [Hkv][S][D].
+// q/k/v rows: token stride *_rs, head stride D, element stride 1. Caches dense [Hkv][S][D].
+// inv_freq: [D/2] pairs (hi, lo), theta^(-2i/D) = hi + lo, split from fp64 on the host.
 struct RopeParams {
   void* q;
   const void* k;
@@ -38,7 +38,7 @@ struct RopeParams {
   void* v_cache;
   const float* gamma_q;
   const float* gamma_k;
-  const float2* cs;
+  const float2* inv_freq;
   uint32_t* err;
   int64_t T, S;
   int64_t q_rs, k_rs, v_rs;
@@ -55,14 +55,15 @@ struct SwigluParams {
   int64_t g_rs, u_rs, o_rs;
 };
 
-// One decoder layer's chain in one launch. Blocks [0, nA) run the two add+RMSNorm
-// steps of one token each, [nA, nA+nB) the RoPE/KV head-rows, the rest SwiGLU tiles.
+// One decoder layer's chain in one launch. Blocks [0, nA) run the two add+RMSNorm steps
+// of one token each, [nA, nA+nB) the RoPE/KV head-rows, the rest SwiGLU tiles.
 struct ChainParams {
   AddNormParams n1;   // h, r0 -> x1, r1
   AddNormParams n2;   // attn_out, (r1 from registers) -> x2, r2; n2.r is unused
   RopeParams rope;
   SwigluParams sw;
   int32_t nA, nB, nC, sw_tiles_per_row;
+  int64_t sw_tiles;  // T * sw_tiles_per_row (valid SwiGLU tiles)
 };
 
 // Kernel entry (host stub address) plus its launch shape rule.

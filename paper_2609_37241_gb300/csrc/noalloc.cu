@@ -1,20 +1,20 @@
 // noalloc.cu -- RoPE + KV-cache append that allocates nothing.
 //
 // The SCM path keeps two pieces of scratch memory in device allocations it makes itself:
-// the cos/sin table of a RoPE version (cudaMalloc at registration) and the device status
-// word (cudaMalloc at creation). Some callers cannot allocate device memory at all: a
-// serving engine that has handed every byte of HBM to its own pool, or code running where
-// a cudaMalloc would synchronise the device and stall other streams. For them,
+// the frequency table of a RoPE version (cudaMalloc at registration) and the device
+// status word (cudaMalloc at creation). Some callers cannot allocate device memory at
+// all: a serving engine that has handed every byte of HBM to its own pool, or code running
+// where a cudaMalloc would synchronise the device and stall other streams. For them,
 // trident_rope_kv_noalloc runs the same vector RoPE/KV kernel with its scratch in a
 // file-scope static device array of fixed size, so no call allocates anything (no
 // cudaMalloc, no cudaFree, no allocating library routine).
 //
-// Scratch layout (kScratchBytes = 256 + 4 MiB, held by every GPU that loads the library
-// until the process exits): bytes [0, 4) the status word, bytes [256, end) the
-// (cos, sin) table [S][D/2] in fp32, at most kMaxPairs = 524288 pairs (for example
-// S 8192 x D 128). The table is recomputed on the device (angles in fp64, rounded once to
-// fp32) only when (theta, D, S) differs from what the array held after the previous call
-// on that device; the status word is cleared at the start of every call.
+// Scratch layout (kScratchBytes = 256 + 1024 bytes, held by every GPU that loads the
+// library until the process exits): bytes [0, 4) the status word, bytes [256, end) the
+// frequency table, (hi, lo) fp32 pairs of theta^(-2i/D) for i < D/2, at most kMaxPairs =
+// 128 pairs (D <= 256). The table is recomputed on the device (fp64, split into two fp32)
+// only when (theta, D) differs from what the array held after the previous call on that
+// device; the status word is cleared at the start of every call.
 #include <cuda_runtime.h>
 
 #include <cmath>
@@ -27,7 +27,7 @@ namespace trident {
 namespace {
 
 constexpr size_t kTableOffset = 256;
-constexpr int64_t kMaxPairs = int64_t(1) << 19;
+constexpr int64_t kMaxPairs = 128;
 constexpr size_t kScratchBytes = kTableOffset + size_t(kMaxPairs) * sizeof(float2);
 constexpr int kMaxDevices = 64;
 
@@ -40,21 +40,16 @@ struct DeviceScratch {
   std::mutex mu;                  // guards the table key below
   double theta = 0.0;
   int32_t D = 0;
-  int64_t S = 0;
 };
 DeviceScratch g_dev[kMaxDevices];
 
-// Fills the (cos, sin) table: angle p * theta^(-2i/D) in fp64, rounded to fp32.
-__global__ void __launch_bounds__(kThreads) fill_cos_sin(float2* cs, int64_t S, int32_t D, double theta) {
-  const int64_t half = D / 2;
-  const int64_t n = S * half;
-  for (int64_t k = (int64_t)blockIdx.x * kThreads + threadIdx.x; k < n; k += (int64_t)gridDim.x * kThreads) {
-    const int64_t p = k / half;
-    const int64_t i = k - p * half;
-    const double ang = (double)p * pow(theta, -2.0 * (double)i / (double)D);
-    double s, c;
-    sincos(ang, &s, &c);
-    cs[k] = make_float2((float)c, (float)s);
+// Fills the frequency table: f_i = theta^(-2i/D) in fp64, stored as (fp32(f), fp32(f - hi)).
+__global__ void fill_inv_freq(float2* tab, int32_t D, double theta) {
+  const int i = threadIdx.x;
+  if (i < D / 2) {
+    const double f = pow(theta, -2.0 * (double)i / (double)D);
+    const float hi = (float)f;
+    tab[i] = make_float2(hi, (float)(f - (double)hi));
   }
 }
 
@@ -77,9 +72,9 @@ extern "C" __attribute__((visibility("default"))) int32_t trident_rope_kv_noallo
   int cur = -1;
   if (cudaGetDevice(&cur) != cudaSuccess || cur != dev)
     return internal_fail(TRIDENT_ERR_INVALID, "the tensors' device must be the current device");
-  if (p.S * (p.D / 2) > kMaxPairs)
+  if (p.D / 2 > kMaxPairs)
     return internal_fail(TRIDENT_ERR_INVALID,
-                         "S * D/2 exceeds the static scratch maximum of 524288 (cos, sin) pairs");
+                         "D/2 exceeds the static scratch maximum of 128 frequency pairs (D <= 256)");
   KernelEntry ke;
   const char* why = "";
   if (!rope_kernel(dtype, TRIDENT_VARIANT_VECTOR, p.D, qknorm, &ke, &why))
@@ -101,17 +96,13 @@ extern "C" __attribute__((visibility("default"))) int32_t trident_rope_kv_noallo
   {
     std::lock_guard<std::mutex> lk(ds.mu);
     clear_word<<<1, 1, 0, s>>>(status);
-    if (!(ds.theta == args->rope_theta && ds.D == p.D && ds.S == p.S)) {
-      const int64_t n = p.S * (p.D / 2);
-      const int64_t blocks = (n + kThreads - 1) / kThreads;
-      fill_cos_sin<<<(unsigned)(blocks < 4096 ? blocks : 4096), kThreads, 0, s>>>(table, p.S, p.D,
-                                                                                 args->rope_theta);
+    if (!(ds.theta == args->rope_theta && ds.D == p.D)) {
+      fill_inv_freq<<<1, (unsigned)kMaxPairs, 0, s>>>(table, p.D, args->rope_theta);
       ds.theta = args->rope_theta;
       ds.D = p.D;
-      ds.S = p.S;
     }
   }
-  p.cs = table;
+  p.inv_freq = table;
   p.err = status;
   const int64_t upb = rope_units_per_block(p.D, 2);
   const int64_t blocks = (p.T * p.NH + upb - 1) / upb;

@@ -5,8 +5,8 @@
 // D/VE lanes (16 lanes for D = 128 in bf16) so that a unit is one 256-byte coalesced
 // access, and exchanges the rotate-half partner with one xor-shuffle per element.
 // The generic kernel gives each unit one warp and scalar accesses (any alignment, any
-// even D). Both read (cos, sin) from the version's fp32 table [S][D/2], which the host
-// builds in fp64 when the version is registered.
+// even D). Both compute (cos, sin) of pos * theta^(-2i/D) in the kernel from the version's
+// double-float frequency table [D/2], which the host splits from fp64 at registration.
 #include "device_common.cuh"
 
 namespace trident {
@@ -63,16 +63,17 @@ __global__ void __launch_bounds__(kThreads) rope_generic_kernel(const RopeParams
       }
       inv = rsqrtf(warp_sum(ss) * p.inv_D + p.eps);
     }
-    const float2* cs = p.cs + (int64_t)pos * half;
     for (int i = lane; i < half; i += 32) {
       float lo = load_elem<DT>(src, so + i), hi = load_elem<DT>(src, so + i + half);
       if (QKNORM) {
         lo = lo * inv * gam[i];
         hi = hi * inv * gam[i + half];
       }
-      const float2 c = cs[i];
-      const float ylo = fmaf(lo, c.x, -hi * c.y);
-      const float yhi = fmaf(hi, c.x, lo * c.y);
+      const float2 f = p.inv_freq[i];
+      float sn, cs;
+      rope_sincos((float)pos, f.x, f.y, &sn, &cs);
+      const float ylo = fmaf(lo, cs, -hi * sn);
+      const float yhi = fmaf(hi, cs, lo * sn);
       if (is_q) {
         store_elem<DT>(p.q, so + i, ylo);
         store_elem<DT>(p.q, so + i + half, yhi);

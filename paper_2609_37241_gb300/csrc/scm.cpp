@@ -367,10 +367,9 @@ bool aligned16(const trident_args* a, const OpInfo& oi) {
 }
 
 // ------------------------------------------------------------------ versions
-struct RopeTable {
+struct RopeTable {  // theta^(-2i/D) = hi + lo for i < D/2, split from fp64
   double theta;
   int32_t D;
-  int64_t S;
   float2* dev;
 };
 
@@ -380,7 +379,7 @@ struct Version {
   bool rope;
   KernelEntry ke;
   CUfunction fn;
-  const float2* cs;
+  const float2* inv_freq;
 };
 
 }  // namespace
@@ -517,7 +516,7 @@ void pack_rope(const trident_args* a, int base, int gq, const Version& v, uint32
   p->k_cache = t[base + 4].data; p->v_cache = t[base + 5].data;
   p->gamma_q = gq >= 0 ? (const float*)t[gq].data : nullptr;
   p->gamma_k = gq >= 0 ? (const float*)t[gq + 1].data : nullptr;
-  p->cs = v.cs;
+  p->inv_freq = v.inv_freq;
   p->err = err;
   p->T = t[base].shape[0];
   p->S = t[base + 4].shape[1];
@@ -549,13 +548,14 @@ int32_t do_launch(trident_scm* scm, const Version& v, const trident_args* a, con
   cfg.blockDimX = kThreads; cfg.blockDimY = 1; cfg.blockDimZ = 1;
   cfg.gridDimY = 1; cfg.gridDimZ = 1;
   cfg.hStream = (CUstream)stream;
-  CUlaunchAttribute attr[1];
+  CUlaunchAttribute attr[2];
   std::memset(attr, 0, sizeof(attr));
+  cfg.attrs = attr;
+  cfg.numAttrs = 0;
   if (scm->opt.flags & TRIDENT_OPT_PDL) {
-    attr[0].id = CU_LAUNCH_ATTRIBUTE_PROGRAMMATIC_STREAM_SERIALIZATION;
-    attr[0].value.programmaticStreamSerializationAllowed = 1;
-    cfg.attrs = attr;
-    cfg.numAttrs = 1;
+    attr[cfg.numAttrs].id = CU_LAUNCH_ATTRIBUTE_PROGRAMMATIC_STREAM_SERIALIZATION;
+    attr[cfg.numAttrs].value.programmaticStreamSerializationAllowed = 1;
+    ++cfg.numAttrs;
   }
   union {
     AddNormParams an;
@@ -602,6 +602,7 @@ int32_t do_launch(trident_scm* scm, const Version& v, const trident_args* a, con
       if (nA + nB + nC > 0x7fffffff) return fail(TRIDENT_ERR_INVALID, "layer chain too large for one launch");
       c.nA = (int32_t)nA; c.nB = (int32_t)nB; c.nC = (int32_t)nC;
       c.sw_tiles_per_row = (int32_t)tiles;
+      c.sw_tiles = nC;
       cfg.gridDimX = (unsigned)(nA + nB + nC);
       break;
     }
@@ -670,27 +671,27 @@ int32_t on_device(trident_scm* scm, F fn) {
   return st;
 }
 
-// cos/sin table [S][D/2] for RoPE base theta: angles in fp64, rounded once to fp32.
-int32_t get_rope_table(trident_scm* scm, double theta, int32_t D, int64_t S, const float2** out) {
+// Frequency table of RoPE base theta: f_i = theta^(-2i/D) in fp64, stored as the fp32
+// pair (hi, lo) with hi = fp32(f_i) and lo = fp32(f_i - hi), so the kernel can form the
+// angle pos * f_i to about 2^-48 relative before reducing it.
+int32_t get_rope_table(trident_scm* scm, double theta, int32_t D, const float2** out) {
   for (const RopeTable& rt : scm->tables)
-    if (rt.theta == theta && rt.D == D && rt.S == S) { *out = rt.dev; return TRIDENT_OK; }
+    if (rt.theta == theta && rt.D == D) { *out = rt.dev; return TRIDENT_OK; }
   const int64_t half = D / 2;
-  std::vector<float2> host((size_t)(S * half));
-  std::vector<double> inv_freq((size_t)half);
-  for (int64_t i = 0; i < half; ++i) inv_freq[i] = std::pow(theta, -2.0 * (double)i / (double)D);
-  for (int64_t p = 0; p < S; ++p)
-    for (int64_t i = 0; i < half; ++i) {
-      const double ang = (double)p * inv_freq[i];
-      host[(size_t)(p * half + i)] = make_float2((float)std::cos(ang), (float)std::sin(ang));
-    }
+  std::vector<float2> host((size_t)half);
+  for (int64_t i = 0; i < half; ++i) {
+    const double f = std::pow(theta, -2.0 * (double)i / (double)D);
+    const float hi = (float)f;
+    host[(size_t)i] = make_float2(hi, (float)(f - (double)hi));
+  }
   float2* dev = nullptr;
   if (cudaMalloc(&dev, host.size() * sizeof(float2)) != cudaSuccess)
-    return fail(TRIDENT_ERR_CUDA, "cudaMalloc of the RoPE table failed");
+    return fail(TRIDENT_ERR_CUDA, "cudaMalloc of the RoPE frequency table failed");
   if (cudaMemcpy(dev, host.data(), host.size() * sizeof(float2), cudaMemcpyHostToDevice) != cudaSuccess) {
     cudaFree(dev);
-    return fail(TRIDENT_ERR_CUDA, "upload of the RoPE table failed");
+    return fail(TRIDENT_ERR_CUDA, "upload of the RoPE frequency table failed");
   }
-  scm->tables.push_back({theta, D, S, dev});
+  scm->tables.push_back({theta, D, dev});
   *out = dev;
   return TRIDENT_OK;
 }
@@ -894,8 +895,7 @@ TRIDENT_API int32_t trident_scm_register_spec(trident_scm_t* scm, const trident_
       if (v.rope) {
         const bool chain = desc->op == TRIDENT_OP_LAYER_CHAIN || desc->op == TRIDENT_OP_LAYER_CHAIN_QKNORM;
         const int32_t D = (int32_t)(chain ? desc->fixed[3] : desc->fixed[2]);
-        const int64_t S = chain ? desc->fixed[4] : desc->fixed[3];
-        return get_rope_table(scm, desc->rope_theta, D, S, &v.cs);
+        return get_rope_table(scm, desc->rope_theta, D, &v.inv_freq);
       }
       return TRIDENT_OK;
     });

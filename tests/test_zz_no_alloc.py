@@ -2,7 +2,7 @@
 
 Callers that cannot allocate device memory -- an engine whose HBM is all held by its own
 pool, or code where a cudaMalloc would synchronise the device -- use the entry point whose
-scratch (status word and cos/sin table) is a static device array. This file is collected
+scratch (status word and RoPE frequency table) is a static device array. This file is collected
 last on purpose. Two calls in a row, each compared with the existing entry point
 (trident_scm_invoke of an equivalent version) on identical inputs, within the parity
 tolerance of the other tests: the second call changes theta (the shared table is rebuilt)
@@ -88,9 +88,9 @@ def test_noalloc_two_calls_in_a_row_match_the_scm(S):
 
 
 def test_noalloc_rejects_sizes_beyond_its_scratch(S):
-    """S * D/2 above 524288 (cos, sin) pairs does not fit the static array: a clear error,
-    nothing launched."""
-    T, Hq, Hkv, D, Sl = 2, 2, 1, 128, 16384
+    """A head size above 256 needs more than the static array's 128 frequency pairs: a clear
+    error, nothing launched."""
+    T, Hq, Hkv, D, Sl = 2, 2, 1, 512, 64
     case = make_case(3, T, Hq, Hkv, D, Sl, False)
     ts = device_tensors(case, False)
     before = P.host_bits(ts[0], BF16)
