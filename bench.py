@@ -267,6 +267,17 @@ def assert_all_hit(scm, what):
     return st.hits
 
 
+def max_over_ranks(x, world, device="cpu"):
+    """The largest value of x over all ranks (the job's time is its slowest replica)."""
+    if world <= 1:
+        return float(x)
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([float(x)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
 def time_steps(c, fn, K, W):
     """Runs fn(i) for W warm-up then K timed steps; returns (us per step on the device
     clock, host us per step)."""
@@ -634,10 +645,7 @@ def run_ours(a):
     c.launches += K
     scm.close()
     del sets
-    t_local = torch.tensor([ms], dtype=torch.float64, device=c.dev)
-    if world > 1:
-        dist.all_reduce(t_local, op=dist.ReduceOp.MAX)
-    ms_max = float(t_local.item())
+    ms_max = max_over_ranks(ms, world, device=c.dev)
     us_step = ms_max * 1e3 / K
 
     extra = {}
