@@ -7,8 +7,8 @@
 // row-local: the block that produces row t of r1 keeps it in registers and runs the
 // second norm of row t itself. So no grid-wide barrier is needed; the launch is a
 // horizontal fusion where block ranges take different roles:
-//   [0, nA)            two add+RMSNorm steps of token b (the longest per-block work,
-//                      so these blocks are scheduled first)
+//   [0, nA)            two add+RMSNorm steps, one or two blocks per token (the longest
+//                      per-block work, so these blocks are scheduled first)
 //   [nA, nA + nB)      RoPE/KV head-rows, (256 / (D/8)) per block
 //   [nA + nB, end)     SwiGLU tiles of one row each
 // One launch replaces four, which is what matters at decode sizes, where each step
@@ -19,7 +19,7 @@ namespace trident {
 
 constexpr int kChainSwigluUnroll = 2;
 
-template <int DT, int VPT, int D, bool QKNORM>
+template <int DT, int VPT, int SPLIT, int D, bool QKNORM>
 __global__ void __launch_bounds__(kThreads) chain_kernel(const ChainParams c) {
   pdl_prologue();
   constexpr int EB = Act<DT>::BYTES;
@@ -27,16 +27,21 @@ __global__ void __launch_bounds__(kThreads) chain_kernel(const ChainParams c) {
   const int tid = threadIdx.x;
   const int b = blockIdx.x;
   if (b < c.nA) {
-    // Both norms of token b. The second residual sum s2 = attn_out + round(s1) is
+    // Both norms of one token. The second residual sum s2 = attn_out + round(s1) is
     // elementwise, so both sums of squares are formed before any reduction and reduced
-    // together: one barrier. s1 and s2 are recomputed from the packed inputs afterwards
-    // rather than kept, which keeps the register count (and occupancy) of the kernel.
+    // together: one barrier. With a_split = 2 two CTAs share a token: each reads the whole
+    // row (the sums need it) but loads only its half of both gamma vectors and writes only
+    // its half of the four outputs, so no SM carries the token's full 56 KB. s1 and s2 are
+    // recomputed from the packed inputs after the reduction rather than kept in registers.
     __shared__ float2 red[kThreads / 32];
-    const int64_t row = b;
+    constexpr int PP = VPT / SPLIT;  // vectors per thread this CTA writes
+    static_assert(VPT % SPLIT == 0, "split");
+    const int64_t row = b / SPLIT;
+    const int part = b - (int)row * SPLIT;
     const AddNormParams& n1 = c.n1;
     const AddNormParams& n2 = c.n2;
     uint4 hv[VPT], rv[VPT], av[VPT];
-    float ga[VPT][VE], gm[VPT][VE];
+    float ga[PP][VE], gm[PP][VE];
     const uint4* hp = reinterpret_cast<const uint4*>(row_ptr(n1.x, row, n1.x_rs, EB));
     const uint4* rp = reinterpret_cast<const uint4*>(row_ptr(n1.r, row, n1.r_rs, EB));
     const uint4* ap = reinterpret_cast<const uint4*>(row_ptr(n2.x, row, n2.x_rs, EB));
@@ -46,12 +51,16 @@ __global__ void __launch_bounds__(kThreads) chain_kernel(const ChainParams c) {
       hv[v] = ldg16(hp + vi);
       rv[v] = ldg16(rp + vi);
       av[v] = ldg16(ap + vi);
+      if (v / PP == part) {
 #pragma unroll
-      for (int q = 0; q < VE / 4; ++q) {
-        const float4 g1 = ldg_f4(n1.gamma + vi * VE + 4 * q);
-        const float4 g2 = ldg_f4(n2.gamma + vi * VE + 4 * q);
-        ga[v][4 * q] = g1.x; ga[v][4 * q + 1] = g1.y; ga[v][4 * q + 2] = g1.z; ga[v][4 * q + 3] = g1.w;
-        gm[v][4 * q] = g2.x; gm[v][4 * q + 1] = g2.y; gm[v][4 * q + 2] = g2.z; gm[v][4 * q + 3] = g2.w;
+        for (int q = 0; q < VE / 4; ++q) {
+          const float4 g1 = ldg_f4(n1.gamma + vi * VE + 4 * q);
+          const float4 g2 = ldg_f4(n2.gamma + vi * VE + 4 * q);
+          float* a = ga[v % PP];
+          float* m = gm[v % PP];
+          a[4 * q] = g1.x; a[4 * q + 1] = g1.y; a[4 * q + 2] = g1.z; a[4 * q + 3] = g1.w;
+          m[4 * q] = g2.x; m[4 * q + 1] = g2.y; m[4 * q + 2] = g2.z; m[4 * q + 3] = g2.w;
+        }
       }
     }
     uint4* r1p = reinterpret_cast<uint4*>(row_ptr(n1.r_out, row, n1.ro_rs, EB));
@@ -77,16 +86,18 @@ __global__ void __launch_bounds__(kThreads) chain_kernel(const ChainParams c) {
         s2[e] = af[e] + r1f[e];
         ss2 = fmaf(s2[e], s2[e], ss2);
       }
-      st16(r1p + vi, r1);              // r1, then r2: in place (r2 = r1) keeps r2
-      st16(r2p + vi, pack<DT>(s2));
+      if (v / PP == part) {
+        st16(r1p + vi, r1);              // r1, then r2: in place (r2 = r1) keeps r2
+        st16(r2p + vi, pack<DT>(s2));
+      }
     }
-    float2 part = make_float2(ss1, ss2);
+    float2 sums = make_float2(ss1, ss2);
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) {
-      part.x += __shfl_xor_sync(0xffffffffu, part.x, o);
-      part.y += __shfl_xor_sync(0xffffffffu, part.y, o);
+      sums.x += __shfl_xor_sync(0xffffffffu, sums.x, o);
+      sums.y += __shfl_xor_sync(0xffffffffu, sums.y, o);
     }
-    if ((tid & 31) == 0) red[tid >> 5] = part;
+    if ((tid & 31) == 0) red[tid >> 5] = sums;
     __syncthreads();
     float2 tot = make_float2(0.f, 0.f);
 #pragma unroll
@@ -100,6 +111,7 @@ __global__ void __launch_bounds__(kThreads) chain_kernel(const ChainParams c) {
     uint4* x2p = reinterpret_cast<uint4*>(row_ptr(n2.y, row, n2.y_rs, EB));
 #pragma unroll
     for (int v = 0; v < VPT; ++v) {
+      if (v / PP != part) continue;
       const int64_t vi = (int64_t)v * kThreads + tid;
       float hf[VE], rf[VE], af[VE], s1[VE], y1[VE], y2[VE];
       unpack<DT>(hv[v], hf);
@@ -111,8 +123,8 @@ __global__ void __launch_bounds__(kThreads) chain_kernel(const ChainParams c) {
       unpack<DT>(pack<DT>(s1), r1f);
 #pragma unroll
       for (int e = 0; e < VE; ++e) {
-        y1[e] = s1[e] * inv1 * ga[v][e];
-        y2[e] = (af[e] + r1f[e]) * inv2 * gm[v][e];
+        y1[e] = s1[e] * inv1 * ga[v % PP][e];
+        y2[e] = (af[e] + r1f[e]) * inv2 * gm[v % PP][e];
       }
       st16(x1p + vi, pack<DT>(y1));
       st16(x2p + vi, pack<DT>(y2));
@@ -131,11 +143,11 @@ __global__ void __launch_bounds__(kThreads) chain_kernel(const ChainParams c) {
   }
 }
 
-template <int DT, bool QK>
+template <int DT, int SPLIT, bool QK>
 static const void* pick(int64_t H) {
   constexpr int per = kThreads * Act<DT>::VE;
-  if (H == per * 2) return (const void*)chain_kernel<DT, 2, 128, QK>;
-  if (H == per * 4) return (const void*)chain_kernel<DT, 4, 128, QK>;
+  if (H == per * 2) return (const void*)chain_kernel<DT, 2, SPLIT, 128, QK>;
+  if (H == per * 4) return (const void*)chain_kernel<DT, 4, SPLIT, 128, QK>;
   return nullptr;
 }
 
@@ -146,8 +158,15 @@ bool chain_kernel(int32_t dtype, int64_t H, int32_t D, bool qknorm, KernelEntry*
   out->kind = KK_CHAIN;
   out->vec = 8;
   out->unroll = kChainSwigluUnroll;
-  if (dtype == DT_BF16) out->fn = qknorm ? pick<DT_BF16, true>(H) : pick<DT_BF16, false>(H);
-  else out->fn = qknorm ? pick<DT_FP16, true>(H) : pick<DT_FP16, false>(H);
+  // fn: two blocks per token for the norms; fn_inplace: one block per token (calls whose
+  // outputs overwrite inputs, and grids too large for one wave)
+  if (dtype == DT_BF16) {
+    out->fn = qknorm ? pick<DT_BF16, 2, true>(H) : pick<DT_BF16, 2, false>(H);
+    out->fn_inplace = qknorm ? pick<DT_BF16, 1, true>(H) : pick<DT_BF16, 1, false>(H);
+  } else {
+    out->fn = qknorm ? pick<DT_FP16, 2, true>(H) : pick<DT_FP16, 2, false>(H);
+    out->fn_inplace = qknorm ? pick<DT_FP16, 1, true>(H) : pick<DT_FP16, 1, false>(H);
+  }
   if (!out->fn) { *why = "layer chain supports H in {4096, 8192}"; return false; }
   return true;
 }

@@ -63,12 +63,14 @@ struct ChainParams {
   RopeParams rope;
   SwigluParams sw;
   int32_t nA, nB, nC, sw_tiles_per_row;
+  int32_t a_split;   // CTAs per token for the norms (2, or 1 for in-place calls)
   int64_t sw_tiles;  // T * sw_tiles_per_row (valid SwiGLU tiles)
 };
 
 // Kernel entry (host stub address) plus its launch shape rule.
 struct KernelEntry {
   const void* fn = nullptr;
+  const void* fn_inplace = nullptr;  // chain only: the entry for calls that write in place
   int32_t kind = 0;      // which grid rule the host applies (KernelKind)
   int32_t vec = 0;       // elements per vector (VE), or tile width for SwiGLU
   int32_t unroll = 1;    // vectors per thread per tile (SwiGLU, chain)

@@ -379,6 +379,8 @@ struct Version {
   bool rope;
   KernelEntry ke;
   CUfunction fn;
+  CUfunction fn_inplace;  // layer chain: one block per token when outputs alias inputs
+  int32_t wave_blocks;    // layer chain: blocks of `fn` resident at once on the whole GPU
   const float2* inv_freq;
 };
 
@@ -598,7 +600,15 @@ int32_t do_launch(trident_scm* scm, const Version& v, const trident_args* a, con
       const int64_t per = (int64_t)v.ke.unroll * kThreads * v.ke.vec;
       const int64_t tiles = (c.sw.I + per - 1) / per;
       const int64_t upb = rope_units_per_block(c.rope.D, 2);
-      const int64_t nA = s.T, nB = (s.T * c.rope.NH + upb - 1) / upb, nC = s.T * tiles;
+      // Two CTAs per token for the norms -- so no SM carries a whole token's norm traffic --
+      // while the grid still fits in one wave, and unless an output is written over an
+      // input the partner CTA still reads (in-place calls keep one CTA per token).
+      const trident_tensor* t = a->t;
+      const bool inplace = t[C_X1].data == t[C_H].data || t[C_R1].data == t[C_R0].data ||
+                           t[C_R2].data == t[C_R0].data || t[C_X2].data == t[C_AO].data;
+      const int64_t nB = (s.T * c.rope.NH + upb - 1) / upb, nC = s.T * tiles;
+      c.a_split = (!inplace && 2 * s.T + nB + nC <= v.wave_blocks) ? 2 : 1;
+      const int64_t nA = s.T * c.a_split;
       if (nA + nB + nC > 0x7fffffff) return fail(TRIDENT_ERR_INVALID, "layer chain too large for one launch");
       c.nA = (int32_t)nA; c.nB = (int32_t)nB; c.nC = (int32_t)nC;
       c.sw_tiles_per_row = (int32_t)tiles;
@@ -609,12 +619,15 @@ int32_t do_launch(trident_scm* scm, const Version& v, const trident_args* a, con
     default:
       return fail(TRIDENT_ERR_INVALID, "op");
   }
+  CUfunction fn = v.fn;
+  if ((op == TRIDENT_OP_LAYER_CHAIN || op == TRIDENT_OP_LAYER_CHAIN_QKNORM) && P.ch.a_split == 1)
+    fn = v.fn_inplace;
   CUcontext cur = nullptr;
   g_drv.ctx_get(&cur);
   const bool swap = cur != scm->ctx;
   if (swap && g_drv.ctx_push(scm->ctx) != CUDA_SUCCESS)
     return fail(TRIDENT_ERR_CUDA, "cannot make the SCM's context current");
-  const CUresult rc = g_drv.launch_ex(&cfg, v.fn, kp, nullptr);
+  const CUresult rc = g_drv.launch_ex(&cfg, fn, kp, nullptr);
   if (swap) {
     CUcontext dummy;
     g_drv.ctx_pop(&dummy);
@@ -892,6 +905,17 @@ TRIDENT_API int32_t trident_scm_register_spec(trident_scm_t* scm, const trident_
       if (cudaGetFuncBySymbol(&f, v.ke.fn) != cudaSuccess || !f)
         return fail(TRIDENT_ERR_CUDA, "cannot resolve the kernel entry");
       v.fn = reinterpret_cast<CUfunction>(f);
+      if (v.ke.fn_inplace) {
+        cudaFunction_t g = nullptr;
+        if (cudaGetFuncBySymbol(&g, v.ke.fn_inplace) != cudaSuccess || !g)
+          return fail(TRIDENT_ERR_CUDA, "cannot resolve the in-place kernel entry");
+        v.fn_inplace = reinterpret_cast<CUfunction>(g);
+        int per_sm = 0, sms = 0;
+        if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, v.ke.fn, kThreads, 0) != cudaSuccess ||
+            cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, scm->device) != cudaSuccess)
+          return fail(TRIDENT_ERR_CUDA, "occupancy query failed");
+        v.wave_blocks = per_sm * sms;
+      }
       if (v.rope) {
         const bool chain = desc->op == TRIDENT_OP_LAYER_CHAIN || desc->op == TRIDENT_OP_LAYER_CHAIN_QKNORM;
         const int32_t D = (int32_t)(chain ? desc->fixed[3] : desc->fixed[2]);
