@@ -163,7 +163,27 @@ class Ctx:
         self.stream = torch.cuda.current_stream()
         self.sp = ctypes.c_void_p(self.stream.cuda_stream)
         self.L = S.lib()
+        self.fc = S.fastcall()  # CPython fast-call shim of the binding (None: ctypes only)
         self.launches = 0
+
+    def invoker(self, scm):
+        """fn(args_struct_or_address) -> status: one trident_scm_invoke from Python."""
+        h, sp = scm.h.value, self.sp.value
+        if self.fc is not None:
+            inv = self.fc.invoke
+            return lambda addr: inv(h, addr, sp)
+        inv, hh, spp = self.L.trident_scm_invoke, scm.h, self.sp
+        P = ctypes.POINTER(self.S.trident_args)
+        return lambda addr: inv(hh, ctypes.cast(addr, P), spp, None)
+
+    def seq_invoker(self, scm):
+        h, sp = scm.h.value, self.sp.value
+        if self.fc is not None:
+            seq = self.fc.invoke_seq
+            return lambda addr, n: seq(h, addr, n, sp)
+        seq, hh, spp = self.L.trident_scm_invoke_seq, scm.h, self.sp
+        P = ctypes.POINTER(self.S.trident_args)
+        return lambda addr, n: seq(hh, ctypes.cast(addr, P), n, spp, None)
 
     def events(self):
         t = self.torch
@@ -304,12 +324,13 @@ def bench_layer(c, cfg, T, K, W, layers=1, min_bytes=2 * L2_BYTES):
     R = sets.R
     fused = [sets.fused_args(c, i, i % layers) for i in range(R)]
     unf = [(S.trident_args * 4)(*sets.unfused_args(c, i, i % layers)) for i in range(R)]
-    inv, seq = c.L.trident_scm_invoke, c.L.trident_scm_invoke_seq
+    inv, seq = c.invoker(scm), c.seq_invoker(scm)
     h, sp = scm.h, c.sp
-    fref = [ctypes.byref(a) for a in fused]
+    faddr = [ctypes.addressof(a) for a in fused]
+    uaddr = [ctypes.addressof(a) for a in unf]
     if layers == 1:
-        f_fused = lambda i: inv(h, fref[i % R], sp, None)
-        f_unf = lambda i: seq(h, unf[i % R], 4, sp, None)
+        f_fused = lambda i: inv(faddr[i % R])
+        f_unf = lambda i: seq(uaddr[i % R], 4)
         n_launch = (1, 4)
     else:  # one step = `layers` layers through one call
         groups = R // layers
@@ -317,8 +338,10 @@ def bench_layer(c, cfg, T, K, W, layers=1, min_bytes=2 * L2_BYTES):
         uarr = [(S.trident_args * (4 * layers))(*[a for l in range(layers) for a in
                                                    sets.unfused_args(c, g * layers + l, l)])
                 for g in range(groups)]
-        f_fused = lambda i: seq(h, farr[i % groups], layers, sp, None)
-        f_unf = lambda i: seq(h, uarr[i % groups], 4 * layers, sp, None)
+        fa = [ctypes.addressof(x) for x in farr]
+        ua = [ctypes.addressof(x) for x in uarr]
+        f_fused = lambda i: seq(fa[i % groups], layers)
+        f_unf = lambda i: seq(ua[i % groups], 4 * layers)
         n_launch = (layers, 4 * layers)
     st, sel = S.trident_scm_invoke(h, fused[0], c.sp.value)
     assert st == S.OK and sel in (0, 1), S.trident_scm_last_error()
@@ -329,7 +352,8 @@ def bench_layer(c, cfg, T, K, W, layers=1, min_bytes=2 * L2_BYTES):
     nat = min(K, R if layers == 1 else R)
     if layers == 1:
         arr = (S.trident_args * nat)(*fused[:nat])
-        nat_fn = lambda i: seq(h, arr, nat, sp, None)
+        arr_addr = ctypes.addressof(arr)
+        nat_fn = lambda i: seq(arr_addr, nat)
         nat_us, _ = time_steps(c, nat_fn, 4, 2)
         nat_us /= nat
         c.launches += 4 * nat
@@ -348,34 +372,66 @@ def bench_layer(c, cfg, T, K, W, layers=1, min_bytes=2 * L2_BYTES):
 
 
 def bench_e2e(c, cfg, T, K, W):
-    """End to end through the public API: per step, pinned host -> device copies of the
-    layer's inputs, one invoke, device -> host copies of its outputs."""
-    t, S = c.torch, c.S
-    sets = ChainSets(c, cfg, T, min_bytes=0, max_sets=1)
+    """End to end through the public API: per step, one pinned host -> device copy of the
+    layer's inputs (h, r0, attn_out, qkv, gate|up, pos laid out in one staging arena),
+    one invoke, one device -> host copy of its outputs (x1, x2, r2, o in one arena)."""
+    t, S, synth = c.torch, c.S, c.synth
+    H, Hq, Hkv, D, Sl, I = (cfg[k] for k in ("H", "Hq", "Hkv", "D", "S", "I"))
+    Wq = (Hq + 2 * Hkv) * D
+
+    def layout(parts):
+        offs, o = [], 0
+        for nbytes in parts:
+            offs.append(o)
+            o += (nbytes + 255) // 256 * 256
+        return offs, o
+
+    in_parts = [T * H * 2, T * H * 2, T * H * 2, T * Wq * 2, T * 2 * I * 2, T * 4]
+    out_parts = [T * H * 2, T * H * 2, T * H * 2, T * I * 2]
+    ioffs, itot = layout(in_parts)
+    ooffs, otot = layout(out_parts)
+    dev_in = t.empty(itot, dtype=t.uint8, device=c.dev)
+    dev_out = t.empty(otot, dtype=t.uint8, device=c.dev)
+    host_in = t.empty(itot, dtype=t.uint8, pin_memory=True)
+    host_out = t.empty(otot, dtype=t.uint8, pin_memory=True)
+    view = lambda buf, o, n, dt, shape: buf[o:o + n].view(dt).view(shape)
+    bf = t.bfloat16
+    h = view(dev_in, ioffs[0], in_parts[0], bf, (T, H))
+    r0 = view(dev_in, ioffs[1], in_parts[1], bf, (T, H))
+    ao = view(dev_in, ioffs[2], in_parts[2], bf, (T, H))
+    qkv = view(dev_in, ioffs[3], in_parts[3], bf, (T, Wq))
+    gu = view(dev_in, ioffs[4], in_parts[4], bf, (T, 2 * I))
+    pos = view(dev_in, ioffs[5], in_parts[5], t.int32, (T,))
+    for k, tv in enumerate((h, r0, ao, qkv, gu)):
+        tv.copy_(synth.act_device(tuple(tv.shape), S.BF16, 40 + k, c.dev))
+    pos.copy_(t.from_numpy(synth.positions(np.random.default_rng(1), T, Sl)).to(c.dev))
+    host_in.copy_(dev_in)
+    x1 = view(dev_out, ooffs[0], out_parts[0], bf, (T, H))
+    x2 = view(dev_out, ooffs[1], out_parts[1], bf, (T, H))
+    r2 = view(dev_out, ooffs[2], out_parts[2], bf, (T, H))
+    o = view(dev_out, ooffs[3], out_parts[3], bf, (T, I))
+    r1 = t.empty((T, H), dtype=bf, device=c.dev)
+    kc = t.zeros((Hkv, Sl, D), dtype=bf, device=c.dev)
+    vc = t.zeros((Hkv, Sl, D), dtype=bf, device=c.dev)
+    ga, gm = synth.gamma_device(H, 50, c.dev), synth.gamma_device(H, 51, c.dev)
+    ts = [h, r0, ga, x1, r1, qkv[:, :Hq * D].view(T, Hq, D), qkv[:, Hq * D:(Hq + Hkv) * D].view(T, Hkv, D),
+          qkv[:, (Hq + Hkv) * D:].view(T, Hkv, D), pos, kc, vc, ao, gm, x2, r2, gu[:, :I], gu[:, I:], o]
     scm = layer_scm(c, cfg)
-    a = sets.fused_args(c, 0)
-    pin = lambda x: t.empty(x.shape, dtype=x.dtype, pin_memory=True).copy_(x)
-    ins = [(sets.h[0], pin(sets.h[0])), (sets.r0[0], pin(sets.r0[0])), (sets.ao[0], pin(sets.ao[0])),
-           (sets.qkv[0], pin(sets.qkv[0])), (sets.gu[0], pin(sets.gu[0])), (sets.pos[0], pin(sets.pos[0]))]
-    outs = [(sets.x1[0], pin(sets.x1[0])), (sets.x2[0], pin(sets.x2[0])), (sets.r2[0], pin(sets.r2[0])),
-            (sets.o[0], pin(sets.o[0]))]
-    inv = c.L.trident_scm_invoke
-    ar = ctypes.byref(a)
+    a = S.make_args(S.OP_LAYER_CHAIN, ts, eps=cfg["eps"], rope_theta=cfg["theta"])
+    addr = ctypes.addressof(a)
+    inv = c.invoker(scm)
 
     def step(i):
-        for d, h in ins:
-            d.copy_(h, non_blocking=True)
-        inv(scm.h, ar, c.sp, None)
-        for d, h in outs:
-            h.copy_(d, non_blocking=True)
+        dev_in.copy_(host_in, non_blocking=True)
+        inv(addr)
+        host_out.copy_(dev_out, non_blocking=True)
 
     us, host_us = time_steps(c, step, K, W)
     assert_all_hit(scm, "e2e")
     c.launches += K
-    bi = sum(h.numel() * h.element_size() for _, h in ins)
-    bo = sum(h.numel() * h.element_size() for _, h in outs)
     scm.close()
-    return dict(value=round(us, 3), unit=UNIT, h2d_bytes_per_step=int(bi), d2h_bytes_per_step=int(bo))
+    return dict(value=round(us, 3), unit=UNIT, h2d_bytes_per_step=int(sum(in_parts)),
+                d2h_bytes_per_step=int(sum(out_parts)), copies_per_step=2)
 
 
 def bench_host_hit(c, n=1000):
@@ -404,6 +460,26 @@ def bench_host_hit(c, n=1000):
         inv(s.h, ar, c.sp, ctypes.byref(sel))
     h1 = time.perf_counter()
     t.cuda.synchronize()
+    fast_us = None
+    if c.fc is not None:
+        finv, hh, addr, sp = c.fc.invoke, s.h.value, ctypes.addressof(a), c.sp.value
+        f0 = time.perf_counter()
+        for _ in range(n):
+            finv(hh, addr, sp)
+        f1 = time.perf_counter()
+        t.cuda.synchronize()
+        fast_us = round((f1 - f0) * 1e6 / n, 3)
+        c.launches += n
+    # guards, validation and packing alone: the same table and call on a dry-run SCM
+    d = S.Scm(device=c.dev.index or 0, flags=S.OPT_TIMING | S.OPT_DRY_RUN)
+    for dt in (S.FP16, S.BF16):
+        for lay in ((S.LAYOUT_CONTIG, S.LAYOUT_ROWSTRIDED) if dt == S.FP16 else
+                    (S.LAYOUT_ROWSTRIDED, S.LAYOUT_CONTIG)):
+            d.register(S.make_spec(S.OP_ADD_RMSNORM, dt, [4096], 1, 1, layout=lay))
+    for _ in range(n + 50):
+        c.L.trident_scm_invoke(d.h, ar, c.sp, None)
+    dns = np.array(S.trident_scm_host_times(d.h, n)[1], np.float64)
+    d.close()
     st, ns = S.trident_scm_host_times(s.h, n)
     hits = S.trident_scm_spec_hits(s.h)[1]
     assert_all_hit(s, "host dispatch")
@@ -412,7 +488,8 @@ def bench_host_hit(c, n=1000):
     s.close()
     return dict(hits_on_bf16_contig=int(hits[3]), calls=n, selected=sel.value,
                 median_ns=float(np.median(ns)), p99_ns=float(np.percentile(ns, 99)),
-                min_ns=float(ns.min()), python_call_us=round((h1 - h0) * 1e6 / n, 3))
+                min_ns=float(ns.min()), guards_only_median_ns=float(np.median(dns)),
+                python_call_us_ctypes=round((h1 - h0) * 1e6 / n, 3), python_call_us_fastcall=fast_us)
 
 
 def bench_guard_stress(c, n_calls=None):
@@ -629,15 +706,15 @@ def run_ours(a):
     scm = layer_scm(c, cfg)
     R = sets.R
     fused_structs = [sets.fused_args(c, i) for i in range(R)]
-    fused = [ctypes.byref(x) for x in fused_structs]
-    inv = c.L.trident_scm_invoke
+    fused = [ctypes.addressof(x) for x in fused_structs]
+    inv = c.invoker(scm)
     for i in range(W):
-        inv(scm.h, fused[i % R], c.sp, None)
+        inv(fused[i % R])
     barrier()
     e0, e1 = c.events()
     e0.record(c.stream)
     for i in range(K):
-        inv(scm.h, fused[(W + i) % R], c.sp, None)
+        inv(fused[(W + i) % R])
     e1.record(c.stream)
     barrier()
     ms = e0.elapsed_time(e1)
@@ -702,7 +779,8 @@ def run_ours(a):
                                 l2="inputs rotated over %d sets (%.0f MB > 2x L2)" % (
                                     R, R * chain_bytes_per_token(cfg) * HEADLINE_T / 2 ** 20),
                                 parallelism="replicas" if world > 1 else "single GPU"),
-                    gpu_launches=headline_launches, gpu_launches_whole_run=c.launches)
+                    gpu_launches=headline_launches, gpu_launches_whole_run=c.launches,
+                    python_binding="fastcall" if c.fc is not None else "ctypes")
         line.update(extra)
         if cpu_us is not None:
             line["cpu_baseline"] = dict(value=round(cpu_us, 1), unit=UNIT, cores=1, kind="oracle",

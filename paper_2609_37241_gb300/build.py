@@ -61,7 +61,28 @@ def build(force=False, verbose=False, extra_flags=()):
     if force or jobs or _stale(LIB, objs):
         run([nvcc(), *ARCH, "-shared", "-o", LIB + ".tmp", *objs])
         os.replace(LIB + ".tmp", LIB)
+    build_fastcall(force, verbose)
     return LIB
+
+
+def build_fastcall(force=False, verbose=False):
+    """The CPython fast-call shim of the binding (linked against the library; built only
+    where the Python headers are installed -- the binding uses ctypes otherwise)."""
+    import sysconfig
+    inc = sysconfig.get_paths()["include"]
+    if not os.path.exists(os.path.join(inc, "Python.h")):
+        return None
+    src = os.path.join(CSRC, "fastcall.c")
+    out = os.path.join(PKG, "_fastcall" + sysconfig.get_config_var("EXT_SUFFIX"))
+    if not force and not _stale(out, [src, LIB, os.path.join(INC, "trident_scm.h")]):
+        return out
+    cmd = ["gcc", "-O2", "-shared", "-fPIC", "-I", inc, "-I", INC, src, "-o", out + ".tmp",
+           "-L", LIBDIR, "-ltrident_scm", "-Wl,-rpath,$ORIGIN/_lib"]
+    if verbose:
+        print(" ".join(cmd), file=sys.stderr)
+    subprocess.run(cmd, check=True)
+    os.replace(out + ".tmp", out)
+    return out
 
 
 if __name__ == "__main__":

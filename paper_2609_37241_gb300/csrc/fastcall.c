@@ -1,0 +1,51 @@
+/* fastcall.c -- CPython entry points for the per-call hot path of the Python binding.
+ *
+ * Argument marshalling only: each function converts Python ints (the SCM handle, the
+ * address of a trident_args array built once with ctypes, a cudaStream_t) and calls the
+ * C ABI. It exists because a ctypes foreign call costs about a microsecond, comparable to
+ * the whole dispatch it wraps; a METH_FASTCALL call costs a few tens of nanoseconds. */
+#define PY_SSIZE_T_CLEAN
+#include <Python.h>
+#include <stdint.h>
+
+#include "trident_scm.h"
+
+/* invoke(scm, args_address, stream) -> status */
+static PyObject* fc_invoke(PyObject* self, PyObject* const* args, Py_ssize_t nargs) {
+  (void)self;
+  if (nargs != 3) {
+    PyErr_SetString(PyExc_TypeError, "invoke(scm, args_address, stream)");
+    return NULL;
+  }
+  void* scm = PyLong_AsVoidPtr(args[0]);
+  void* a = PyLong_AsVoidPtr(args[1]);
+  void* stream = PyLong_AsVoidPtr(args[2]);
+  if (PyErr_Occurred()) return NULL;
+  return PyLong_FromLong(trident_scm_invoke((trident_scm_t*)scm, (const trident_args*)a, stream, NULL));
+}
+
+/* invoke_seq(scm, args_address, n, stream) -> status */
+static PyObject* fc_invoke_seq(PyObject* self, PyObject* const* args, Py_ssize_t nargs) {
+  (void)self;
+  if (nargs != 4) {
+    PyErr_SetString(PyExc_TypeError, "invoke_seq(scm, args_address, n, stream)");
+    return NULL;
+  }
+  void* scm = PyLong_AsVoidPtr(args[0]);
+  void* a = PyLong_AsVoidPtr(args[1]);
+  long n = PyLong_AsLong(args[2]);
+  void* stream = PyLong_AsVoidPtr(args[3]);
+  if (PyErr_Occurred()) return NULL;
+  return PyLong_FromLong(
+      trident_scm_invoke_seq((trident_scm_t*)scm, (const trident_args*)a, (int32_t)n, stream, NULL));
+}
+
+static PyMethodDef methods[] = {
+    {"invoke", (PyCFunction)(void (*)(void))fc_invoke, METH_FASTCALL, "trident_scm_invoke"},
+    {"invoke_seq", (PyCFunction)(void (*)(void))fc_invoke_seq, METH_FASTCALL, "trident_scm_invoke_seq"},
+    {NULL, NULL, 0, NULL}};
+
+static struct PyModuleDef module = {PyModuleDef_HEAD_INIT, "_fastcall", NULL, -1, methods,
+                                    NULL, NULL, NULL, NULL};
+
+PyMODINIT_FUNC PyInit__fastcall(void) { return PyModule_Create(&module); }

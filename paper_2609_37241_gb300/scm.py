@@ -93,6 +93,18 @@ def lib():
     return _lib
 
 
+def fastcall():
+    """The CPython fast-call shim (`invoke(scm, args_address, stream)` and
+    `invoke_seq(scm, args_address, n, stream)` on raw addresses), or None if it was not
+    built. Same C calls as trident_scm_invoke / _seq, without ctypes' per-call cost."""
+    try:
+        lib()
+        from . import _fastcall
+        return _fastcall
+    except ImportError:
+        return None
+
+
 class ScmError(RuntimeError):
     def __init__(self, status, where):
         self.status = status
