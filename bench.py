@@ -600,6 +600,76 @@ def bench_guard_stress(c, n_calls=None):
     return results
 
 
+def bench_motivation(c, warmup=20, rounds=5, repeats=10):
+    """The paper's motivation experiment (§2.3, Fig. 2) on this GPU: rms_norm of x (1024, 128)
+    with weight (128,), warm path. Per call, host latency (until the Python call returns)
+    and end-to-end latency (until the GPU finishes), after `warmup` calls, `rounds` x
+    `repeats` samples, median -- for this library's SCM, torch eager F.rms_norm, and default
+    torch.compile. Context only: torch is a comparison system here, not the oracle."""
+    t, S, synth = c.torch, c.S, c.synth
+    T, H = 1024, 128
+    x = synth.act_device((T, H), S.BF16, 60, c.dev)
+    w32 = synth.gamma_device(H, 61, c.dev)
+    w16 = w32.to(t.bfloat16).float()  # the same weights, representable in bf16
+    w32.copy_(w16)
+    w_bf = w16.to(t.bfloat16)
+    y = t.empty_like(x)
+    scm = S.Scm(device=c.dev.index or 0)
+    scm.register(S.make_spec(S.OP_RMSNORM, S.BF16, [H], 1, 4096))
+    a = S.make_args(S.OP_RMSNORM, [x, w32, y], eps=1e-6)
+    inv = c.invoker(scm)
+    addr = ctypes.addressof(a)
+    F = t.nn.functional
+
+    def eager():
+        return F.rms_norm(x, (H,), weight=w_bf, eps=1e-6)
+
+    def ours():
+        return inv(addr)
+
+    def measure(fn):
+        for _ in range(warmup):
+            fn()
+        t.cuda.synchronize()
+        host, e2e = [], []
+        for _ in range(rounds):
+            for _ in range(repeats):
+                t.cuda.synchronize()
+                h0 = time.perf_counter()
+                fn()
+                h1 = time.perf_counter()
+                t.cuda.synchronize()
+                h2 = time.perf_counter()
+                host.append((h1 - h0) * 1e6)
+                e2e.append((h2 - h0) * 1e6)
+        return float(np.median(host)), float(np.median(e2e))
+
+    res = {}
+    res["scm"] = dict(zip(("host_us", "e2e_us"), measure(ours)))
+    assert_all_hit(scm, "motivation")
+    c.launches += warmup + rounds * repeats
+    res["torch_eager"] = dict(zip(("host_us", "e2e_us"), measure(eager)))
+    try:
+        compiled = t.compile(eager)
+        compiled()  # compile outside the timed samples
+        res["torch_compile_default"] = dict(zip(("host_us", "e2e_us"), measure(compiled)))
+    except Exception as e:  # context only
+        res["torch_compile_default"] = dict(unavailable=str(e).splitlines()[0][:200])
+    t.cuda.synchronize()
+    agree = float((y.float() - eager().float()).abs().max())
+    scm.close()
+    base = res["torch_eager"]
+    for k, v in res.items():
+        if "host_us" in v:
+            v["speedup_vs_eager_host"] = round(base["host_us"] / v["host_us"], 3)
+            v["speedup_vs_eager_e2e"] = round(base["e2e_us"] / v["e2e_us"], 3)
+            v["host_us"], v["e2e_us"] = round(v["host_us"], 3), round(v["e2e_us"], 3)
+    res["max_abs_diff_scm_vs_eager"] = agree
+    res["shape"] = "x (1024, 128) bf16, weight (128,), eps 1e-6"
+    res["paper_h800_context"] = "Trident vs eager 1.18x host, 1.11x e2e; default torch.compile 0.39x host, 0.43x e2e (§2.3)"
+    return res
+
+
 def bench_sweep(c, reps=20, quick=False):
     """HBM bandwidth sweep: add+RMSNorm (H 8192) and SwiGLU (I 28672) at T = 2^0..2^15,
     bf16. Each size: `reps` back-to-back launches from one native call, rotating across
@@ -746,6 +816,9 @@ def run_ours(a):
     if rank == 0 and want("stress"):
         progress("guard stress")
         extra["guard_stress"] = bench_guard_stress(c, n_calls=20000 if a.quick else None)
+    if rank == 0 and want("motivation"):
+        progress("motivation microbenchmark")
+        extra["motivation_rms_norm"] = bench_motivation(c)
     if rank == 0 and want("sweep"):
         progress("hbm sweep")
         extra["hbm_sweep"] = bench_sweep(c, quick=a.quick)
@@ -848,7 +921,7 @@ def main():
     p.add_argument("--impl", default="ours", choices=["ours", "reference"])
     p.add_argument("--quick", action="store_true", help="smaller sections (for smoke runs)")
     p.add_argument("--sections", default="all",
-                   help="comma list of: layers,qwen3,host,stress,sweep,roofline,e2e,cpu (default all;"
+                   help="comma list of: layers,qwen3,host,stress,motivation,sweep,roofline,e2e,cpu (default all;"
                         " the headline always runs)")
     a = p.parse_args()
     if a.warmup < 3:

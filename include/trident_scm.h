@@ -70,6 +70,11 @@ typedef enum trident_dtype {
  *   s = x + r;  r_out = round(s);  y = round(s * rsqrt(mean(s^2) + eps) * gamma)
  *   In place: y may be x and r_out may be r (same pointer, shape and strides).
  *
+ * TRIDENT_OP_RMSNORM (3 tensors; act = bf16 | fp16 | fp32; rank 2 [T,H] or 3 [B,S,H], T = B*S)
+ *   0 x [T,H] act   1 gamma [H] fp32   2 y [T,H] act (out)
+ *   y = round(x * rsqrt(mean(x^2) + eps) * gamma) -- the paper's running example operator,
+ *   rms_norm (§2.3, Fig. 1). In place: y may be x.
+ *
  * TRIDENT_OP_ROPE_KV (6 tensors; act = bf16 | fp16)
  *   0 q [T,Hq,D] act (in/out)  1 k [T,Hkv,D] act  2 v [T,Hkv,D] act  3 pos [T] i32
  *   4 k_cache [Hkv,S,D] act (out)  5 v_cache [Hkv,S,D] act (out)
@@ -110,7 +115,8 @@ typedef enum trident_op {
   TRIDENT_OP_QKNORM_ROPE_KV = 3,
   TRIDENT_OP_SWIGLU = 4,
   TRIDENT_OP_LAYER_CHAIN = 5,
-  TRIDENT_OP_LAYER_CHAIN_QKNORM = 6
+  TRIDENT_OP_LAYER_CHAIN_QKNORM = 6,
+  TRIDENT_OP_RMSNORM = 7
 } trident_op;
 
 /* Layout class of an argument tuple (guard field, §2.2.1 "shape-related metadata").
@@ -173,10 +179,10 @@ typedef struct trident_args {
 typedef struct trident_spec_desc {
   int32_t op;                       /* trident_op                                        */
   int32_t dtype;                    /* activation dtype                                  */
-  int32_t rank;                     /* rank of slot 0 (2 or 3 for ADD_RMSNORM/SWIGLU,
+  int32_t rank;                     /* rank of slot 0 (2 or 3 for the norms and SWIGLU,
                                        3 for ROPE ops, 2 for the chains)                  */
   int32_t layout;                   /* trident_layout                                    */
-  int64_t fixed[TRIDENT_MAX_FIXED]; /* fixed sizes: ADD_RMSNORM {H}; SWIGLU {I};
+  int64_t fixed[TRIDENT_MAX_FIXED]; /* fixed sizes: ADD_RMSNORM, RMSNORM {H}; SWIGLU {I};
                                        ROPE ops {Hq, Hkv, D, S};
                                        chains {H, Hq, Hkv, D, S, I}; unused entries 0    */
   int64_t tok_lo, tok_hi;           /* inclusive token-count bucket, 1 <= lo <= hi       */

@@ -31,7 +31,7 @@ OK, MISS, INVALID = "OK", "MISS", "INVALID"
 BF16, FP16, FP32, I32, I64 = 1, 2, 3, 4, 5
 ELEM_SIZE = {BF16: 2, FP16: 2, FP32: 4, I32: 4, I64: 8}
 
-ADD_RMSNORM, ROPE_KV, QKNORM_ROPE_KV, SWIGLU, LAYER_CHAIN, LAYER_CHAIN_QKNORM = 1, 2, 3, 4, 5, 6
+ADD_RMSNORM, ROPE_KV, QKNORM_ROPE_KV, SWIGLU, LAYER_CHAIN, LAYER_CHAIN_QKNORM, RMSNORM = 1, 2, 3, 4, 5, 6, 7
 
 CONTIG, ROWSTRIDED, ANY = 0, 1, 2
 LAYOUT_NONE = -1
@@ -54,6 +54,7 @@ SLOTS = {
                   ("x2", "act_H", True), ("r2", "act_H", True),
                   ("g", "act_I", False), ("u", "act_I", False), ("o", "act_I", True)],
 }
+SLOTS[RMSNORM] = [("x", "act_H", False), ("gamma", "gamma_H", False), ("y", "act_H", True)]
 SLOTS[QKNORM_ROPE_KV] = SLOTS[ROPE_KV] + [("gamma_q", "gamma_D", False), ("gamma_k", "gamma_D", False)]
 SLOTS[LAYER_CHAIN_QKNORM] = SLOTS[LAYER_CHAIN] + [("gamma_q", "gamma_D", False),
                                                   ("gamma_k", "gamma_D", False)]
@@ -67,16 +68,17 @@ INPLACE_GROUPS = {
     LAYER_CHAIN: [{"h", "x1"}, {"r0", "r1", "r2"}, {"attn_out", "x2"}, {"g", "u", "o"}],
 }
 INPLACE_GROUPS[LAYER_CHAIN_QKNORM] = INPLACE_GROUPS[LAYER_CHAIN]
+INPLACE_GROUPS[RMSNORM] = [{"x", "y"}]
 
 # Names of the fixed sizes of each op, in spec["fixed"] order.
 FIXED_NAMES = {
-    ADD_RMSNORM: ("H",), SWIGLU: ("I",),
+    ADD_RMSNORM: ("H",), SWIGLU: ("I",), RMSNORM: ("H",),
     ROPE_KV: ("Hq", "Hkv", "D", "S"), QKNORM_ROPE_KV: ("Hq", "Hkv", "D", "S"),
     LAYER_CHAIN: ("H", "Hq", "Hkv", "D", "S", "I"),
     LAYER_CHAIN_QKNORM: ("H", "Hq", "Hkv", "D", "S", "I"),
 }
 ROPE_OPS = (ROPE_KV, QKNORM_ROPE_KV, LAYER_CHAIN, LAYER_CHAIN_QKNORM)
-FLATTENING_OPS = (ADD_RMSNORM, SWIGLU)  # activations may be rank 2 [T,W] or rank 3 [B,S,W]
+FLATTENING_OPS = (ADD_RMSNORM, SWIGLU, RMSNORM)  # activations: rank 2 [T,W] or 3 [B,S,W]
 
 
 def numel(t):

@@ -30,6 +30,8 @@ def lib():
         L.orc_round.argtypes = [dbl, c_int]
         L.orc_add_rmsnorm.restype = None
         L.orc_add_rmsnorm.argtypes = [i64, i64, c_int, P, P, P, dbl, P, P, P]
+        L.orc_rmsnorm.restype = None
+        L.orc_rmsnorm.argtypes = [i64, i64, c_int, P, P, dbl, P, P]
         L.orc_rms_scale.restype = None
         L.orc_rms_scale.argtypes = [i64, P, P, dbl]
         L.orc_rope_apply.restype = None
@@ -89,6 +91,18 @@ def add_rmsnorm(x, r, gamma, eps, dtype):
     lib().orc_add_rmsnorm(T, H, dtype, _p(x), _p(r), _p(gamma), float(eps), _p(y_ref), _p(y),
                           _p(r_out))
     return y_ref, y, r_out
+
+
+def rmsnorm(x, gamma, eps, dtype):
+    """x: [T,H] bits; gamma: [H] float32. Returns (y_ref f64, y bits)."""
+    bd = _bits_dtype(dtype)
+    x = _c(x, bd)
+    gamma = _c(gamma, np.float32)
+    T, H = x.shape
+    y_ref = np.empty((T, H), np.float64)
+    y = np.empty((T, H), bd)
+    lib().orc_rmsnorm(T, H, dtype, _p(x), _p(gamma), float(eps), _p(y_ref), _p(y))
+    return y_ref, y
 
 
 def rms_scale(x, gamma, eps):

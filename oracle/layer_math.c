@@ -9,6 +9,8 @@
  * (§4.1: Qwen3-8B, DeepSeek-V2-Lite), but prints no formula. The functions below are
  * the standard definitions of those layer steps, written out one element at a time:
  *
+ *   RMSNorm       y = x / sqrt(mean(x^2) + eps) * gamma in fp64 (the paper's running
+ *                 example operator, rms_norm, §2.3 and Fig. 1).
  *   add+RMSNorm   s = x + r (fp32 add, the kernel's precision: r_out = round(s) is a
  *                 rounding decision, so both sides take it from the same fp32 value);
  *                 ms = sum(s^2)/H in fp64; y = s / sqrt(ms + eps) * gamma in fp64.
@@ -147,6 +149,26 @@ void orc_add_rmsnorm(int64_t T, int64_t H, int dtype, const void* x, const void*
     for (int64_t j = 0; j < H; ++j) {
       float s = (float)load_act(x, t * H + j, dtype) + (float)load_act(r, t * H + j, dtype);
       double y = (double)s * inv * (double)gamma[j];
+      y_ref[t * H + j] = y;
+      store_act(y_bits, t * H + j, dtype, orc_round(y, dtype));
+    }
+  }
+}
+
+/* ------------------------------------------------------------------ RMSNorm
+ * x, y_bits: contiguous [T,H]; gamma [H]; y_ref [T,H] unrounded:
+ * y = x / sqrt(mean(x^2) + eps) * gamma, in fp64. */
+void orc_rmsnorm(int64_t T, int64_t H, int dtype, const void* x, const float* gamma, double eps,
+                 double* y_ref, void* y_bits) {
+  for (int64_t t = 0; t < T; ++t) {
+    double sumsq = 0.0;
+    for (int64_t j = 0; j < H; ++j) {
+      double v = load_act(x, t * H + j, dtype);
+      sumsq += v * v;
+    }
+    double inv = 1.0 / sqrt(sumsq / (double)H + eps);
+    for (int64_t j = 0; j < H; ++j) {
+      double y = load_act(x, t * H + j, dtype) * inv * (double)gamma[j];
       y_ref[t * H + j] = y;
       store_act(y_bits, t * H + j, dtype, orc_round(y, dtype));
     }

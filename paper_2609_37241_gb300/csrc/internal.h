@@ -26,6 +26,16 @@ struct AddNormParams {
   float eps, inv_H;
 };
 
+// RMSNorm over T rows of H elements (no residual). Row strides in elements.
+struct RmsNormParams {
+  const void* x;
+  const float* gamma;
+  void* y;
+  int64_t T, H;
+  int64_t x_rs, y_rs;
+  float eps, inv_H;
+};
+
 // RoPE on q/k (optionally after per-head RMSNorm) plus KV-cache append.
 // q/k/v rows: token stride *_rs, head stride D, element stride 1. Caches dense [Hkv][S][D].
 // inv_freq: [D/2] pairs (hi, lo), theta^(-2i/D) = hi + lo, split from fp64 on the host.
@@ -74,6 +84,7 @@ struct KernelEntry {
   int32_t kind = 0;      // which grid rule the host applies (KernelKind)
   int32_t vec = 0;       // elements per vector (VE), or tile width for SwiGLU
   int32_t unroll = 1;    // vectors per thread per tile (SwiGLU, chain)
+  int32_t rows = 1;      // rows per block (KK_NORM_ROWS)
 };
 
 enum KernelKind : int32_t {
@@ -82,11 +93,13 @@ enum KernelKind : int32_t {
   KK_ROPE_WARP = 3,     // generic: one warp per head-row
   KK_SWIGLU_TILE = 4,   // grid = (tiles per row, rows)
   KK_SWIGLU_FLAT = 5,   // generic: flat grid-stride
-  KK_CHAIN = 6
+  KK_CHAIN = 6,
+  KK_NORM_ROWS = 7      // grid = ceil(T / rows): several rows per block
 };
 
 // Lookup of compiled kernels. Return false (with a reason) if no kernel fits.
 bool addnorm_kernel(int32_t dtype, int32_t variant, int64_t H, KernelEntry* out, const char** why);
+bool rmsnorm_kernel(int32_t dtype, int32_t variant, int64_t H, KernelEntry* out, const char** why);
 bool rope_kernel(int32_t dtype, int32_t variant, int32_t D, bool qknorm, KernelEntry* out,
                  const char** why);
 bool swiglu_kernel(int32_t dtype, int32_t variant, int64_t I, KernelEntry* out, const char** why);

@@ -103,7 +103,7 @@ struct OpInfo {
   uint8_t group[TRIDENT_MAX_TENSORS];  // in-place group id (0: none)
 };
 
-constexpr int kMaxOp = 6;
+constexpr int kMaxOp = 7;
 OpInfo g_ops[kMaxOp + 1];
 
 // slot index constants of the chains
@@ -137,6 +137,7 @@ struct OpInit {
         {{K_HEADS_Q, true, 0}, {K_HEADS_KV, false, 0}, {K_HEADS_KV, false, 0}, {K_POS, false, 0},
          {K_CACHE, true, 0}, {K_CACHE, true, 0}, {K_GAMMA_D, false, 0}, {K_GAMMA_D, false, 0}});
     set(TRIDENT_OP_SWIGLU, 1, true, false, {{K_ACT_I, false, 1}, {K_ACT_I, false, 1}, {K_ACT_I, true, 1}});
+    set(TRIDENT_OP_RMSNORM, 1, true, false, {{K_ACT_H, false, 1}, {K_GAMMA_H, false, 0}, {K_ACT_H, true, 1}});
     const std::initializer_list<std::tuple<Kind, bool, int>> chain = {
         {K_ACT_H, false, 1},  {K_ACT_H, false, 2},    {K_GAMMA_H, false, 0}, {K_ACT_H, true, 1},
         {K_ACT_H, true, 2},   {K_HEADS_Q, true, 0},   {K_HEADS_KV, false, 0}, {K_HEADS_KV, false, 0},
@@ -290,7 +291,7 @@ void compute_sig(const trident_args* a, const OpInfo& oi, Sig* s) {
   }
   int64_t H = -1, I = -1, Hq = -1, Hkv = -1, D = -1, S = -1;
   const int op = a->op;
-  if (op == TRIDENT_OP_ADD_RMSNORM) {
+  if (op == TRIDENT_OP_ADD_RMSNORM || op == TRIDENT_OP_RMSNORM) {
     H = t[0].shape[s->rank - 1];
     s->fixed[0] = H;
   } else if (op == TRIDENT_OP_SWIGLU) {
@@ -510,6 +511,16 @@ void pack_addnorm(const trident_args* a, int x, int r, int g, int y, int ro, con
   p->inv_H = (float)(1.0 / (double)p->H);
 }
 
+void pack_rmsnorm(const trident_args* a, const Sig& s, RmsNormParams* p) {
+  const trident_tensor* t = a->t;
+  p->x = t[0].data; p->gamma = (const float*)t[1].data; p->y = t[2].data;
+  p->T = s.T;
+  p->H = t[1].shape[0];
+  p->x_rs = row_stride(t[0], K_ACT_H); p->y_rs = row_stride(t[2], K_ACT_H);
+  p->eps = (float)a->eps;
+  p->inv_H = (float)(1.0 / (double)p->H);
+}
+
 void pack_rope(const trident_args* a, int base, int gq, const Version& v, uint32_t* err,
                RopeParams* p) {
   const trident_tensor* t = a->t;
@@ -561,6 +572,7 @@ int32_t do_launch(trident_scm* scm, const Version& v, const trident_args* a, con
   }
   union {
     AddNormParams an;
+    RmsNormParams rn;
     RopeParams rp;
     SwigluParams sw;
     ChainParams ch;
@@ -570,6 +582,10 @@ int32_t do_launch(trident_scm* scm, const Version& v, const trident_args* a, con
     case TRIDENT_OP_ADD_RMSNORM:
       pack_addnorm(a, 0, 1, 2, 3, 4, s, K_ACT_H, &P.an);
       cfg.gridDimX = cap_grid(s.T);
+      break;
+    case TRIDENT_OP_RMSNORM:
+      pack_rmsnorm(a, s, &P.rn);
+      cfg.gridDimX = v.ke.kind == KK_NORM_ROWS ? cap_grid((s.T + v.ke.rows - 1) / v.ke.rows) : cap_grid(s.T);
       break;
     case TRIDENT_OP_ROPE_KV:
     case TRIDENT_OP_QKNORM_ROPE_KV: {
@@ -757,6 +773,7 @@ int32_t resolve_kernel(const trident_spec_desc& d, KernelEntry* ke) {
   auto try_variant = [&](int32_t var) -> bool {
     switch (d.op) {
       case TRIDENT_OP_ADD_RMSNORM: return addnorm_kernel(d.dtype, var, d.fixed[0], ke, &why);
+      case TRIDENT_OP_RMSNORM: return rmsnorm_kernel(d.dtype, var, d.fixed[0], ke, &why);
       case TRIDENT_OP_SWIGLU: return swiglu_kernel(d.dtype, var, d.fixed[0], ke, &why);
       case TRIDENT_OP_ROPE_KV:
       case TRIDENT_OP_QKNORM_ROPE_KV:

@@ -17,12 +17,13 @@ ERR_INVALID, ERR_CUDA, ERR_HOOK, ERR_CAPACITY, ERR_STATE = -1, -2, -3, -4, -5
 NOT_RUN = -2
 BF16, FP16, FP32, I32, I64 = 1, 2, 3, 4, 5
 OP_ADD_RMSNORM, OP_ROPE_KV, OP_QKNORM_ROPE_KV, OP_SWIGLU, OP_LAYER_CHAIN, OP_LAYER_CHAIN_QKNORM = 1, 2, 3, 4, 5, 6
+OP_RMSNORM = 7
 LAYOUT_CONTIG, LAYOUT_ROWSTRIDED, LAYOUT_ANY = 0, 1, 2
 VARIANT_AUTO, VARIANT_GENERIC, VARIANT_VECTOR = 0, 1, 2
 OPT_DRY_RUN, OPT_NO_ALIAS_CHECK, OPT_PDL, OPT_TIMING = 0x1, 0x2, 0x4, 0x8
 DEVERR_POS = 0x1
 MAX_TENSORS, MAX_FIXED = 20, 8
-OP_NTENSORS = {1: 5, 2: 6, 3: 8, 4: 3, 5: 18, 6: 20}
+OP_NTENSORS = {1: 5, 2: 6, 3: 8, 4: 3, 5: 18, 6: 20, 7: 3}
 
 c_i32, c_i64, c_u32, c_u64, c_dbl, c_vp = (ctypes.c_int32, ctypes.c_int64, ctypes.c_uint32,
                                            ctypes.c_uint64, ctypes.c_double, ctypes.c_void_p)

@@ -69,7 +69,12 @@ def make_args(d):
     mis = d.get("misalign", False)
     alloc = _Alloc()
     T = d["T"]
-    if op in (1, 4):
+    if op == 7:
+        lead = (T,) if d.get("rank", 2) == 2 else (d["B"], T // d["B"])
+        W = d["H"]
+        ts = [_rows(alloc, dt, lead, W, layout, dev, mis), tensor(alloc(), 3, (W,), device=dev),
+              _rows(alloc, dt, lead, W, layout, dev)]
+    elif op in (1, 4):
         if d.get("rank", 2) == 3:
             B = d["B"]
             lead = (B, T // B)

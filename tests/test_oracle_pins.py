@@ -149,6 +149,30 @@ def test_add_rmsnorm_residual_zero_passes_x_through():
         assert np.array_equal(r_out, x)
 
 
+# ---------------------------------------------------------------------------- RMSNorm
+def test_rmsnorm_hand_example_and_closed_forms():
+    x = synth.to_bits(np.array([[3, 4, 0, 0]], np.float32), BF16)     # mean(x^2) = 25/4
+    gamma = np.array([1, 2, 3, 4], np.float32)
+    y_ref, y = L.rmsnorm(x, gamma, 0.0, BF16)
+    assert np.allclose(y_ref[0], [3 / 2.5, 4 / 2.5 * 2, 0, 0], rtol=1e-15, atol=0)
+    c, H, eps = -0.75, 128, 1e-6
+    xc = synth.to_bits(np.full((1, H), c, np.float32), BF16)
+    yc, _ = L.rmsnorm(xc, np.ones(H, np.float32), eps, BF16)
+    assert np.allclose(yc[0], c / math.sqrt(c * c + eps), rtol=1e-14)
+
+
+def test_rmsnorm_equals_add_rmsnorm_with_zero_residual():
+    """Two oracle functions, one definition: rms_norm(x) = add+RMSNorm(x, 0).y, bit for bit."""
+    g = np.random.default_rng(14)
+    for dt in (BF16, FP16, FP32):
+        x = synth.act(g, (5, 128), dt)
+        zero = synth.to_bits(np.zeros((5, 128), np.float32), dt)
+        gam = synth.gamma(g, 128)
+        a_ref, a = L.rmsnorm(x, gam, 1e-6, dt)
+        b_ref, b, _ = L.add_rmsnorm(x, zero, gam, 1e-6, dt)
+        assert np.array_equal(a, b) and np.allclose(a_ref, b_ref, rtol=1e-15, atol=0)
+
+
 # ---------------------------------------------------------------------------- RoPE
 def test_rope_position_zero_is_identity():
     g = np.random.default_rng(6)

@@ -144,6 +144,67 @@ def test_add_rmsnorm_degenerate_rows(S):
     s.close()
 
 
+# ---------------------------------------------------------------------------- RMSNorm
+RMSNORM_CASES = [
+    # (dtype, H, T, layout, variant, note)
+    (BF16, 128, 1024, "contig", 0, "the paper's rms_norm shape: 16-lane groups"),
+    (BF16, 128, 37, "strided", 0, "16-lane groups, strided, ragged"),
+    (BF16, 64, 5, "contig", 0, "8-lane groups"),
+    (BF16, 256, 9, "contig", 0, "32-lane groups"),
+    (BF16, 8, 300, "contig", 0, "one lane per row"),
+    (BF16, 4096, 7, "contig", 0, "register row"),
+    (BF16, 1000, 5, "contig", 0, "two-pass loop"),
+    (BF16, 100, 4, "contig", 0, "generic (200-byte rows)"),
+    (BF16, 128, 9, "misaligned", 1, "generic on a misaligned base"),
+    (FP16, 128, 33, "contig", 0, "fp16 lane groups"),
+    (FP32, 128, 17, "contig", 0, "fp32 32-lane groups"),
+    (FP32, 4096, 3, "contig", 0, "fp32 register row"),
+]
+
+
+@pytest.mark.parametrize("dtype,H,T,layout,variant,note", RMSNORM_CASES,
+                         ids=[c[-1] for c in RMSNORM_CASES])
+def test_rmsnorm_parity(S, dtype, H, T, layout, variant, note):
+    g = np.random.default_rng(H + T)
+    x = synth.act(g, (T, H), dtype)
+    gam = synth.gamma(g, H)
+    y_ref, y_bits = L.rmsnorm(x, gam, 1e-6, dtype)
+    es = 4 if dtype == FP32 else 2
+    if layout == "strided":
+        xd, yd = P.padded(x, dtype, 16), P.padded(np.zeros_like(x), dtype, 40)
+        lay = S.LAYOUT_ROWSTRIDED
+    elif layout == "misaligned":
+        buf = torch.zeros(2 * T * H + 2, dtype=synth._TORCH_DT[dtype], device="cuda")
+        xd = buf[1:T * H + 1].view(T, H)
+        xd.copy_(P.dev(x, dtype))
+        yd = buf[T * H + 1:2 * T * H + 1].view(T, H)
+        lay = S.LAYOUT_CONTIG
+    else:
+        xd = P.dev(x, dtype)
+        yd = torch.empty_like(xd)
+        lay = S.LAYOUT_CONTIG
+    align = 16 if variant != 1 and layout != "misaligned" and (H * es) % 16 == 0 else es
+    s = one_version_scm(S, S.make_spec(S.OP_RMSNORM, dtype, [H], 1, 1 << 20, layout=lay,
+                                       align_bytes=align, variant=variant))
+    invoke_ok(s, S, S.make_args(S.OP_RMSNORM, [xd, torch.from_numpy(gam).cuda(), yd], eps=1e-6))
+    torch.cuda.synchronize()
+    s.close()
+    P.check_act(P.host_bits(yd, dtype), y_ref, y_bits, dtype, note, exact_frac=0.99)
+
+
+def test_rmsnorm_in_place(S):
+    g = np.random.default_rng(3)
+    x = synth.act(g, (64, 128), BF16)
+    gam = synth.gamma(g, 128)
+    y_ref, y_bits = L.rmsnorm(x, gam, 1e-6, BF16)
+    xd = P.dev(x, BF16)
+    s = one_version_scm(S, S.make_spec(S.OP_RMSNORM, BF16, [128], 1, 4096))
+    invoke_ok(s, S, S.make_args(S.OP_RMSNORM, [xd, torch.from_numpy(gam).cuda(), xd], eps=1e-6))
+    torch.cuda.synchronize()
+    s.close()
+    P.check_act(P.host_bits(xd, BF16), y_ref, y_bits, BF16, "rmsnorm in place")
+
+
 # ---------------------------------------------------------------------------- RoPE + KV
 def rope_inputs(g, T, Hq, Hkv, D, S_, dtype):
     q, k, v = (synth.act(g, (T, h, D), dtype) for h in (Hq, Hkv, Hkv))

@@ -150,7 +150,7 @@ def _mutations(args, g):
     return out
 
 
-@pytest.mark.parametrize("op", [2, 3, 4, 5, 6])
+@pytest.mark.parametrize("op", [2, 3, 4, 5, 6, 7])
 def test_mutated_arguments_every_op(S, op):
     """Library and oracle agree on valid and mutated tuples of every op."""
     g = np.random.default_rng(100 + op)
@@ -161,6 +161,10 @@ def test_mutated_arguments_every_op(S, op):
     elif op == 4:
         base = dict(op=4, I=48)
         fixed = [48]
+        mk = lambda **k: cases.make_args({**base, **k})
+    elif op == 7:
+        base = dict(op=7, H=128)
+        fixed = [128]
         mk = lambda **k: cases.make_args({**base, **k})
     else:  # a chain version needs a size with a fused kernel (H 4096, D 128)
         base = dict(op=op, H=4096, Hq=4, Hkv=2, D=128, S=64, I=48, theta=10000.0)
@@ -217,7 +221,7 @@ def test_registration_validation(S):
     s = dry(S, max_specs=4)
     good = dict(op=1, dtype=1, fixed=[64], tok_lo=1, tok_hi=8)
     assert s.register(S.make_spec(**good)) == 0
-    bad = [dict(good, op=7), dict(good, dtype=4), dict(good, fixed=[0]), dict(good, fixed=[64, 1]),
+    bad = [dict(good, op=9), dict(good, dtype=4), dict(good, fixed=[0]), dict(good, fixed=[64, 1]),
            dict(good, tok_lo=0), dict(good, tok_lo=5, tok_hi=4), dict(good, align_bytes=8),
            dict(good, rank=4), dict(good, layout=3), dict(good, variant=3),
            dict(good, variant=2, align_bytes=2), dict(good, rope_theta=1.0),
