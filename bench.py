@@ -168,7 +168,7 @@ class Ctx:
 
     def invoker(self, scm):
         """fn(args_struct_or_address) -> status: one trident_scm_invoke from Python."""
-        h, sp = scm.h.value, self.sp.value
+        h, sp = scm.h.value, self.sp.value or 0  # the default stream is NULL
         if self.fc is not None:
             inv = self.fc.invoke
             return lambda addr: inv(h, addr, sp)
@@ -177,7 +177,7 @@ class Ctx:
         return lambda addr: inv(hh, ctypes.cast(addr, P), spp, None)
 
     def seq_invoker(self, scm):
-        h, sp = scm.h.value, self.sp.value
+        h, sp = scm.h.value, self.sp.value or 0
         if self.fc is not None:
             seq = self.fc.invoke_seq
             return lambda addr, n: seq(h, addr, n, sp)
@@ -462,7 +462,7 @@ def bench_host_hit(c, n=1000):
     t.cuda.synchronize()
     fast_us = None
     if c.fc is not None:
-        finv, hh, addr, sp = c.fc.invoke, s.h.value, ctypes.addressof(a), c.sp.value
+        finv, hh, addr, sp = c.fc.invoke, s.h.value, ctypes.addressof(a), c.sp.value or 0
         f0 = time.perf_counter()
         for _ in range(n):
             finv(hh, addr, sp)

@@ -96,8 +96,9 @@ def lib():
 
 def fastcall():
     """The CPython fast-call shim (`invoke(scm, args_address, stream)` and
-    `invoke_seq(scm, args_address, n, stream)` on raw addresses), or None if it was not
-    built. Same C calls as trident_scm_invoke / _seq, without ctypes' per-call cost."""
+    `invoke_seq(scm, args_address, n, stream)` on raw integer addresses; the default stream
+    is 0), or None if it was not built. Same C calls as trident_scm_invoke / _seq, without
+    ctypes' per-call cost."""
     try:
         lib()
         from . import _fastcall

@@ -388,3 +388,27 @@ def test_concurrent_growth_and_invoke(S):
     assert not errors
     assert s.stats().num_specs == 500
     s.close()
+
+
+def test_fastcall_shim_matches_ctypes(S):
+    """The CPython fast-call shim calls the same entry points (dry run, NULL stream = 0)."""
+    import ctypes
+    fc = S.fastcall()
+    if fc is None:
+        pytest.skip("Python headers not installed: the binding uses ctypes only")
+    s = dry(S)
+    s.register(S.make_spec(1, 1, [64], 1, 8))
+    hit = cases.lib_args(cases.make_args({"op": 1, "T": 4, "H": 64}))
+    miss = cases.lib_args(cases.make_args({"op": 1, "T": 40, "H": 64}))
+    bad = cases.lib_args(cases.make_args({"op": 1, "T": 4, "H": 64, "ntensors_delta": -1}))
+    h = s.h.value
+    assert fc.invoke(h, ctypes.addressof(hit), 0) == S.OK
+    assert fc.invoke(h, ctypes.addressof(miss), 0) == S.MISS
+    assert fc.invoke(h, ctypes.addressof(bad), 0) == S.ERR_INVALID
+    arr = (S.trident_args * 3)(hit, hit, miss)
+    assert fc.invoke_seq(h, ctypes.addressof(arr), 3, 0) == S.MISS
+    st = s.stats()
+    assert (st.hits, st.misses, st.err_invalid) == (3, 2, 1)
+    with pytest.raises(TypeError):
+        fc.invoke(h, ctypes.addressof(hit), None)
+    s.close()
