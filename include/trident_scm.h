@@ -34,7 +34,7 @@
 extern "C" {
 #endif
 
-#define TRIDENT_ABI_VERSION 1
+#define TRIDENT_ABI_VERSION 2
 #define TRIDENT_MAX_TENSORS 20
 #define TRIDENT_MAX_FIXED 8
 /* out_selected value for a sequence element that was not run (trident_scm_invoke_seq). */
@@ -58,7 +58,8 @@ typedef enum trident_dtype {
   TRIDENT_FP16 = 2,  /* 2 bytes */
   TRIDENT_FP32 = 3,  /* 4 bytes */
   TRIDENT_I32 = 4,   /* 4 bytes */
-  TRIDENT_I64 = 5    /* 8 bytes */
+  TRIDENT_I64 = 5,   /* 8 bytes */
+  TRIDENT_U8 = 6     /* 1 byte (masks: 0 false, non-zero true) */
 } trident_dtype;
 
 /* ---------------------------------------------------------------- operations
@@ -74,6 +75,15 @@ typedef enum trident_dtype {
  *   0 x [T,H] act   1 gamma [H] fp32   2 y [T,H] act (out)
  *   y = round(x * rsqrt(mean(x^2) + eps) * gamma) -- the paper's running example operator,
  *   rms_norm (§2.3, Fig. 1). In place: y may be x.
+ *
+ * Pointwise operators of the paper's kernel benchmark (§4.1, §4.2; FlagGems-style), over
+ * rows [T,W] or [B,S,W] (T = B*S), act = bf16 | fp16 | fp32, W the version's fixed size:
+ * TRIDENT_OP_SILU (2 tensors)         0 x, 1 y (out):  y = round(x / (1 + exp(-x)))
+ * TRIDENT_OP_ADD (3 tensors)          0 a, 1 b, 2 y (out):  y = round(a + b), summed in fp32
+ * TRIDENT_OP_NEG (2 tensors)          0 x, 1 y (out):  y = -x
+ * TRIDENT_OP_MASKED_FILL (3 tensors)  0 x, 1 mask [T,W] u8, 2 y (out):
+ *                                     y = mask != 0 ? round(args.scalar) : x
+ *   In place: y may be x (or a or b for ADD).
  *
  * TRIDENT_OP_ROPE_KV (6 tensors; act = bf16 | fp16)
  *   0 q [T,Hq,D] act (in/out)  1 k [T,Hkv,D] act  2 v [T,Hkv,D] act  3 pos [T] i32
@@ -116,7 +126,11 @@ typedef enum trident_op {
   TRIDENT_OP_SWIGLU = 4,
   TRIDENT_OP_LAYER_CHAIN = 5,
   TRIDENT_OP_LAYER_CHAIN_QKNORM = 6,
-  TRIDENT_OP_RMSNORM = 7
+  TRIDENT_OP_RMSNORM = 7,
+  TRIDENT_OP_SILU = 8,
+  TRIDENT_OP_ADD = 9,
+  TRIDENT_OP_NEG = 10,
+  TRIDENT_OP_MASKED_FILL = 11
 } trident_op;
 
 /* Layout class of an argument tuple (guard field, §2.2.1 "shape-related metadata").
@@ -170,6 +184,7 @@ typedef struct trident_args {
   int32_t ntensors;      /* must equal the op's slot count */
   double eps;            /* RMSNorm epsilon (runtime scalar, not guarded), must be >= 0 */
   double rope_theta;     /* RoPE base; a specialised constant (guarded by equality, §3.3) */
+  double scalar;         /* MASKED_FILL's fill value (runtime scalar, not guarded) */
   int32_t flags;         /* reserved, must be 0 */
   int32_t reserved;
   trident_tensor t[TRIDENT_MAX_TENSORS];
@@ -179,10 +194,12 @@ typedef struct trident_args {
 typedef struct trident_spec_desc {
   int32_t op;                       /* trident_op                                        */
   int32_t dtype;                    /* activation dtype                                  */
-  int32_t rank;                     /* rank of slot 0 (2 or 3 for the norms and SWIGLU,
+  int32_t rank;                     /* rank of slot 0 (2 or 3 for the norms, SWIGLU and
+                                       the pointwise ops,
                                        3 for ROPE ops, 2 for the chains)                  */
   int32_t layout;                   /* trident_layout                                    */
   int64_t fixed[TRIDENT_MAX_FIXED]; /* fixed sizes: ADD_RMSNORM, RMSNORM {H}; SWIGLU {I};
+                                       SILU, ADD, NEG, MASKED_FILL {W};
                                        ROPE ops {Hq, Hkv, D, S};
                                        chains {H, Hq, Hkv, D, S, I}; unused entries 0    */
   int64_t tok_lo, tok_hi;           /* inclusive token-count bucket, 1 <= lo <= hi       */

@@ -28,10 +28,11 @@ Everything is plain Python over plain dicts:
 
 OK, MISS, INVALID = "OK", "MISS", "INVALID"
 
-BF16, FP16, FP32, I32, I64 = 1, 2, 3, 4, 5
-ELEM_SIZE = {BF16: 2, FP16: 2, FP32: 4, I32: 4, I64: 8}
+BF16, FP16, FP32, I32, I64, U8 = 1, 2, 3, 4, 5, 6
+ELEM_SIZE = {BF16: 2, FP16: 2, FP32: 4, I32: 4, I64: 8, U8: 1}
 
 ADD_RMSNORM, ROPE_KV, QKNORM_ROPE_KV, SWIGLU, LAYER_CHAIN, LAYER_CHAIN_QKNORM, RMSNORM = 1, 2, 3, 4, 5, 6, 7
+SILU, ADD, NEG, MASKED_FILL = 8, 9, 10, 11
 
 CONTIG, ROWSTRIDED, ANY = 0, 1, 2
 LAYOUT_NONE = -1
@@ -55,6 +56,11 @@ SLOTS = {
                   ("g", "act_I", False), ("u", "act_I", False), ("o", "act_I", True)],
 }
 SLOTS[RMSNORM] = [("x", "act_H", False), ("gamma", "gamma_H", False), ("y", "act_H", True)]
+# pointwise operators over [T, W] rows (W is the version's fixed size, named "H" here)
+SLOTS[SILU] = [("x", "act_H", False), ("y", "act_H", True)]
+SLOTS[NEG] = [("x", "act_H", False), ("y", "act_H", True)]
+SLOTS[ADD] = [("a", "act_H", False), ("b", "act_H", False), ("y", "act_H", True)]
+SLOTS[MASKED_FILL] = [("x", "act_H", False), ("mask", "mask_H", False), ("y", "act_H", True)]
 SLOTS[QKNORM_ROPE_KV] = SLOTS[ROPE_KV] + [("gamma_q", "gamma_D", False), ("gamma_k", "gamma_D", False)]
 SLOTS[LAYER_CHAIN_QKNORM] = SLOTS[LAYER_CHAIN] + [("gamma_q", "gamma_D", False),
                                                   ("gamma_k", "gamma_D", False)]
@@ -69,16 +75,21 @@ INPLACE_GROUPS = {
 }
 INPLACE_GROUPS[LAYER_CHAIN_QKNORM] = INPLACE_GROUPS[LAYER_CHAIN]
 INPLACE_GROUPS[RMSNORM] = [{"x", "y"}]
+INPLACE_GROUPS[SILU] = [{"x", "y"}]
+INPLACE_GROUPS[NEG] = [{"x", "y"}]
+INPLACE_GROUPS[ADD] = [{"a", "b", "y"}]
+INPLACE_GROUPS[MASKED_FILL] = [{"x", "y"}]
 
 # Names of the fixed sizes of each op, in spec["fixed"] order.
 FIXED_NAMES = {
     ADD_RMSNORM: ("H",), SWIGLU: ("I",), RMSNORM: ("H",),
+    SILU: ("H",), NEG: ("H",), ADD: ("H",), MASKED_FILL: ("H",),
     ROPE_KV: ("Hq", "Hkv", "D", "S"), QKNORM_ROPE_KV: ("Hq", "Hkv", "D", "S"),
     LAYER_CHAIN: ("H", "Hq", "Hkv", "D", "S", "I"),
     LAYER_CHAIN_QKNORM: ("H", "Hq", "Hkv", "D", "S", "I"),
 }
 ROPE_OPS = (ROPE_KV, QKNORM_ROPE_KV, LAYER_CHAIN, LAYER_CHAIN_QKNORM)
-FLATTENING_OPS = (ADD_RMSNORM, SWIGLU, RMSNORM)  # activations: rank 2 [T,W] or 3 [B,S,W]
+FLATTENING_OPS = (ADD_RMSNORM, SWIGLU, RMSNORM, SILU, ADD, NEG, MASKED_FILL)  # rank 2 or 3
 
 
 def numel(t):
@@ -127,7 +138,7 @@ def token_count(op, slot0):
 
 
 def expected_rank(op, kind, spec_rank):
-    if kind in ("act_H", "act_I"):
+    if kind in ("act_H", "act_I", "mask_H"):
         return spec_rank if op in FLATTENING_OPS else 2
     return {"gamma_H": 1, "gamma_D": 1, "pos": 1, "heads_q": 3, "heads_kv": 3, "cache": 3}[kind]
 
@@ -137,13 +148,15 @@ def expected_dtype(kind, spec_dtype):
         return FP32
     if kind == "pos":
         return I32
+    if kind == "mask_H":
+        return U8
     return spec_dtype
 
 
 def shape_ok(kind, shape, lead, fx):
     """Does `shape` equal what slot `kind` must have, given the leading dims `lead` of slot 0
     (one entry for rank 2, two for rank 3) and the version's fixed sizes `fx`?"""
-    if kind == "act_H":
+    if kind in ("act_H", "mask_H"):
         return list(shape) == list(lead) + [fx["H"]]
     if kind == "act_I":
         return list(shape) == list(lead) + [fx["I"]]
@@ -184,7 +197,7 @@ def layout_class(args):
     op = args["op"]
     all_contig = True
     for (name, kind, _), t in zip(SLOTS[op], args["tensors"]):
-        if kind not in ("act_H", "act_I", "heads_q", "heads_kv"):
+        if kind not in ("act_H", "act_I", "mask_H", "heads_q", "heads_kv"):
             continue
         rows, width, rstride, packed = rows_of(t, kind)
         if not packed:

@@ -39,6 +39,12 @@ def lib():
         L.orc_rope_kv.restype = c_int
         L.orc_rope_kv.argtypes = [i64, i64, i64, i64, i64, c_int, dbl, c_int, P, P, dbl,
                                   P, P, P, P, P, P, P, P]
+        for name, nin in (("orc_silu", 1), ("orc_neg", 1), ("orc_add", 2)):
+            f = getattr(L, name)
+            f.restype = None
+            f.argtypes = [i64, c_int] + [P] * nin + [P, P]
+        L.orc_masked_fill.restype = None
+        L.orc_masked_fill.argtypes = [i64, c_int, P, P, dbl, P, P]
         L.orc_swiglu.restype = None
         L.orc_swiglu.argtypes = [i64, c_int, P, P, P, P]
         _lib = L
@@ -142,6 +148,40 @@ def rope_kv(q, k, v, pos, k_cache, v_cache, theta, dtype, qknorm=False, gamma_q=
     if bad < 0:
         raise ValueError("head_dim too large for the oracle")
     return dict(q=q, q_ref=q_ref, k_ref=k_ref, k_cache=kc, v_cache=vc, bad=bad)
+
+
+def _pointwise(name, dtype, *arrays):
+    bd = _bits_dtype(dtype)
+    arrs = [_c(a, bd) for a in arrays]
+    ref = np.empty(arrs[0].shape, np.float64)
+    out = np.empty(arrs[0].shape, bd)
+    getattr(lib(), name)(arrs[0].size, dtype, *[_p(a) for a in arrs], _p(ref), _p(out))
+    return ref, out
+
+
+def silu(x, dtype):
+    """Returns (ref f64, out bits) of x / (1 + exp(-x))."""
+    return _pointwise("orc_silu", dtype, x)
+
+
+def neg(x, dtype):
+    return _pointwise("orc_neg", dtype, x)
+
+
+def add(a, b, dtype):
+    """a + b summed in fp32, then rounded to dtype."""
+    return _pointwise("orc_add", dtype, a, b)
+
+
+def masked_fill(x, mask, value, dtype):
+    """mask != 0 -> value (rounded once to dtype), else x."""
+    bd = _bits_dtype(dtype)
+    x = _c(x, bd)
+    m = _c(mask, np.uint8)
+    ref = np.empty(x.shape, np.float64)
+    out = np.empty(x.shape, bd)
+    lib().orc_masked_fill(x.size, dtype, _p(x), _p(m), float(value), _p(ref), _p(out))
+    return ref, out
 
 
 def swiglu(g, u, dtype):

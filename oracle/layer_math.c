@@ -244,6 +244,56 @@ int orc_rope_kv(int64_t T, int64_t Hq, int64_t Hkv, int64_t D, int64_t S, int dt
   return bad;
 }
 
+/* ------------------------------------------------------------------ pointwise operators
+ * The FlagGems-style operators of the paper's kernel benchmark (§4.1): silu, add, neg,
+ * masked_fill, over n contiguous elements; ref = unrounded result, out = its rounding.
+ *   silu(x) = x / (1 + exp(-x))                     (fp64)
+ *   add     = a + b, summed in fp32 (the kernels' precision: the rounding of the sum is a
+ *             rounding decision, taken from the same fp32 value on both sides)
+ *   neg     = -x                                    (exact)
+ *   masked_fill: mask != 0 ? value : x, with value converted to fp32 and then rounded to
+ *             the activation type */
+void orc_silu(int64_t n, int dtype, const void* x, double* ref, void* out_bits) {
+  for (int64_t i = 0; i < n; ++i) {
+    double v = load_act(x, i, dtype);
+    double o = v / (1.0 + exp(-v));
+    ref[i] = o;
+    store_act(out_bits, i, dtype, orc_round(o, dtype));
+  }
+}
+
+void orc_add(int64_t n, int dtype, const void* a, const void* b, double* ref, void* out_bits) {
+  for (int64_t i = 0; i < n; ++i) {
+    float s = (float)load_act(a, i, dtype) + (float)load_act(b, i, dtype);
+    ref[i] = (double)s;
+    store_act(out_bits, i, dtype, orc_round((double)s, dtype));
+  }
+}
+
+void orc_neg(int64_t n, int dtype, const void* x, double* ref, void* out_bits) {
+  for (int64_t i = 0; i < n; ++i) {
+    double v = -load_act(x, i, dtype);
+    ref[i] = v;
+    store_act(out_bits, i, dtype, orc_round(v, dtype));
+  }
+}
+
+void orc_masked_fill(int64_t n, int dtype, const void* x, const uint8_t* mask, double value,
+                     double* ref, void* out_bits) {
+  /* the fill value is converted to fp32 first, then rounded to the activation type, as a
+     framework scalar reaches a bf16/fp16 tensor */
+  uint32_t vbits = orc_round((double)(float)value, dtype);
+  for (int64_t i = 0; i < n; ++i) {
+    if (mask[i]) {
+      ref[i] = orc_widen(vbits, dtype);
+      store_act(out_bits, i, dtype, vbits);
+    } else {
+      ref[i] = load_act(x, i, dtype);
+      store_act(out_bits, i, dtype, (dtype == OR_FP32) ? ((const uint32_t*)x)[i] : ((const uint16_t*)x)[i]);
+    }
+  }
+}
+
 /* ------------------------------------------------------------------ SwiGLU
  * g, u, out_bits: n contiguous elements; ref: n unrounded results. */
 void orc_swiglu(int64_t n, int dtype, const void* g, const void* u, double* ref,

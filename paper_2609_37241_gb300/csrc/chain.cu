@@ -19,8 +19,10 @@ namespace trident {
 
 constexpr int kChainSwigluUnroll = 2;
 
+// Four resident blocks per SM for H 4096 (64 registers): the 64-token grid (576 blocks)
+// then fits one wave on 152 SMs; a fifth register would drop it to three blocks per SM.
 template <int DT, int VPT, int SPLIT, int D, bool QKNORM>
-__global__ void __launch_bounds__(kThreads) chain_kernel(const ChainParams c) {
+__global__ void __launch_bounds__(kThreads, VPT == 2 ? 4 : 2) chain_kernel(const ChainParams c) {
   pdl_prologue();
   constexpr int EB = Act<DT>::BYTES;
   constexpr int VE = Act<DT>::VE;

@@ -36,6 +36,19 @@ struct RmsNormParams {
   float eps, inv_H;
 };
 
+// Pointwise operators over T rows of W elements (a: x or the first addend; b: the second
+// addend; mask: u8 for MASKED_FILL). Row strides in elements.
+enum PointwiseOp : int32_t { PW_SILU = 8, PW_ADD = 9, PW_NEG = 10, PW_MASKED_FILL = 11 };
+struct PointwiseParams {
+  const void* a;
+  const void* b;
+  const uint8_t* mask;
+  void* y;
+  int64_t T, W;
+  int64_t a_rs, b_rs, m_rs, y_rs;
+  float scalar;
+};
+
 // RoPE on q/k (optionally after per-head RMSNorm) plus KV-cache append.
 // q/k/v rows: token stride *_rs, head stride D, element stride 1. Caches dense [Hkv][S][D].
 // inv_freq: [D/2] pairs (hi, lo), theta^(-2i/D) = hi + lo, split from fp64 on the host.
@@ -100,6 +113,8 @@ enum KernelKind : int32_t {
 // Lookup of compiled kernels. Return false (with a reason) if no kernel fits.
 bool addnorm_kernel(int32_t dtype, int32_t variant, int64_t H, KernelEntry* out, const char** why);
 bool rmsnorm_kernel(int32_t dtype, int32_t variant, int64_t H, KernelEntry* out, const char** why);
+bool pointwise_kernel(int32_t op, int32_t dtype, int32_t variant, int64_t W, KernelEntry* out,
+                      const char** why);
 bool rope_kernel(int32_t dtype, int32_t variant, int32_t D, bool qknorm, KernelEntry* out,
                  const char** why);
 bool swiglu_kernel(int32_t dtype, int32_t variant, int64_t I, KernelEntry* out, const char** why);

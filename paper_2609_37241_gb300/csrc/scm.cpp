@@ -91,7 +91,8 @@ bool driver() {
 }
 
 // ------------------------------------------------------------------ op tables
-enum Kind : uint8_t { K_ACT_H, K_ACT_I, K_GAMMA_H, K_GAMMA_D, K_HEADS_Q, K_HEADS_KV, K_POS, K_CACHE };
+enum Kind : uint8_t { K_ACT_H, K_ACT_I, K_GAMMA_H, K_GAMMA_D, K_HEADS_Q, K_HEADS_KV, K_POS, K_CACHE,
+                     K_MASK_H };
 
 struct OpInfo {
   int32_t nslots;
@@ -103,7 +104,7 @@ struct OpInfo {
   uint8_t group[TRIDENT_MAX_TENSORS];  // in-place group id (0: none)
 };
 
-constexpr int kMaxOp = 7;
+constexpr int kMaxOp = 11;
 OpInfo g_ops[kMaxOp + 1];
 
 // slot index constants of the chains
@@ -138,6 +139,10 @@ struct OpInit {
          {K_CACHE, true, 0}, {K_CACHE, true, 0}, {K_GAMMA_D, false, 0}, {K_GAMMA_D, false, 0}});
     set(TRIDENT_OP_SWIGLU, 1, true, false, {{K_ACT_I, false, 1}, {K_ACT_I, false, 1}, {K_ACT_I, true, 1}});
     set(TRIDENT_OP_RMSNORM, 1, true, false, {{K_ACT_H, false, 1}, {K_GAMMA_H, false, 0}, {K_ACT_H, true, 1}});
+    set(TRIDENT_OP_SILU, 1, true, false, {{K_ACT_H, false, 1}, {K_ACT_H, true, 1}});
+    set(TRIDENT_OP_NEG, 1, true, false, {{K_ACT_H, false, 1}, {K_ACT_H, true, 1}});
+    set(TRIDENT_OP_ADD, 1, true, false, {{K_ACT_H, false, 1}, {K_ACT_H, false, 1}, {K_ACT_H, true, 1}});
+    set(TRIDENT_OP_MASKED_FILL, 1, true, false, {{K_ACT_H, false, 1}, {K_MASK_H, false, 0}, {K_ACT_H, true, 1}});
     const std::initializer_list<std::tuple<Kind, bool, int>> chain = {
         {K_ACT_H, false, 1},  {K_ACT_H, false, 2},    {K_GAMMA_H, false, 0}, {K_ACT_H, true, 1},
         {K_ACT_H, true, 2},   {K_HEADS_Q, true, 0},   {K_HEADS_KV, false, 0}, {K_HEADS_KV, false, 0},
@@ -159,10 +164,13 @@ inline int elem_size(int32_t dt) {
     case TRIDENT_BF16: case TRIDENT_FP16: return 2;
     case TRIDENT_FP32: case TRIDENT_I32: return 4;
     case TRIDENT_I64: return 8;
+    case TRIDENT_U8: return 1;
     default: return 0;
   }
 }
 inline bool is_act(Kind k) { return k == K_ACT_H || k == K_ACT_I || k == K_HEADS_Q || k == K_HEADS_KV; }
+// Tensors with activation-like rows (they take part in the layout class): activations and masks.
+inline bool is_rowlike(Kind k) { return is_act(k) || k == K_MASK_H; }
 
 // Rows view of a tensor: (rows, row width in elements, row stride in elements, packed).
 struct Rows {
@@ -175,7 +183,7 @@ inline Rows rows_of(const trident_tensor& t, Kind k) {
   const int64_t* st = t.stride;
   if (k == K_HEADS_Q || k == K_HEADS_KV)
     return {sh[0], sh[1] * sh[2], st[0], st[2] == 1 && (sh[1] <= 1 || st[1] == sh[2])};
-  if (k == K_ACT_H || k == K_ACT_I) {
+  if (k == K_ACT_H || k == K_ACT_I || k == K_MASK_H) {
     if (t.ndim == 2) return {sh[0], sh[1], st[0], st[1] == 1};
     const bool inner = st[2] == 1;
     if (sh[1] == 1) return {sh[0], sh[2], st[0], inner};
@@ -258,6 +266,8 @@ void compute_sig(const trident_args* a, const OpInfo& oi, Sig* s) {
       else if (s->act_dtype != t[i].dtype) s->act_dtype = kMixed;
     } else if (k == K_POS) {
       s->aux_dtype_ok &= t[i].dtype == TRIDENT_I32;
+    } else if (k == K_MASK_H) {
+      s->aux_dtype_ok &= t[i].dtype == TRIDENT_U8;
     } else {
       s->aux_dtype_ok &= t[i].dtype == TRIDENT_FP32;
     }
@@ -268,7 +278,7 @@ void compute_sig(const trident_args* a, const OpInfo& oi, Sig* s) {
   s->ranks_ok = !oi.flattening || s->rank == 2 || s->rank == 3;
   for (int i = 0; i < n && s->ranks_ok; ++i) {
     const Kind k = oi.kind[i];
-    const int want = (k == K_ACT_H || k == K_ACT_I) ? act_rank
+    const int want = (k == K_ACT_H || k == K_ACT_I || k == K_MASK_H) ? act_rank
                    : (k == K_HEADS_Q || k == K_HEADS_KV || k == K_CACHE) ? 3 : 1;
     s->ranks_ok = t[i].ndim == want;
   }
@@ -291,7 +301,7 @@ void compute_sig(const trident_args* a, const OpInfo& oi, Sig* s) {
   }
   int64_t H = -1, I = -1, Hq = -1, Hkv = -1, D = -1, S = -1;
   const int op = a->op;
-  if (op == TRIDENT_OP_ADD_RMSNORM || op == TRIDENT_OP_RMSNORM) {
+  if (op == TRIDENT_OP_ADD_RMSNORM || op == TRIDENT_OP_RMSNORM || op >= TRIDENT_OP_SILU) {
     H = t[0].shape[s->rank - 1];
     s->fixed[0] = H;
   } else if (op == TRIDENT_OP_SWIGLU) {
@@ -317,8 +327,8 @@ void compute_sig(const trident_args* a, const OpInfo& oi, Sig* s) {
   for (int i = 0; i < n && ok; ++i) {
     const trident_tensor& x = t[i];
     switch (oi.kind[i]) {
-      case K_ACT_H: case K_ACT_I: {
-        const int64_t w = oi.kind[i] == K_ACT_H ? H : I;
+      case K_ACT_H: case K_ACT_I: case K_MASK_H: {
+        const int64_t w = oi.kind[i] == K_ACT_I ? I : H;
         ok = s->nlead == 2 ? shape_is(x, {s->lead[0], s->lead[1], w}) : shape_is(x, {T0, w});
         break;
       }
@@ -334,7 +344,7 @@ void compute_sig(const trident_args* a, const OpInfo& oi, Sig* s) {
   // layout class over the activations
   bool all_contig = true, none = false;
   for (int i = 0; i < n; ++i) {
-    if (!is_act(oi.kind[i])) continue;
+    if (!is_rowlike(oi.kind[i])) continue;
     const Rows r = rows_of(t[i], oi.kind[i]);
     if (!r.packed) { none = true; break; }
     if (r.n <= 1) continue;
@@ -521,6 +531,23 @@ void pack_rmsnorm(const trident_args* a, const Sig& s, RmsNormParams* p) {
   p->inv_H = (float)(1.0 / (double)p->H);
 }
 
+void pack_pointwise(const trident_args* a, const Sig& s, PointwiseParams* p) {
+  const trident_tensor* t = a->t;
+  const int op = a->op;
+  const int yi = (op == TRIDENT_OP_SILU || op == TRIDENT_OP_NEG) ? 1 : 2;
+  p->a = t[0].data;
+  p->b = op == TRIDENT_OP_ADD ? t[1].data : nullptr;
+  p->mask = op == TRIDENT_OP_MASKED_FILL ? (const uint8_t*)t[1].data : nullptr;
+  p->y = t[yi].data;
+  p->T = s.T;
+  p->W = s.fixed[0];
+  p->a_rs = row_stride(t[0], K_ACT_H);
+  p->b_rs = op == TRIDENT_OP_ADD ? row_stride(t[1], K_ACT_H) : 0;
+  p->m_rs = op == TRIDENT_OP_MASKED_FILL ? row_stride(t[1], K_MASK_H) : 0;
+  p->y_rs = row_stride(t[yi], K_ACT_H);
+  p->scalar = (float)a->scalar;
+}
+
 void pack_rope(const trident_args* a, int base, int gq, const Version& v, uint32_t* err,
                RopeParams* p) {
   const trident_tensor* t = a->t;
@@ -573,6 +600,7 @@ int32_t do_launch(trident_scm* scm, const Version& v, const trident_args* a, con
   union {
     AddNormParams an;
     RmsNormParams rn;
+    PointwiseParams pw;
     RopeParams rp;
     SwigluParams sw;
     ChainParams ch;
@@ -596,16 +624,28 @@ int32_t do_launch(trident_scm* scm, const Version& v, const trident_args* a, con
       break;
     }
     case TRIDENT_OP_SWIGLU:
-      pack_swiglu(a, 0, 1, 2, s.T, &P.sw);
-      if (v.ke.kind == KK_SWIGLU_TILE) {
-        const int64_t per = (int64_t)v.ke.unroll * kThreads * v.ke.vec;
-        cfg.gridDimX = cap_grid((P.sw.I + per - 1) / per);
-        cfg.gridDimY = (unsigned)(s.T < 65535 ? (s.T < 1 ? 1 : s.T) : 65535);
+    case TRIDENT_OP_SILU:
+    case TRIDENT_OP_ADD:
+    case TRIDENT_OP_NEG:
+    case TRIDENT_OP_MASKED_FILL: {
+      int64_t W;
+      if (op == TRIDENT_OP_SWIGLU) {
+        pack_swiglu(a, 0, 1, 2, s.T, &P.sw);
+        W = P.sw.I;
       } else {
-        const int64_t total = s.T * P.sw.I;
-        cfg.gridDimX = cap_grid((total + kThreads - 1) / kThreads < 152 * 64 ? (total + kThreads - 1) / kThreads : 152 * 64);
+        pack_pointwise(a, s, &P.pw);
+        W = P.pw.W;
+      }
+      if (v.ke.kind == KK_SWIGLU_TILE) {  // (column tiles, rows)
+        const int64_t per = (int64_t)v.ke.unroll * kThreads * v.ke.vec;
+        cfg.gridDimX = cap_grid((W + per - 1) / per);
+        cfg.gridDimY = (unsigned)(s.T < 65535 ? (s.T < 1 ? 1 : s.T) : 65535);
+      } else {  // flat grid-stride
+        const int64_t blocks = (s.T * W + kThreads - 1) / kThreads;
+        cfg.gridDimX = cap_grid(blocks < 152 * 64 ? blocks : 152 * 64);
       }
       break;
+    }
     case TRIDENT_OP_LAYER_CHAIN:
     case TRIDENT_OP_LAYER_CHAIN_QKNORM: {
       ChainParams& c = P.ch;
@@ -774,6 +814,10 @@ int32_t resolve_kernel(const trident_spec_desc& d, KernelEntry* ke) {
     switch (d.op) {
       case TRIDENT_OP_ADD_RMSNORM: return addnorm_kernel(d.dtype, var, d.fixed[0], ke, &why);
       case TRIDENT_OP_RMSNORM: return rmsnorm_kernel(d.dtype, var, d.fixed[0], ke, &why);
+      case TRIDENT_OP_SILU:
+      case TRIDENT_OP_ADD:
+      case TRIDENT_OP_NEG:
+      case TRIDENT_OP_MASKED_FILL: return pointwise_kernel(d.op, d.dtype, var, d.fixed[0], ke, &why);
       case TRIDENT_OP_SWIGLU: return swiglu_kernel(d.dtype, var, d.fixed[0], ke, &why);
       case TRIDENT_OP_ROPE_KV:
       case TRIDENT_OP_QKNORM_ROPE_KV:

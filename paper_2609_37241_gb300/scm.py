@@ -15,15 +15,16 @@ LIB_PATH = os.path.join(PKG, "_lib", "libtrident_scm.so")
 OK, MISS_HANDLED, MISS = 0, 1, 2
 ERR_INVALID, ERR_CUDA, ERR_HOOK, ERR_CAPACITY, ERR_STATE = -1, -2, -3, -4, -5
 NOT_RUN = -2
-BF16, FP16, FP32, I32, I64 = 1, 2, 3, 4, 5
+BF16, FP16, FP32, I32, I64, U8 = 1, 2, 3, 4, 5, 6
 OP_ADD_RMSNORM, OP_ROPE_KV, OP_QKNORM_ROPE_KV, OP_SWIGLU, OP_LAYER_CHAIN, OP_LAYER_CHAIN_QKNORM = 1, 2, 3, 4, 5, 6
 OP_RMSNORM = 7
+OP_SILU, OP_ADD, OP_NEG, OP_MASKED_FILL = 8, 9, 10, 11
 LAYOUT_CONTIG, LAYOUT_ROWSTRIDED, LAYOUT_ANY = 0, 1, 2
 VARIANT_AUTO, VARIANT_GENERIC, VARIANT_VECTOR = 0, 1, 2
 OPT_DRY_RUN, OPT_NO_ALIAS_CHECK, OPT_PDL, OPT_TIMING = 0x1, 0x2, 0x4, 0x8
 DEVERR_POS = 0x1
 MAX_TENSORS, MAX_FIXED = 20, 8
-OP_NTENSORS = {1: 5, 2: 6, 3: 8, 4: 3, 5: 18, 6: 20, 7: 3}
+OP_NTENSORS = {1: 5, 2: 6, 3: 8, 4: 3, 5: 18, 6: 20, 7: 3, 8: 2, 9: 3, 10: 2, 11: 3}
 
 c_i32, c_i64, c_u32, c_u64, c_dbl, c_vp = (ctypes.c_int32, ctypes.c_int64, ctypes.c_uint32,
                                            ctypes.c_uint64, ctypes.c_double, ctypes.c_void_p)
@@ -36,7 +37,8 @@ class trident_tensor(ctypes.Structure):
 
 class trident_args(ctypes.Structure):
     _fields_ = [("op", c_i32), ("ntensors", c_i32), ("eps", c_dbl), ("rope_theta", c_dbl),
-                ("flags", c_i32), ("reserved", c_i32), ("t", trident_tensor * MAX_TENSORS)]
+                ("scalar", c_dbl), ("flags", c_i32), ("reserved", c_i32),
+                ("t", trident_tensor * MAX_TENSORS)]
 
 
 class trident_spec_desc(ctypes.Structure):
@@ -208,7 +210,7 @@ def _torch_dtypes():
     if _TORCH_DT is None:
         import torch
         _TORCH_DT = {torch.bfloat16: BF16, torch.float16: FP16, torch.float32: FP32,
-                     torch.int32: I32, torch.int64: I64}
+                     torch.int32: I32, torch.int64: I64, torch.uint8: U8, torch.bool: U8}
     return _TORCH_DT
 
 
@@ -238,13 +240,14 @@ def fill_tensor_dict(dst, d):
     return dst
 
 
-def make_args(op, tensors, eps=1e-6, rope_theta=0.0):
+def make_args(op, tensors, eps=1e-6, rope_theta=0.0, scalar=0.0):
     """trident_args from torch tensors (or plain dicts) in the op's slot order."""
     a = trident_args()
     a.op = op
     a.ntensors = len(tensors)
     a.eps = eps
     a.rope_theta = rope_theta
+    a.scalar = scalar
     for i, t in enumerate(tensors):
         if isinstance(t, dict):
             fill_tensor_dict(a.t[i], t)

@@ -4,8 +4,8 @@ Tensors here are descriptors only (fake addresses), for host-side selection test
 The same dicts are handed to the oracle (`oracle.guards`) and, converted field by
 field, to the library (`paper_2609_37241_gb300.scm`).
 """
-DT = {"bf16": 1, "fp16": 2, "fp32": 3, "i32": 4, "i64": 5}
-ES = {1: 2, 2: 2, 3: 4, 4: 4, 5: 8}
+DT = {"bf16": 1, "fp16": 2, "fp32": 3, "i32": 4, "i64": 5, "u8": 6}
+ES = {1: 2, 2: 2, 3: 4, 4: 4, 5: 8, 6: 1}
 LAYOUT = {"contig": 0, "strided": 1, "any": 2}
 BASE = 0x7F0000000000
 SPAN = 1 << 32  # address distance between buffers
@@ -74,6 +74,15 @@ def make_args(d):
         W = d["H"]
         ts = [_rows(alloc, dt, lead, W, layout, dev, mis), tensor(alloc(), 3, (W,), device=dev),
               _rows(alloc, dt, lead, W, layout, dev)]
+    elif op in (8, 9, 10, 11):
+        lead = (T,) if d.get("rank", 2) == 2 else (d["B"], T // d["B"])
+        W = d["H"]
+        ts = [_rows(alloc, dt, lead, W, layout, dev, mis)]
+        if op == 9:
+            ts.append(_rows(alloc, dt, lead, W, layout, dev))
+        if op == 11:
+            ts.append(_rows(alloc, 6, lead, W, layout, dev))
+        ts.append(_rows(alloc, dt, lead, W, layout, dev))
     elif op in (1, 4):
         if d.get("rank", 2) == 3:
             B = d["B"]
@@ -113,7 +122,7 @@ def make_args(d):
     elif delta > 0:
         ts = ts + [tensor(alloc(), 3, (1,), device=dev)] * delta
     return dict(op=op, tensors=ts, eps=float(d.get("eps", 1e-6)),
-                theta=float(d.get("theta", 0.0)), flags=0)
+                theta=float(d.get("theta", 0.0)), flags=0, scalar=float(d.get("scalar", 0.0)))
 
 
 def make_chain_args(d):
@@ -161,7 +170,8 @@ def lib_spec(spec):
 def lib_args(args):
     """Library argument tuple (ctypes) from an oracle-style args dict."""
     from paper_2609_37241_gb300 import scm
-    return scm.make_args(args["op"], args["tensors"], eps=args["eps"], rope_theta=args["theta"])
+    return scm.make_args(args["op"], args["tensors"], eps=args["eps"], rope_theta=args["theta"],
+                         scalar=args.get("scalar", 0.0))
 
 
 STATUS = {0: "OK", 2: "MISS", -1: "INVALID"}

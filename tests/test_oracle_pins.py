@@ -278,6 +278,48 @@ def test_swiglu_closed_forms():
     assert np.allclose(ref3, 3 * ref, rtol=1e-15)
 
 
+# ---------------------------------------------------------------------------- pointwise
+def test_pointwise_closed_forms_and_library_casts():
+    g = np.random.default_rng(15)
+    xf = (g.normal(size=4000) * 3).astype(np.float32)
+    for dt in (BF16, FP16, FP32):
+        x = synth.to_bits(xf, dt)
+        xv = L.widen(x[:64], dt)
+        # silu against its closed form at special points and the SwiGLU oracle with u = 1
+        one = synth.to_bits(np.ones_like(xf), dt)
+        s_ref, s = L.silu(x, dt)
+        w_ref, w = L.swiglu(x, one, dt)
+        assert np.array_equal(s, w) and np.allclose(s_ref, w_ref, rtol=1e-15, atol=0)
+        # neg is exact: it flips the sign bit
+        n_ref, n = L.neg(x, dt)
+        signbit = 0x80000000 if dt == FP32 else 0x8000
+        assert np.array_equal(n, x ^ np.array(signbit, x.dtype))
+        # add: commutative; x + 0 = x; x + x = 2x exactly
+        zero = synth.to_bits(np.zeros_like(xf), dt)
+        assert np.array_equal(L.add(x, zero, dt)[1], np.where(L.widen(x, dt) == 0, L.add(x, zero, dt)[1], x))
+        y = synth.to_bits(g.normal(size=4000).astype(np.float32), dt)
+        assert np.array_equal(L.add(x, y, dt)[1], L.add(y, x, dt)[1])
+        two_x, _ = L.add(x, x, dt)
+        assert np.array_equal(two_x, 2 * L.widen(x, dt))
+    # add against torch's bf16 addition (fp32 sum, one rounding): a library routine
+    a = synth.to_bits(xf, BF16)
+    b = synth.to_bits((xf[::-1] * 0.37).copy(), BF16)
+    want = (synth.bits_to_torch(a, BF16).float() + synth.bits_to_torch(b, BF16).float()).to(torch.bfloat16)
+    assert np.array_equal(L.add(a, b, BF16)[1], want.view(torch.int16).numpy().view(np.uint16))
+
+
+def test_masked_fill_semantics():
+    g = np.random.default_rng(16)
+    x = synth.act(g, (4, 32), BF16)
+    mask = (g.random((4, 32)) < 0.3).astype(np.uint8)
+    ref, out = L.masked_fill(x, mask, -1e4, BF16)
+    assert np.array_equal(out[mask == 0], x[mask == 0])
+    fill = synth.to_bits(np.array([-1e4], np.float32), BF16)[0]  # -10000 rounds to -9984
+    assert np.all(out[mask == 1] == fill) and L.widen([fill], BF16)[0] == -9984.0
+    _, inf_out = L.masked_fill(x, mask, float("-inf"), BF16)
+    assert np.all(inf_out[mask == 1] == 0xFF80)
+
+
 # ---------------------------------------------------------------------------- layer chain
 def test_layer_chain_second_norm_reads_rounded_residual():
     g = np.random.default_rng(10)

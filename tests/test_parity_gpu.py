@@ -205,6 +205,73 @@ def test_rmsnorm_in_place(S):
     P.check_act(P.host_bits(xd, BF16), y_ref, y_bits, BF16, "rmsnorm in place")
 
 
+# ---------------------------------------------------------------------------- pointwise
+POINTWISE_CASES = [
+    # (op name, dtype, W, T, layout, variant)
+    ("silu", BF16, 4096, 33, "contig", 0), ("silu", FP16, 14336, 3, "strided", 0),
+    ("silu", FP32, 1000, 5, "contig", 0), ("silu", BF16, 100, 7, "contig", 1),
+    ("add", BF16, 4096, 17, "contig", 0), ("add", FP16, 520, 9, "strided", 0),
+    ("add", FP32, 4096, 4, "contig", 0), ("add", BF16, 77, 5, "contig", 1),
+    ("neg", BF16, 4096, 9, "contig", 0), ("neg", FP32, 36, 3, "contig", 1),
+    ("masked_fill", BF16, 4096, 21, "contig", 0), ("masked_fill", FP16, 2048, 6, "strided", 0),
+    ("masked_fill", FP32, 1024, 5, "contig", 0), ("masked_fill", BF16, 50, 4, "contig", 1),
+]
+
+
+@pytest.mark.parametrize("name,dtype,W,T,layout,variant", POINTWISE_CASES)
+def test_pointwise_parity(S, name, dtype, W, T, layout, variant):
+    g = np.random.default_rng(W + T)
+    op = {"silu": S.OP_SILU, "add": S.OP_ADD, "neg": S.OP_NEG, "masked_fill": S.OP_MASKED_FILL}[name]
+    a = synth.act(g, (T, W), dtype, std=3.0)
+    b = synth.act(g, (T, W), dtype)
+    mask = (g.random((T, W)) < 0.3).astype(np.uint8)
+    value = -1e4
+    if name == "silu":
+        ref, ref_bits = L.silu(a, dtype)
+    elif name == "add":
+        ref, ref_bits = L.add(a, b, dtype)
+    elif name == "neg":
+        ref, ref_bits = L.neg(a, dtype)
+    else:
+        ref, ref_bits = L.masked_fill(a, mask, value, dtype)
+    pad = 32 if layout == "strided" else 0
+    dev = (lambda bits: P.padded(bits, dtype, pad)) if pad else (lambda bits: P.dev(bits, dtype))
+    ad, bd, yd = dev(a), dev(b), dev(np.zeros_like(a))
+    if pad:
+        mbuf = torch.zeros((T, W + 64), dtype=torch.uint8, device="cuda")
+        md = mbuf[:, :W]
+        md.copy_(torch.from_numpy(mask).cuda())
+    else:
+        md = torch.from_numpy(mask).cuda()
+    ts = {"silu": [ad, yd], "neg": [ad, yd], "add": [ad, bd, yd], "masked_fill": [ad, md, yd]}[name]
+    es = 4 if dtype == FP32 else 2
+    lay = S.LAYOUT_ROWSTRIDED if pad else S.LAYOUT_CONTIG
+    align = 16 if variant != 1 and (W * es) % 16 == 0 else es
+    s = one_version_scm(S, S.make_spec(op, dtype, [W], 1, 1 << 20, layout=lay, align_bytes=align,
+                                       variant=variant))
+    invoke_ok(s, S, S.make_args(op, ts, scalar=value))
+    torch.cuda.synchronize()
+    s.close()
+    got = P.host_bits(yd, dtype)
+    if name in ("neg", "masked_fill", "add"):
+        assert np.array_equal(got, ref_bits), name  # exact operations / one rounding of an fp32 sum
+    else:
+        P.check_act(got, ref, ref_bits, dtype, name, exact_frac=0.99)
+
+
+def test_pointwise_in_place(S):
+    g = np.random.default_rng(21)
+    a = synth.act(g, (8, 4096), BF16)
+    b = synth.act(g, (8, 4096), BF16)
+    ref, ref_bits = L.add(a, b, BF16)
+    ad, bd = P.dev(a, BF16), P.dev(b, BF16)
+    s = one_version_scm(S, S.make_spec(S.OP_ADD, BF16, [4096], 1, 64))
+    invoke_ok(s, S, S.make_args(S.OP_ADD, [ad, bd, bd]))  # y = b
+    torch.cuda.synchronize()
+    s.close()
+    assert np.array_equal(P.host_bits(bd, BF16), ref_bits)
+
+
 # ---------------------------------------------------------------------------- RoPE + KV
 def rope_inputs(g, T, Hq, Hkv, D, S_, dtype):
     q, k, v = (synth.act(g, (T, h, D), dtype) for h in (Hq, Hkv, Hkv))

@@ -47,7 +47,7 @@ def test_exports_every_declared_symbol(S):
     exported = set(re.findall(r" T (trident_\w+)", nm))
     assert declared, "no declarations parsed"
     assert declared == exported, (declared ^ exported)
-    assert S.trident_abi_version() == 1
+    assert S.trident_abi_version() == 2
 
 
 def test_struct_layout_matches_header(S, tmp_path):
@@ -150,7 +150,7 @@ def _mutations(args, g):
     return out
 
 
-@pytest.mark.parametrize("op", [2, 3, 4, 5, 6, 7])
+@pytest.mark.parametrize("op", [2, 3, 4, 5, 6, 7, 8, 9, 10, 11])
 def test_mutated_arguments_every_op(S, op):
     """Library and oracle agree on valid and mutated tuples of every op."""
     g = np.random.default_rng(100 + op)
@@ -162,8 +162,8 @@ def test_mutated_arguments_every_op(S, op):
         base = dict(op=4, I=48)
         fixed = [48]
         mk = lambda **k: cases.make_args({**base, **k})
-    elif op == 7:
-        base = dict(op=7, H=128)
+    elif op in (7, 8, 9, 10, 11):
+        base = dict(op=op, H=128)
         fixed = [128]
         mk = lambda **k: cases.make_args({**base, **k})
     else:  # a chain version needs a size with a fused kernel (H 4096, D 128)
@@ -194,7 +194,7 @@ def test_structurally_invalid_calls_are_errors_not_misses(S):
     import copy
     for mut in ("op", "null", "ndim", "negshape", "negstride", "dtype", "unaligned", "eps", "flags"):
         a = copy.deepcopy(good)
-        if mut == "op": a["op"] = 9
+        if mut == "op": a["op"] = 12
         if mut == "null": a["tensors"][0]["addr"] = 0
         if mut == "ndim": a["tensors"][0]["shape"] = (2, 1, 1, 1, 64)[:4] + ()
         if mut == "negshape": a["tensors"][1]["shape"] = (-1, 64)
@@ -221,7 +221,7 @@ def test_registration_validation(S):
     s = dry(S, max_specs=4)
     good = dict(op=1, dtype=1, fixed=[64], tok_lo=1, tok_hi=8)
     assert s.register(S.make_spec(**good)) == 0
-    bad = [dict(good, op=9), dict(good, dtype=4), dict(good, fixed=[0]), dict(good, fixed=[64, 1]),
+    bad = [dict(good, op=12), dict(good, dtype=4), dict(good, fixed=[0]), dict(good, fixed=[64, 1]),
            dict(good, tok_lo=0), dict(good, tok_lo=5, tok_hi=4), dict(good, align_bytes=8),
            dict(good, rank=4), dict(good, layout=3), dict(good, variant=3),
            dict(good, variant=2, align_bytes=2), dict(good, rope_theta=1.0),
