@@ -670,6 +670,77 @@ def bench_motivation(c, warmup=20, rounds=5, repeats=10):
     return res
 
 
+def bench_kernels(c, n_calls=30):
+    """The paper's kernel-benchmark method (§4.1) on this library's FlagGems-style operators
+    (rms_norm, silu, add, neg, masked_fill), five shapes from LLM dimensions each: 30
+    consecutive calls, the first reported as cold, the median of the rest as warm; host
+    latency (until the call returns) and end-to-end latency (until the GPU finishes). The SCM
+    writes into preallocated outputs; torch eager allocates its results (as the eager
+    wrapper the paper compares against does). Per operator the arithmetic mean of the
+    per-shape warm ratios eager / SCM, as the paper aggregates (§4.2)."""
+    t, S, synth = c.torch, c.S, c.synth
+    F = t.nn.functional
+    shapes = [(1, 4096), (16, 4096), (128, 4096), (1024, 4096), (256, 14336)]
+    ops = ["rms_norm", "silu", "add", "neg", "masked_fill"]
+    out = {}
+
+    def timed(fn, n):
+        host, e2e = [], []
+        for _ in range(n):
+            t.cuda.synchronize()
+            h0 = time.perf_counter()
+            fn()
+            h1 = time.perf_counter()
+            t.cuda.synchronize()
+            h2 = time.perf_counter()
+            host.append((h1 - h0) * 1e6)
+            e2e.append((h2 - h0) * 1e6)
+        return dict(cold_host_us=round(host[0], 2), cold_e2e_us=round(e2e[0], 2),
+                    warm_host_us=round(float(np.median(host[1:])), 3),
+                    warm_e2e_us=round(float(np.median(e2e[1:])), 3))
+
+    seed = 70
+    for name in ops:
+        rows = []
+        for (T, W) in shapes:
+            seed += 1
+            x = synth.act_device((T, W), S.BF16, seed, c.dev)
+            b = synth.act_device((T, W), S.BF16, seed + 1000, c.dev)
+            mask = t.rand((T, W), device=c.dev) < 0.3
+            y = t.empty_like(x)
+            w32 = synth.gamma_device(W, seed + 2000, c.dev).to(t.bfloat16).float()
+            w_bf = w32.to(t.bfloat16)
+            op = {"rms_norm": S.OP_RMSNORM, "silu": S.OP_SILU, "add": S.OP_ADD, "neg": S.OP_NEG,
+                  "masked_fill": S.OP_MASKED_FILL}[name]
+            ts = {"rms_norm": [x, w32, y], "silu": [x, y], "add": [x, b, y], "neg": [x, y],
+                  "masked_fill": [x, mask.view(t.uint8), y]}[name]
+            eager = {"rms_norm": lambda: F.rms_norm(x, (W,), weight=w_bf, eps=1e-6),
+                     "silu": lambda: F.silu(x), "add": lambda: t.add(x, b), "neg": lambda: t.neg(x),
+                     "masked_fill": lambda: x.masked_fill(mask, -1e4)}[name]
+            r0 = time.perf_counter()
+            scm = S.Scm(device=c.dev.index or 0)
+            scm.register(S.make_spec(op, S.BF16, [W], 1, 1 << 20))
+            reg_us = (time.perf_counter() - r0) * 1e6
+            a = S.make_args(op, ts, eps=1e-6, scalar=-1e4)
+            inv, addr = c.invoker(scm), ctypes.addressof(a)
+            ours = timed(lambda: inv(addr), n_calls)
+            assert_all_hit(scm, name)
+            c.launches += n_calls
+            diff = float((y.float() - eager().float()).abs().max())
+            ref = timed(eager, n_calls)
+            scm.close()
+            rows.append(dict(shape=[T, W], scm=ours, scm_register_us=round(reg_us, 1), torch_eager=ref,
+                             speedup_host=round(ref["warm_host_us"] / ours["warm_host_us"], 3),
+                             speedup_e2e=round(ref["warm_e2e_us"] / ours["warm_e2e_us"], 3),
+                             max_abs_diff_vs_eager=diff))
+        out[name] = dict(shapes=rows,
+                         mean_speedup_host=round(float(np.mean([r["speedup_host"] for r in rows])), 3),
+                         mean_speedup_e2e=round(float(np.mean([r["speedup_e2e"] for r in rows])), 3))
+    out["paper_h800_context"] = ("21 FlagGems ops, Trident vs eager: mean 1.10x host, 1.07x e2e; silu 1.74x host, "
+                                 "1.73x e2e; masked_fill 1.67x e2e (§4.2)")
+    return out
+
+
 def bench_sweep(c, reps=20, quick=False):
     """HBM bandwidth sweep: add+RMSNorm (H 8192) and SwiGLU (I 28672) at T = 2^0..2^15,
     bf16. Each size: `reps` back-to-back launches from one native call, rotating across
@@ -819,6 +890,9 @@ def run_ours(a):
     if rank == 0 and want("motivation"):
         progress("motivation microbenchmark")
         extra["motivation_rms_norm"] = bench_motivation(c)
+    if rank == 0 and want("kernels"):
+        progress("kernel benchmark (paper method)")
+        extra["kernel_benchmark"] = bench_kernels(c)
     if rank == 0 and want("sweep"):
         progress("hbm sweep")
         extra["hbm_sweep"] = bench_sweep(c, quick=a.quick)
@@ -921,7 +995,8 @@ def main():
     p.add_argument("--impl", default="ours", choices=["ours", "reference"])
     p.add_argument("--quick", action="store_true", help="smaller sections (for smoke runs)")
     p.add_argument("--sections", default="all",
-                   help="comma list of: layers,qwen3,host,stress,motivation,sweep,roofline,e2e,cpu (default all;"
+                   help="comma list of: layers,qwen3,host,stress,motivation,kernels,sweep,roofline,e2e,cpu"
+                        " (default all;"
                         " the headline always runs)")
     a = p.parse_args()
     if a.warmup < 3:
