@@ -163,6 +163,8 @@ typedef enum trident_variant {
 #define TRIDENT_OPT_NO_ALIAS_CHECK 0x2 /* skip the output-overlap launch precondition */
 #define TRIDENT_OPT_PDL 0x4            /* launch with programmatic stream serialisation */
 #define TRIDENT_OPT_TIMING 0x8         /* record host ns per hit (trident_scm_host_times) */
+#define TRIDENT_OPT_FAIL_LAUNCHES 0x10 /* fault injection on the host, for tests: every launch
+                                          step of a hit reports ERR_CUDA without launching */
 
 /* ---------------------------------------------------------------- structs */
 /* Caller-owned tensor descriptor (DLPack-like, §3.4: tensors cross the boundary as

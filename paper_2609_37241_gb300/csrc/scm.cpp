@@ -899,7 +899,8 @@ TRIDENT_API int32_t trident_scm_create(const trident_scm_options* opt, trident_c
   if (o.max_specs < 1 || o.max_specs > 4096) return fail(TRIDENT_ERR_INVALID, "max_specs must be 1..4096");
   if (o.timing_ring == 0) o.timing_ring = 65536;
   if (o.timing_ring < 1 || o.timing_ring > (1 << 24)) return fail(TRIDENT_ERR_INVALID, "timing_ring");
-  if (o.flags & ~(TRIDENT_OPT_DRY_RUN | TRIDENT_OPT_NO_ALIAS_CHECK | TRIDENT_OPT_PDL | TRIDENT_OPT_TIMING))
+  if (o.flags & ~(TRIDENT_OPT_DRY_RUN | TRIDENT_OPT_NO_ALIAS_CHECK | TRIDENT_OPT_PDL | TRIDENT_OPT_TIMING |
+                  TRIDENT_OPT_FAIL_LAUNCHES))
     return fail(TRIDENT_ERR_INVALID, "unknown option flags");
   if (o.device < 0) return fail(TRIDENT_ERR_INVALID, "device");
   trident_scm* s = new (std::nothrow) trident_scm();
@@ -1019,6 +1020,10 @@ TRIDENT_API int32_t trident_scm_invoke(trident_scm_t* scm, const trident_args* a
   int32_t st = dispatch(scm, args, &oi, &s, &sel, !(scm->opt.flags & TRIDENT_OPT_NO_ALIAS_CHECK));
   if (st == TRIDENT_OK) {
     const Version& v = scm->versions[sel];
+    if (scm->opt.flags & TRIDENT_OPT_FAIL_LAUNCHES) {  // injected failure of P_i
+      if (out_selected) *out_selected = sel;
+      return count_error(scm, fail(TRIDENT_ERR_CUDA, "launch failure injected (TRIDENT_OPT_FAIL_LAUNCHES)"));
+    }
     if (!scm->dry) {
       st = do_launch(scm, v, args, s, stream);
       if (st != TRIDENT_OK) return count_error(scm, st);  // Algorithm 1: raise, no next version

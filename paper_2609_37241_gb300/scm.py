@@ -21,7 +21,7 @@ OP_RMSNORM = 7
 OP_SILU, OP_ADD, OP_NEG, OP_MASKED_FILL = 8, 9, 10, 11
 LAYOUT_CONTIG, LAYOUT_ROWSTRIDED, LAYOUT_ANY = 0, 1, 2
 VARIANT_AUTO, VARIANT_GENERIC, VARIANT_VECTOR = 0, 1, 2
-OPT_DRY_RUN, OPT_NO_ALIAS_CHECK, OPT_PDL, OPT_TIMING = 0x1, 0x2, 0x4, 0x8
+OPT_DRY_RUN, OPT_NO_ALIAS_CHECK, OPT_PDL, OPT_TIMING, OPT_FAIL_LAUNCHES = 0x1, 0x2, 0x4, 0x8, 0x10
 DEVERR_POS = 0x1
 MAX_TENSORS, MAX_FIXED = 20, 8
 OP_NTENSORS = {1: 5, 2: 6, 3: 8, 4: 3, 5: 18, 6: 20, 7: 3, 8: 2, 9: 3, 10: 2, 11: 3}

@@ -412,3 +412,27 @@ def test_fastcall_shim_matches_ctypes(S):
     with pytest.raises(TypeError):
         fc.invoke(h, ctypes.addressof(hit), None)
     s.close()
+
+
+def test_execution_error_is_raised_not_retried(S):
+    """Algorithm 1 (§3.2): when the selected P_i fails, the error propagates at once -- no
+    later version is tried, the compile hook is not called, nothing is registered (§3.5).
+    The failure is injected on the host (no GPU fault)."""
+    calls = []
+    s = dry(S, hook=lambda scm, args, stream: calls.append(1), flags=S.OPT_FAIL_LAUNCHES)
+    s.register(S.make_spec(1, 1, [64], 1, 8))
+    s.register(S.make_spec(1, 1, [64], 1, 8))  # a second matching version is never reached
+    a = cases.lib_args(cases.make_args({"op": 1, "T": 4, "H": 64}))
+    st, sel = s.invoke(a)
+    assert st == S.ERR_CUDA and sel == 0
+    assert "injected" in S.trident_scm_last_error()
+    stt = s.stats()
+    assert (stt.hits, stt.misses, stt.err_cuda, stt.hook_calls, stt.num_specs) == (0, 0, 1, 0, 2)
+    assert not calls
+    # a miss still takes the hook path, and an error inside a sequence stops it
+    miss = cases.lib_args(cases.make_args({"op": 1, "T": 40, "H": 64}))
+    assert s.invoke(miss) == (S.MISS_HANDLED, -1) and len(calls) == 1
+    arr = (S.trident_args * 3)(miss, a, miss)
+    st, sels = S.trident_scm_invoke_seq(s.h, arr)
+    assert st == S.ERR_CUDA and sels == [-1, 0, S.NOT_RUN] and len(calls) == 2
+    s.close()
