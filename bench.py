@@ -486,7 +486,31 @@ def bench_host_hit(c, n=1000):
     ns = np.array(ns[-n:], np.float64)
     c.launches += n
     s.close()
-    return dict(hits_on_bf16_contig=int(hits[3]), calls=n, selected=sel.value,
+    # the fused layer chain (18 tensors, 64 tokens): host ns per hit with the launch, and alone
+    cfg = synth.LLAMA
+    sets = ChainSets(c, cfg, HEADLINE_T, min_bytes=0, max_sets=1)
+    chain_ns = {}
+    for label, flags in (("live", S.OPT_TIMING | S.OPT_PDL), ("guards_only", S.OPT_TIMING | S.OPT_DRY_RUN)):
+        cs = layer_scm(c, cfg) if label == "live" else None
+        if cs is not None:
+            cs.close()
+        cs = S.Scm(device=c.dev.index or 0, flags=flags)
+        fixed = [cfg[k] for k in ("H", "Hq", "Hkv", "D", "S", "I")]
+        cs.register(S.make_spec(S.OP_LAYER_CHAIN, S.BF16, fixed, 1, 4096, layout=S.LAYOUT_ROWSTRIDED,
+                                rope_theta=cfg["theta"]))
+        ca = sets.fused_args(c, 0)
+        cinv, caddr = c.invoker(cs), ctypes.addressof(ca)
+        for _ in range(n + 50):
+            cinv(caddr)
+        t.cuda.synchronize()
+        cns = np.array(S.trident_scm_host_times(cs.h, n)[1], np.float64)
+        chain_ns[label] = dict(median_ns=float(np.median(cns)), p99_ns=float(np.percentile(cns, 99)))
+        if label == "live":
+            assert_all_hit(cs, "chain host")
+            c.launches += n + 50
+        cs.close()
+    del sets
+    return dict(hits_on_bf16_contig=int(hits[3]), calls=n, selected=sel.value, layer_chain=chain_ns,
                 median_ns=float(np.median(ns)), p99_ns=float(np.percentile(ns, 99)),
                 min_ns=float(ns.min()), guards_only_median_ns=float(np.median(dns)),
                 python_call_us_ctypes=round((h1 - h0) * 1e6 / n, 3), python_call_us_fastcall=fast_us)

@@ -211,35 +211,6 @@ struct Sig {
   int64_t fixed[TRIDENT_MAX_FIXED];
 };
 
-// Structural validation: everything that makes a call malformed rather than a miss.
-int32_t validate(const trident_args* a, const OpInfo** info) {
-  if (!a) return fail(TRIDENT_ERR_INVALID, "args is NULL");
-  if (a->op < 1 || a->op > kMaxOp) return fail(TRIDENT_ERR_INVALID, "unknown op %d", a->op);
-  const OpInfo& oi = g_ops[a->op];
-  if (a->ntensors != oi.nslots)
-    return fail(TRIDENT_ERR_INVALID, "op %d takes %d tensors, got %d", a->op, oi.nslots, a->ntensors);
-  if (a->flags != 0) return fail(TRIDENT_ERR_INVALID, "args.flags must be 0");
-  if (!(a->eps >= 0.0)) return fail(TRIDENT_ERR_INVALID, "eps must be >= 0");
-  for (int i = 0; i < oi.nslots; ++i) {
-    const trident_tensor& t = a->t[i];
-    const int es = elem_size(t.dtype);
-    if (es == 0) return fail(TRIDENT_ERR_INVALID, "tensor %d: unknown dtype %d", i, t.dtype);
-    if (t.ndim < 1 || t.ndim > 4) return fail(TRIDENT_ERR_INVALID, "tensor %d: ndim %d", i, t.ndim);
-    if (t.device < -1) return fail(TRIDENT_ERR_INVALID, "tensor %d: device %d", i, t.device);
-    bool empty = false;
-    for (int d = 0; d < t.ndim; ++d) {
-      if (t.shape[d] < 0 || t.stride[d] < 0)
-        return fail(TRIDENT_ERR_INVALID, "tensor %d: negative shape or stride", i);
-      if (t.shape[d] == 0) empty = true;
-    }
-    const uintptr_t p = reinterpret_cast<uintptr_t>(t.data);
-    if (!p && !empty) return fail(TRIDENT_ERR_INVALID, "tensor %d: NULL data", i);
-    if (p % (uintptr_t)es != 0) return fail(TRIDENT_ERR_INVALID, "tensor %d: not element-aligned", i);
-  }
-  *info = &oi;
-  return TRIDENT_OK;
-}
-
 inline bool shape_is(const trident_tensor& t, std::initializer_list<int64_t> want) {
   int d = 0;
   for (int64_t w : want) {
@@ -249,45 +220,72 @@ inline bool shape_is(const trident_tensor& t, std::initializer_list<int64_t> wan
   return true;
 }
 
-void compute_sig(const trident_args* a, const OpInfo& oi, Sig* s) {
+// Structural validation -- everything that makes a call malformed rather than a miss --
+// fused with the per-tensor guarded properties (common device, dtypes, ranks, 16-byte
+// alignment) in one pass over the tensors; a second pass checks shapes and layouts against
+// the sizes read off the arguments. Returns ERR_INVALID for a malformed tuple.
+int32_t analyze(const trident_args* a, const OpInfo** info, Sig* s) {
+  if (!a) return fail(TRIDENT_ERR_INVALID, "args is NULL");
+  if (a->op < 1 || a->op > kMaxOp) return fail(TRIDENT_ERR_INVALID, "unknown op %d", a->op);
+  const OpInfo& oi = g_ops[a->op];
+  if (a->ntensors != oi.nslots)
+    return fail(TRIDENT_ERR_INVALID, "op %d takes %d tensors, got %d", a->op, oi.nslots, a->ntensors);
+  if (a->flags != 0) return fail(TRIDENT_ERR_INVALID, "args.flags must be 0");
+  if (!(a->eps >= 0.0)) return fail(TRIDENT_ERR_INVALID, "eps must be >= 0");
   const trident_tensor* t = a->t;
   const int n = oi.nslots;
-  // device
   s->device = t[0].device;
-  for (int i = 1; i < n; ++i)
-    if (t[i].device != s->device) { s->device = kMixed; break; }
-  // dtypes
   s->act_dtype = -1;
   s->aux_dtype_ok = true;
-  for (int i = 0; i < n; ++i) {
-    const Kind k = oi.kind[i];
-    if (is_act(k) || k == K_CACHE) {
-      if (s->act_dtype == -1) s->act_dtype = t[i].dtype;
-      else if (s->act_dtype != t[i].dtype) s->act_dtype = kMixed;
-    } else if (k == K_POS) {
-      s->aux_dtype_ok &= t[i].dtype == TRIDENT_I32;
-    } else if (k == K_MASK_H) {
-      s->aux_dtype_ok &= t[i].dtype == TRIDENT_U8;
-    } else {
-      s->aux_dtype_ok &= t[i].dtype == TRIDENT_FP32;
-    }
-  }
-  // ranks
   s->rank = t[0].ndim;
   const int act_rank = oi.flattening ? s->rank : 2;
   s->ranks_ok = !oi.flattening || s->rank == 2 || s->rank == 3;
-  for (int i = 0; i < n && s->ranks_ok; ++i) {
+  s->aligned16 = true;
+  for (int i = 0; i < n; ++i) {  // pass 1: validation and per-tensor properties
+    const trident_tensor& x = t[i];
+    const int es = elem_size(x.dtype);
+    if (es == 0) return fail(TRIDENT_ERR_INVALID, "tensor %d: unknown dtype %d", i, x.dtype);
+    if (x.ndim < 1 || x.ndim > 4) return fail(TRIDENT_ERR_INVALID, "tensor %d: ndim %d", i, x.ndim);
+    if (x.device < -1) return fail(TRIDENT_ERR_INVALID, "tensor %d: device %d", i, x.device);
+    bool empty = false;
+    for (int d = 0; d < x.ndim; ++d) {
+      if (x.shape[d] < 0 || x.stride[d] < 0)
+        return fail(TRIDENT_ERR_INVALID, "tensor %d: negative shape or stride", i);
+      if (x.shape[d] == 0) empty = true;
+    }
+    const uintptr_t ptr = reinterpret_cast<uintptr_t>(x.data);
+    if (!ptr && !empty) return fail(TRIDENT_ERR_INVALID, "tensor %d: NULL data", i);
+    if (ptr % (uintptr_t)es != 0) return fail(TRIDENT_ERR_INVALID, "tensor %d: not element-aligned", i);
+    if (x.device != t[0].device) s->device = kMixed;
     const Kind k = oi.kind[i];
+    if (is_act(k) || k == K_CACHE) {
+      if (s->act_dtype == -1) s->act_dtype = x.dtype;
+      else if (s->act_dtype != x.dtype) s->act_dtype = kMixed;
+    } else if (k == K_POS) {
+      s->aux_dtype_ok &= x.dtype == TRIDENT_I32;
+    } else if (k == K_MASK_H) {
+      s->aux_dtype_ok &= x.dtype == TRIDENT_U8;
+    } else {
+      s->aux_dtype_ok &= x.dtype == TRIDENT_FP32;
+    }
     const int want = (k == K_ACT_H || k == K_ACT_I || k == K_MASK_H) ? act_rank
                    : (k == K_HEADS_Q || k == K_HEADS_KV || k == K_CACHE) ? 3 : 1;
-    s->ranks_ok = t[i].ndim == want;
+    s->ranks_ok &= x.ndim == want;
+    // 16-byte alignment of every tensor the kernels move in 16-byte units (positions are
+    // read one element at a time and only need their natural alignment)
+    if (k != K_POS && s->aligned16) {
+      if (ptr % 16 != 0) s->aligned16 = false;
+      for (int d = 0; d + 1 < x.ndim; ++d)
+        if (x.shape[d] > 1 && (x.stride[d] * es) % 16 != 0) s->aligned16 = false;
+    }
   }
+  *info = &oi;
   s->shapes_ok = false;
   s->layout = -1;
   s->aux_layout_ok = false;
   for (int i = 0; i < TRIDENT_MAX_FIXED; ++i) s->fixed[i] = -1;
   s->T = -1;
-  if (!s->ranks_ok) return;
+  if (!s->ranks_ok) return TRIDENT_OK;
   // leading dims, T and the fixed sizes read off the arguments
   if (oi.flattening && s->rank == 3) {
     s->nlead = 2;
@@ -322,59 +320,43 @@ void compute_sig(const trident_args* a, const OpInfo& oi, Sig* s) {
       s->fixed[5] = I;
     }
   }
+  // pass 2: shapes, the layout class over the activation-like rows, and the auxiliary
+  // layouts (gamma and pos dense, caches dense [Hkv, S, D])
   const int64_t T0 = s->lead[0];
-  bool ok = true;
-  for (int i = 0; i < n && ok; ++i) {
+  bool shapes = true, all_contig = true, none = false, aux = true;
+  for (int i = 0; i < n; ++i) {
     const trident_tensor& x = t[i];
-    switch (oi.kind[i]) {
+    const Kind k = oi.kind[i];
+    switch (k) {
       case K_ACT_H: case K_ACT_I: case K_MASK_H: {
-        const int64_t w = oi.kind[i] == K_ACT_I ? I : H;
-        ok = s->nlead == 2 ? shape_is(x, {s->lead[0], s->lead[1], w}) : shape_is(x, {T0, w});
+        const int64_t w = k == K_ACT_I ? I : H;
+        shapes &= s->nlead == 2 ? shape_is(x, {s->lead[0], s->lead[1], w}) : shape_is(x, {T0, w});
         break;
       }
-      case K_GAMMA_H: ok = shape_is(x, {H}); break;
-      case K_GAMMA_D: ok = shape_is(x, {D}); break;
-      case K_HEADS_Q: ok = shape_is(x, {T0, Hq, D}); break;
-      case K_HEADS_KV: ok = shape_is(x, {T0, Hkv, D}); break;
-      case K_POS: ok = shape_is(x, {T0}); break;
-      case K_CACHE: ok = shape_is(x, {Hkv, S, D}); break;
+      case K_GAMMA_H: shapes &= shape_is(x, {H}); break;
+      case K_GAMMA_D: shapes &= shape_is(x, {D}); break;
+      case K_HEADS_Q: shapes &= shape_is(x, {T0, Hq, D}); break;
+      case K_HEADS_KV: shapes &= shape_is(x, {T0, Hkv, D}); break;
+      case K_POS: shapes &= shape_is(x, {T0}); break;
+      case K_CACHE: shapes &= shape_is(x, {Hkv, S, D}); break;
+    }
+    if (is_rowlike(k)) {
+      const Rows r = rows_of(x, k);
+      if (!r.packed) none = true;
+      else if (r.n > 1) {
+        if (r.stride < r.width) none = true;
+        else if (r.stride != r.width) all_contig = false;
+      }
+    } else if (k == K_GAMMA_H || k == K_GAMMA_D || k == K_POS) {
+      aux &= x.shape[0] <= 1 || x.stride[0] == 1;
+    } else if (k == K_CACHE) {
+      aux &= x.stride[0] == S * D && x.stride[1] == D && x.stride[2] == 1;
     }
   }
-  s->shapes_ok = ok;
-  // layout class over the activations
-  bool all_contig = true, none = false;
-  for (int i = 0; i < n; ++i) {
-    if (!is_rowlike(oi.kind[i])) continue;
-    const Rows r = rows_of(t[i], oi.kind[i]);
-    if (!r.packed) { none = true; break; }
-    if (r.n <= 1) continue;
-    if (r.stride < r.width) { none = true; break; }
-    if (r.stride != r.width) all_contig = false;
-  }
+  s->shapes_ok = shapes;
   s->layout = none ? -1 : (all_contig ? TRIDENT_LAYOUT_CONTIG : TRIDENT_LAYOUT_ROWSTRIDED);
-  // gamma and pos dense, caches dense [Hkv, S, D]
-  bool aux = true;
-  for (int i = 0; i < n && aux; ++i) {
-    const Kind k = oi.kind[i];
-    if (k == K_GAMMA_H || k == K_GAMMA_D || k == K_POS) aux = t[i].shape[0] <= 1 || t[i].stride[0] == 1;
-    else if (k == K_CACHE)
-      aux = t[i].stride[0] == S * D && t[i].stride[1] == D && t[i].stride[2] == 1;
-  }
   s->aux_layout_ok = aux;
-}
-
-// 16-byte alignment of every tensor the kernels move in 16-byte units (positions are
-// read one element at a time and only need their natural alignment).
-bool aligned16(const trident_args* a, const OpInfo& oi) {
-  for (int i = 0; i < oi.nslots; ++i) {
-    if (oi.kind[i] == K_POS) continue;
-    const trident_tensor& t = a->t[i];
-    if (reinterpret_cast<uintptr_t>(t.data) % 16 != 0) return false;
-    const int es = elem_size(t.dtype);
-    for (int d = 0; d + 1 < t.ndim; ++d)
-      if (t.shape[d] > 1 && (t.stride[d] * es) % 16 != 0) return false;
-  }
-  return true;
+  return TRIDENT_OK;
 }
 
 // ------------------------------------------------------------------ versions
@@ -421,8 +403,7 @@ struct trident_scm {
 
 namespace {
 
-bool guard_holds(const Version& v, const Sig& s, const trident_args* a, const OpInfo& oi,
-                 int* aligned_cache) {
+bool guard_holds(const Version& v, const Sig& s, const trident_args* a) {
   const trident_spec_desc& d = v.d;
   if (d.device != s.device || d.dtype != s.act_dtype || !s.aux_dtype_ok) return false;
   if (d.rank != s.rank || !s.ranks_ok || !s.shapes_ok) return false;
@@ -432,10 +413,7 @@ bool guard_holds(const Version& v, const Sig& s, const trident_args* a, const Op
   if (s.T < d.tok_lo || s.T > d.tok_hi) return false;
   if (s.layout < 0 || (d.layout != TRIDENT_LAYOUT_ANY && d.layout != s.layout)) return false;
   if (!s.aux_layout_ok) return false;
-  if (d.align_bytes == 16) {
-    if (*aligned_cache < 0) *aligned_cache = aligned16(a, oi) ? 1 : 0;
-    if (!*aligned_cache) return false;
-  }
+  if (d.align_bytes == 16 && !s.aligned16) return false;
   return true;
 }
 
@@ -481,10 +459,14 @@ bool same_desc(const trident_tensor& x, const trident_tensor& y) {
 
 // Launch precondition (checked after a hit, before the launch): no output shares a byte
 // with another slot unless the two are the same tensor in one of the op's in-place groups.
+// Slots are sorted by the start of their byte extent and swept once, so only pairs whose
+// extents intersect (views into one buffer, in practice) reach the exact row test.
 int32_t check_overlap(const trident_args* a, const OpInfo& oi) {
   const int n = oi.nslots;
   int64_t base[TRIDENT_MAX_TENSORS], nr[TRIDENT_MAX_TENSORS], w[TRIDENT_MAX_TENSORS],
-      rs[TRIDENT_MAX_TENSORS];
+      rs[TRIDENT_MAX_TENSORS], end[TRIDENT_MAX_TENSORS];
+  int order[TRIDENT_MAX_TENSORS];
+  int m = 0;
   for (int i = 0; i < n; ++i) {
     const Rows r = rows_of(a->t[i], oi.kind[i]);
     const int es = elem_size(a->t[i].dtype);
@@ -492,14 +474,24 @@ int32_t check_overlap(const trident_args* a, const OpInfo& oi) {
     nr[i] = r.n;
     w[i] = r.width * es;
     rs[i] = r.stride * es;
+    if (nr[i] <= 0 || w[i] <= 0) continue;  // no bytes: overlaps nothing
+    end[i] = base[i] + (nr[i] - 1) * rs[i] + w[i];
+    int k = m++;  // insertion sort by extent start
+    while (k > 0 && base[order[k - 1]] > base[i]) {
+      order[k] = order[k - 1];
+      --k;
+    }
+    order[k] = i;
   }
-  for (int i = 0; i < n; ++i) {
-    if (!oi.out[i]) continue;
-    for (int j = 0; j < n; ++j) {
-      if (j == i) continue;
+  for (int x = 0; x < m; ++x) {
+    const int i = order[x];
+    for (int y = x + 1; y < m && base[order[y]] < end[i]; ++y) {  // extents intersect
+      const int j = order[y];
+      if (!oi.out[i] && !oi.out[j]) continue;  // inputs may share bytes
       if (!rows_overlap(base[i], nr[i], w[i], rs[i], base[j], nr[j], w[j], rs[j])) continue;
       if (oi.group[i] != 0 && oi.group[i] == oi.group[j] && same_desc(a->t[i], a->t[j])) continue;
-      return fail(TRIDENT_ERR_INVALID, "output tensor %d overlaps tensor %d", i, j);
+      const int o = oi.out[i] ? i : j;
+      return fail(TRIDENT_ERR_INVALID, "output tensor %d overlaps tensor %d", o, o == i ? j : i);
     }
   }
   return TRIDENT_OK;
@@ -696,16 +688,14 @@ int32_t do_launch(trident_scm* scm, const Version& v, const trident_args* a, con
 int32_t dispatch(const trident_scm* scm, const trident_args* a, const OpInfo** oi_out, Sig* s,
                  int32_t* sel, bool check_alias) {
   const OpInfo* oi = nullptr;
-  int32_t st = validate(a, &oi);
+  int32_t st = analyze(a, &oi, s);
   if (st != TRIDENT_OK) return st;
   *oi_out = oi;
-  compute_sig(a, *oi, s);
   const int32_t n = scm->count.load(std::memory_order_acquire);
-  int aligned = -1;
   for (int32_t i = 0; i < n; ++i) {
     const Version& v = scm->versions[i];
     if (v.d.op != a->op) continue;
-    if (!guard_holds(v, *s, a, *oi, &aligned)) continue;
+    if (!guard_holds(v, *s, a)) continue;
     if (check_alias) {
       st = check_overlap(a, *oi);
       if (st != TRIDENT_OK) return st;
@@ -842,12 +832,11 @@ int32_t resolve_kernel(const trident_spec_desc& d, KernelEntry* ke) {
 int32_t trident::prepare_rope_args(const void* args_ptr, RopeParams* p, int32_t* dtype, bool* qknorm) {
   const trident_args* a = static_cast<const trident_args*>(args_ptr);
   const OpInfo* oi = nullptr;
-  int32_t st = validate(a, &oi);
+  Sig s;
+  int32_t st = analyze(a, &oi, &s);
   if (st != TRIDENT_OK) return st;
   if (a->op != TRIDENT_OP_ROPE_KV && a->op != TRIDENT_OP_QKNORM_ROPE_KV)
     return fail(TRIDENT_ERR_INVALID, "op %d is not a RoPE op", a->op);
-  Sig s;
-  compute_sig(a, *oi, &s);
   if (s.device == kMixed || s.device < 0) return fail(TRIDENT_ERR_INVALID, "tensors must share one CUDA device");
   if (s.act_dtype != TRIDENT_BF16 && s.act_dtype != TRIDENT_FP16)
     return fail(TRIDENT_ERR_INVALID, "activations must all be bf16 or all fp16");
@@ -855,7 +844,7 @@ int32_t trident::prepare_rope_args(const void* args_ptr, RopeParams* p, int32_t*
   if (!s.ranks_ok || !s.shapes_ok) return fail(TRIDENT_ERR_INVALID, "inconsistent ranks or shapes");
   if (s.T < 1) return fail(TRIDENT_ERR_INVALID, "no tokens");
   if (s.layout < 0 || !s.aux_layout_ok) return fail(TRIDENT_ERR_INVALID, "unsupported layout");
-  if (!aligned16(a, *oi)) return fail(TRIDENT_ERR_INVALID, "tensors must be 16-byte aligned");
+  if (!s.aligned16) return fail(TRIDENT_ERR_INVALID, "tensors must be 16-byte aligned");
   if (!(a->rope_theta > 0.0 && std::isfinite(a->rope_theta)))
     return fail(TRIDENT_ERR_INVALID, "rope_theta must be positive");
   st = check_overlap(a, *oi);
