@@ -491,9 +491,6 @@ def bench_host_hit(c, n=1000):
     sets = ChainSets(c, cfg, HEADLINE_T, min_bytes=0, max_sets=1)
     chain_ns = {}
     for label, flags in (("live", S.OPT_TIMING | S.OPT_PDL), ("guards_only", S.OPT_TIMING | S.OPT_DRY_RUN)):
-        cs = layer_scm(c, cfg) if label == "live" else None
-        if cs is not None:
-            cs.close()
         cs = S.Scm(device=c.dev.index or 0, flags=flags)
         fixed = [cfg[k] for k in ("H", "Hq", "Hkv", "D", "S", "I")]
         cs.register(S.make_spec(S.OP_LAYER_CHAIN, S.BF16, fixed, 1, 4096, layout=S.LAYOUT_ROWSTRIDED,
