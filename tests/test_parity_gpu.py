@@ -474,6 +474,28 @@ def test_layer_chain_fused_matches_oracle(S, cfg_name, T):
     check_chain(ref, out, inp)
 
 
+@pytest.mark.parametrize("dtype,H,Hq,I,T,qk", [
+    (FP16, 4096, 32, 14336, 4, False),     # fp16 chain
+    (BF16, 8192, 64, 28672, 3, False),     # H 8192 instantiation (4 vectors per thread)
+    (BF16, 8192, 64, 28672, 200, True),    # H 8192, grid beyond one wave: one block per token
+    (FP16, 8192, 64, 28672, 5, True),
+])
+def test_layer_chain_other_sizes_and_dtypes(S, dtype, H, Hq, I, T, qk):
+    cfg = dict(H=H, Hq=Hq, Hkv=8, D=128, S=2048, I=I, theta=1e6, qknorm=qk, eps=1e-6)
+    g = np.random.default_rng(H + T)
+    inp = synth.layer_inputs(g, T, cfg, dtype=dtype)
+    ref = L.layer_chain(inp, cfg["theta"], cfg["eps"], dtype, qknorm=qk)
+    op = S.OP_LAYER_CHAIN_QKNORM if qk else S.OP_LAYER_CHAIN
+    fixed = [H, Hq, 8, 128, 2048, I]
+    lay = S.LAYOUT_ROWSTRIDED if T > 1 else S.LAYOUT_CONTIG
+    s = one_version_scm(S, S.make_spec(op, dtype, fixed, 1, 4096, layout=lay, rope_theta=cfg["theta"]))
+    ts, out = chain_device(inp, dtype, qk)
+    invoke_ok(s, S, S.make_args(op, ts, eps=cfg["eps"], rope_theta=cfg["theta"]))
+    torch.cuda.synchronize()
+    s.close()
+    check_chain(ref, out, inp, dtype)
+
+
 @pytest.mark.parametrize("pdl", [False, True])
 def test_layer_chain_unfused_four_invokes_match(S, pdl):
     """The same layer as four invokes (one SCM, four versions) equals the oracle."""
