@@ -14,6 +14,7 @@ roofline of the dominant kernel, the end-to-end step with host copies, and the C
 oracle as a reported baseline.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl reference] [--quick]
+                 [--sections LIST] [--tokens LIST]
 """
 import argparse
 import ctypes
@@ -185,6 +186,15 @@ class Ctx:
         P = ctypes.POINTER(self.S.trident_args)
         return lambda addr, n: seq(hh, ctypes.cast(addr, P), n, spp, None)
 
+    def step_invoker(self, scm):
+        h, sp = scm.h.value, self.sp.value or 0
+        if self.fc is not None:
+            stp = self.fc.invoke_step
+            return lambda addr, n: stp(h, addr, n, sp)
+        stp, hh, spp = self.L.trident_scm_invoke_step, scm.h, self.sp
+        P = ctypes.POINTER(self.S.trident_args)
+        return lambda addr, n: stp(hh, ctypes.cast(addr, P), n, spp, None)
+
     def events(self):
         t = self.torch
         return t.cuda.Event(enable_timing=True), t.cuda.Event(enable_timing=True)
@@ -348,6 +358,16 @@ def bench_layer(c, cfg, T, K, W, layers=1, min_bytes=2 * L2_BYTES):
     fus_dev, fus_host = time_steps(c, f_fused, K, W)
     unf_dev, unf_host = time_steps(c, f_unf, K, W)
     c.launches += K * (n_launch[0] + n_launch[1])
+    step = None
+    if layers > 1:  # the same layers through invoke_step: independent chains, one launch
+        stp = c.step_invoker(scm)
+        before = scm.stats().fused_launches
+        step_dev, step_host = time_steps(c, lambda i: stp(fa[i % groups], layers), K, W)
+        per_step = -(-layers // S.STEP_MAX)
+        fused_n = scm.stats().fused_launches - before
+        assert fused_n == (K + W) * per_step, ("step launches not fused", fused_n)
+        c.launches += K * per_step
+        step = dict(us=round(step_dev, 3), host_us=round(step_host, 3), launches_per_step=per_step)
     # device throughput floor: the same launches issued from one native call
     nat = min(K, R if layers == 1 else R)
     if layers == 1:
@@ -368,6 +388,8 @@ def bench_layer(c, cfg, T, K, W, layers=1, min_bytes=2 * L2_BYTES):
                working_set_mb=round(R * chain_bytes_per_token(cfg) * T / 2 ** 20, 1))
     if nat_us is not None:
         res["fused_native_seq_us"] = round(nat_us, 3)
+    if step is not None:
+        res["one_launch_step"] = step
     return res, sets
 
 
@@ -898,7 +920,9 @@ def run_ours(a):
     if rank == 0 and want("qwen3"):
         progress("qwen3 36-layer steps")
         qw = {}
-        for T in ((1, 8, 32, 128) if not a.quick else (1, 128)):
+        toks = [int(x) for x in a.tokens.split(",")] if a.tokens else (
+            (1, 8, 32, 128) if not a.quick else (1, 128))
+        for T in toks:
             qw[str(T)], _ = bench_layer(c, synth.QWEN3, T, K=max(20, min(K, 2000) // 36), W=W,
                                         layers=36)
         extra["qwen3_36layer_step"] = qw
@@ -1015,6 +1039,7 @@ def main():
     p.add_argument("--warmup", type=int, default=20)
     p.add_argument("--impl", default="ours", choices=["ours", "reference"])
     p.add_argument("--quick", action="store_true", help="smaller sections (for smoke runs)")
+    p.add_argument("--tokens", default="", help="comma list of token counts for the qwen3 section")
     p.add_argument("--sections", default="all",
                    help="comma list of: layers,qwen3,host,stress,motivation,kernels,sweep,roofline,e2e,cpu"
                         " (default all;"

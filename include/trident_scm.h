@@ -34,7 +34,7 @@
 extern "C" {
 #endif
 
-#define TRIDENT_ABI_VERSION 2
+#define TRIDENT_ABI_VERSION 3
 #define TRIDENT_MAX_TENSORS 20
 #define TRIDENT_MAX_FIXED 8
 /* out_selected value for a sequence element that was not run (trident_scm_invoke_seq). */
@@ -233,6 +233,8 @@ typedef struct trident_scm_stats_t {
   uint64_t guard_evals;     /* versions whose guard was evaluated                    */
   int32_t num_specs;        /* versions in the current table                         */
   int32_t reserved;
+  uint64_t fused_launches;  /* invoke_step launches that ran several calls at once   */
+  uint64_t fused_calls;     /* calls run by those launches                           */
 } trident_scm_stats_t;
 
 typedef struct trident_scm trident_scm_t; /* opaque; owns the table, kernels and device state */
@@ -291,6 +293,29 @@ int32_t trident_scm_invoke(trident_scm_t* scm, const trident_args* args, void* s
  * if some misses were handled. */
 int32_t trident_scm_invoke_seq(trident_scm_t* scm, const trident_args* args, int32_t n,
                                void* stream, int32_t* out_selected);
+
+/* A decoder step's layer-chain calls with as few launches as the data allows: a step
+ * toward the mega-kernel systems that §5 of the paper discusses as related work (several
+ * operators per device launch), while keeping the paper's per-call guarded selection; the
+ * paper itself launches once per call. Same contract as trident_scm_invoke_seq -- statuses, out_selected,
+ * hook, statistics -- with one difference in how hits run: the calls are taken in chunks
+ * of up to 48 (TRIDENT_STEP_MAX); a chunk of two or more calls runs as ONE launch when
+ *   - every call hits (Algorithm 1, per call, including its launch preconditions),
+ *   - every selected version is a layer chain (LAYER_CHAIN or LAYER_CHAIN_QKNORM) with the
+ *     same kernel (same dtype, H and q/k-norm choice; theta may differ), and
+ *   - the calls are independent: no output byte of one call is a byte of any tensor of
+ *     another call (exact for row-strided views with equal strides, conservative
+ *     otherwise), so running them together equals running them in order.
+ * Otherwise the chunk runs call by call exactly as invoke_seq (so a miss, the hook and
+ * errors are reported at their position). Chunks run in order on `stream`. A fused chunk
+ * counts one invoke and one hit per call, plus fused_launches and fused_calls in the
+ * statistics; no host time is recorded for it. If its launch fails, the call returns
+ * ERR_CUDA with the chunk's out_selected set to the versions it selected and the calls
+ * after the chunk set to TRIDENT_NOT_RUN. Host cost of the independence test: one sort of
+ * the chunk's tensor extents (about 20 per call). */
+#define TRIDENT_STEP_MAX 48
+int32_t trident_scm_invoke_step(trident_scm_t* scm, const trident_args* args, int32_t n,
+                                void* stream, int32_t* out_selected);
 
 /* Selection only: validation plus Algorithm 1's guard loop, with no launch, no hook
  * and no statistics. Returns OK (*out_selected = index), MISS (-1) or ERR_INVALID.

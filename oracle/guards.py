@@ -329,6 +329,21 @@ def launch_precondition(args):
     return True
 
 
+def calls_independent(calls):
+    """Several argument tuples may run in any order -- and so in one launch -- iff no
+    output byte of one call is a byte of any tensor of another call (brute force over
+    byte sets, as launch_precondition does within one call)."""
+    sets = [[byte_set(t) for t in c["tensors"]] for c in calls]
+    for i, ci in enumerate(calls):
+        for j in range(len(calls)):
+            if j == i:
+                continue
+            for si, (_, _, out_i) in enumerate(SLOTS[ci["op"]]):
+                if out_i and any(sets[i][si] & other for other in sets[j]):
+                    return False
+    return True
+
+
 # ----------------------------------------------------------------------------- Algorithm 1
 def select(table, args, check_overlap=True):
     """Algorithm 1 over `table` (list of specs in creation order).

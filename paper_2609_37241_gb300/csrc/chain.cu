@@ -19,15 +19,12 @@ namespace trident {
 
 constexpr int kChainSwigluUnroll = 2;
 
-// Four resident blocks per SM for H 4096 (64 registers): the 64-token grid (576 blocks)
-// then fits one wave on 152 SMs; a fifth register would drop it to three blocks per SM.
+// Block b of one call's grid (b < nA + nB + nC).
 template <int DT, int VPT, int SPLIT, int D, bool QKNORM>
-__global__ void __launch_bounds__(kThreads, VPT == 2 ? 4 : 2) chain_kernel(const ChainParams c) {
-  pdl_prologue();
+__device__ __forceinline__ void chain_block(const ChainParams& c, const int b) {
   constexpr int EB = Act<DT>::BYTES;
   constexpr int VE = Act<DT>::VE;
   const int tid = threadIdx.x;
-  const int b = blockIdx.x;
   if (b < c.nA) {
     // Both norms of one token. The second residual sum s2 = attn_out + round(s1) is
     // elementwise, so both sums of squares are formed before any reduction and reduced
@@ -145,12 +142,41 @@ __global__ void __launch_bounds__(kThreads, VPT == 2 ? 4 : 2) chain_kernel(const
   }
 }
 
+// Four resident blocks per SM for H 4096 (64 registers): the 64-token grid (576 blocks)
+// then fits one wave on 152 SMs; a fifth register would drop it to three blocks per SM.
+template <int DT, int VPT, int SPLIT, int D, bool QKNORM>
+__global__ void __launch_bounds__(kThreads, VPT == 2 ? 4 : 2)
+    chain_kernel(const __grid_constant__ ChainParams c) {
+  pdl_prologue();
+  chain_block<DT, VPT, SPLIT, D, QKNORM>(c, blockIdx.x);
+}
+
+// Several independent calls in one launch: a block finds its call by binary search over
+// the first-block table (uniform across the block, so the parameter reads broadcast).
+template <int DT, int VPT, int SPLIT, int D, bool QKNORM>
+__global__ void __launch_bounds__(kThreads, VPT == 2 ? 4 : 2)
+    chain_step_kernel(const __grid_constant__ ChainStepParams p) {
+  pdl_prologue();
+  const int b = blockIdx.x;
+  int lo = 0, hi = p.n - 1;
+  while (lo < hi) {
+    const int mid = (lo + hi + 1) >> 1;
+    if (b >= p.first[mid]) lo = mid;
+    else hi = mid - 1;
+  }
+  chain_block<DT, VPT, SPLIT, D, QKNORM>(p.c[lo], b - p.first[lo]);
+}
+
 template <int DT, int SPLIT, bool QK>
-static const void* pick(int64_t H) {
+static void pick(int64_t H, const void** one, const void** step) {
   constexpr int per = kThreads * Act<DT>::VE;
-  if (H == per * 2) return (const void*)chain_kernel<DT, 2, SPLIT, 128, QK>;
-  if (H == per * 4) return (const void*)chain_kernel<DT, 4, SPLIT, 128, QK>;
-  return nullptr;
+  if (H == per * 2) {
+    *one = (const void*)chain_kernel<DT, 2, SPLIT, 128, QK>;
+    *step = (const void*)chain_step_kernel<DT, 2, SPLIT, 128, QK>;
+  } else if (H == per * 4) {
+    *one = (const void*)chain_kernel<DT, 4, SPLIT, 128, QK>;
+    *step = (const void*)chain_step_kernel<DT, 4, SPLIT, 128, QK>;
+  }
 }
 
 bool chain_kernel(int32_t dtype, int64_t H, int32_t D, bool qknorm, KernelEntry* out,
@@ -161,13 +187,25 @@ bool chain_kernel(int32_t dtype, int64_t H, int32_t D, bool qknorm, KernelEntry*
   out->vec = 8;
   out->unroll = kChainSwigluUnroll;
   // fn: two blocks per token for the norms; fn_inplace: one block per token (calls whose
-  // outputs overwrite inputs, and grids too large for one wave)
+  // outputs overwrite inputs, and grids too large for one wave); fn_step*: the same for
+  // several calls per launch
+  out->fn = out->fn_inplace = out->fn_step = out->fn_step_inplace = nullptr;
   if (dtype == DT_BF16) {
-    out->fn = qknorm ? pick<DT_BF16, 2, true>(H) : pick<DT_BF16, 2, false>(H);
-    out->fn_inplace = qknorm ? pick<DT_BF16, 1, true>(H) : pick<DT_BF16, 1, false>(H);
+    if (qknorm) {
+      pick<DT_BF16, 2, true>(H, &out->fn, &out->fn_step);
+      pick<DT_BF16, 1, true>(H, &out->fn_inplace, &out->fn_step_inplace);
+    } else {
+      pick<DT_BF16, 2, false>(H, &out->fn, &out->fn_step);
+      pick<DT_BF16, 1, false>(H, &out->fn_inplace, &out->fn_step_inplace);
+    }
   } else {
-    out->fn = qknorm ? pick<DT_FP16, 2, true>(H) : pick<DT_FP16, 2, false>(H);
-    out->fn_inplace = qknorm ? pick<DT_FP16, 1, true>(H) : pick<DT_FP16, 1, false>(H);
+    if (qknorm) {
+      pick<DT_FP16, 2, true>(H, &out->fn, &out->fn_step);
+      pick<DT_FP16, 1, true>(H, &out->fn_inplace, &out->fn_step_inplace);
+    } else {
+      pick<DT_FP16, 2, false>(H, &out->fn, &out->fn_step);
+      pick<DT_FP16, 1, false>(H, &out->fn_inplace, &out->fn_step_inplace);
+    }
   }
   if (!out->fn) { *why = "layer chain supports H in {4096, 8192}"; return false; }
   return true;

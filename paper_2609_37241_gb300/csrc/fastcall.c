@@ -24,11 +24,12 @@ static PyObject* fc_invoke(PyObject* self, PyObject* const* args, Py_ssize_t nar
   return PyLong_FromLong(trident_scm_invoke((trident_scm_t*)scm, (const trident_args*)a, stream, NULL));
 }
 
-/* invoke_seq(scm, args_address, n, stream) -> status */
-static PyObject* fc_invoke_seq(PyObject* self, PyObject* const* args, Py_ssize_t nargs) {
-  (void)self;
+typedef int32_t (*seq_fn)(trident_scm_t*, const trident_args*, int32_t, void*, int32_t*);
+
+/* (scm, args_address, n, stream) -> status of fn */
+static PyObject* call_seq(seq_fn fn, const char* usage, PyObject* const* args, Py_ssize_t nargs) {
   if (nargs != 4) {
-    PyErr_SetString(PyExc_TypeError, "invoke_seq(scm, args_address, n, stream)");
+    PyErr_SetString(PyExc_TypeError, usage);
     return NULL;
   }
   void* scm = PyLong_AsVoidPtr(args[0]);
@@ -36,13 +37,29 @@ static PyObject* fc_invoke_seq(PyObject* self, PyObject* const* args, Py_ssize_t
   long n = PyLong_AsLong(args[2]);
   void* stream = PyLong_AsVoidPtr(args[3]);
   if (PyErr_Occurred()) return NULL;
-  return PyLong_FromLong(
-      trident_scm_invoke_seq((trident_scm_t*)scm, (const trident_args*)a, (int32_t)n, stream, NULL));
+  if (n < 0 || n > INT32_MAX) {
+    PyErr_SetString(PyExc_ValueError, "n out of range");
+    return NULL;
+  }
+  return PyLong_FromLong(fn((trident_scm_t*)scm, (const trident_args*)a, (int32_t)n, stream, NULL));
+}
+
+/* invoke_seq(scm, args_address, n, stream) -> status */
+static PyObject* fc_invoke_seq(PyObject* self, PyObject* const* args, Py_ssize_t nargs) {
+  (void)self;
+  return call_seq(trident_scm_invoke_seq, "invoke_seq(scm, args_address, n, stream)", args, nargs);
+}
+
+/* invoke_step(scm, args_address, n, stream) -> status */
+static PyObject* fc_invoke_step(PyObject* self, PyObject* const* args, Py_ssize_t nargs) {
+  (void)self;
+  return call_seq(trident_scm_invoke_step, "invoke_step(scm, args_address, n, stream)", args, nargs);
 }
 
 static PyMethodDef methods[] = {
     {"invoke", (PyCFunction)(void (*)(void))fc_invoke, METH_FASTCALL, "trident_scm_invoke"},
     {"invoke_seq", (PyCFunction)(void (*)(void))fc_invoke_seq, METH_FASTCALL, "trident_scm_invoke_seq"},
+    {"invoke_step", (PyCFunction)(void (*)(void))fc_invoke_step, METH_FASTCALL, "trident_scm_invoke_step"},
     {NULL, NULL, 0, NULL}};
 
 static struct PyModuleDef module = {PyModuleDef_HEAD_INIT, "_fastcall", NULL, -1, methods,

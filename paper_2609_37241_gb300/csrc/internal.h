@@ -90,10 +90,23 @@ struct ChainParams {
   int64_t sw_tiles;  // T * sw_tiles_per_row (valid SwiGLU tiles)
 };
 
+// Several independent layer-chain calls in one launch (a decoder step's chains). Call i
+// owns blocks [first[i], first[i+1]); inside its range a block plays the same role as in
+// the single-call kernel. The struct is passed as the kernel parameter (about 21 KB, under
+// the 32 KB parameter limit), so no device buffer is written before the launch.
+constexpr int kStepMax = 48;
+struct ChainStepParams {
+  int32_t n;
+  int32_t first[kStepMax + 1];
+  ChainParams c[kStepMax];
+};
+
 // Kernel entry (host stub address) plus its launch shape rule.
 struct KernelEntry {
   const void* fn = nullptr;
   const void* fn_inplace = nullptr;  // chain only: the entry for calls that write in place
+  const void* fn_step = nullptr;          // chain only: several calls per launch (ChainStepParams)
+  const void* fn_step_inplace = nullptr;  // ... one block per token for the norms
   int32_t kind = 0;      // which grid rule the host applies (KernelKind)
   int32_t vec = 0;       // elements per vector (VE), or tile width for SwiGLU
   int32_t unroll = 1;    // vectors per thread per tile (SwiGLU, chain)

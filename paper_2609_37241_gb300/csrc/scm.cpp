@@ -21,6 +21,7 @@
 #include <cuda.h>
 #include <cuda_runtime.h>
 
+#include <algorithm>
 #include <atomic>
 #include <chrono>
 #include <cmath>
@@ -374,6 +375,9 @@ struct Version {
   CUfunction fn;
   CUfunction fn_inplace;  // layer chain: one block per token when outputs alias inputs
   int32_t wave_blocks;    // layer chain: blocks of `fn` resident at once on the whole GPU
+  CUfunction step_fn;           // layer chain: several calls per launch (two blocks per token)
+  CUfunction step_fn_inplace;   // ... one block per token
+  int32_t step_wave_blocks;     // blocks of `step_fn` resident at once
   const float2* inv_freq;
 };
 
@@ -389,7 +393,8 @@ struct trident_scm {
   std::mutex reg_mu;
   std::atomic<uint64_t>* hits_per = nullptr;
   std::atomic<uint64_t> invokes{0}, hits{0}, misses{0}, hook_calls{0}, hook_failures{0},
-      hook_registered{0}, err_invalid{0}, err_cuda{0}, guard_evals{0};
+      hook_registered{0}, err_invalid{0}, err_cuda{0}, guard_evals{0}, fused_launches{0},
+      fused_calls{0};
   // device state
   int32_t device = 0;
   CUcontext ctx = nullptr;
@@ -570,25 +575,82 @@ void pack_swiglu(const trident_args* a, int g, int u, int o, int64_t T, SwigluPa
   p->o_rs = row_stride(t[o], K_ACT_I);
 }
 
+// Launches fn with the SCM's context current on this thread.
+int32_t launch_on(trident_scm* scm, CUlaunchConfig* cfg, CUfunction fn, void** kp) {
+  CUcontext cur = nullptr;
+  g_drv.ctx_get(&cur);
+  const bool swap = cur != scm->ctx;
+  if (swap && g_drv.ctx_push(scm->ctx) != CUDA_SUCCESS)
+    return fail(TRIDENT_ERR_CUDA, "cannot make the SCM's context current");
+  const CUresult rc = g_drv.launch_ex(cfg, fn, kp, nullptr);
+  if (swap) {
+    CUcontext dummy;
+    g_drv.ctx_pop(&dummy);
+  }
+  if (rc != CUDA_SUCCESS) return fail(TRIDENT_ERR_CUDA, "cuLaunchKernelEx failed (%d)", (int)rc);
+  return TRIDENT_OK;
+}
+
+// Launch configuration with the block size and, with TRIDENT_OPT_PDL, programmatic
+// stream serialisation (attr must outlive the launch).
+void base_config(const trident_scm* scm, void* stream, CUlaunchConfig* cfg, CUlaunchAttribute* attr) {
+  std::memset(cfg, 0, sizeof(*cfg));
+  std::memset(attr, 0, sizeof(*attr));
+  cfg->blockDimX = kThreads; cfg->blockDimY = 1; cfg->blockDimZ = 1;
+  cfg->gridDimY = 1; cfg->gridDimZ = 1;
+  cfg->hStream = (CUstream)stream;
+  cfg->attrs = attr;
+  cfg->numAttrs = 0;
+  if (scm->opt.flags & TRIDENT_OPT_PDL) {
+    attr->id = CU_LAUNCH_ATTRIBUTE_PROGRAMMATIC_STREAM_SERIALIZATION;
+    attr->value.programmaticStreamSerializationAllowed = 1;
+    cfg->numAttrs = 1;
+  }
+}
+
+// Packs one layer-chain call: both norms, RoPE/KV, SwiGLU and the RoPE and SwiGLU block
+// counts. The norm split (set_chain_split) is decided by the caller.
+int32_t pack_chain(trident_scm* scm, const Version& v, const trident_args* a, const Sig& s,
+                   ChainParams* c) {
+  pack_addnorm(a, C_H, C_R0, C_GA, C_X1, C_R1, s, K_ACT_H, &c->n1);
+  pack_addnorm(a, C_AO, C_R1, C_GM, C_X2, C_R2, s, K_ACT_H, &c->n2);
+  pack_rope(a, C_Q, a->op == TRIDENT_OP_LAYER_CHAIN_QKNORM ? C_GQ : -1, v, scm->d_err, &c->rope);
+  pack_swiglu(a, C_G, C_U, C_O, s.T, &c->sw);
+  const int64_t per = (int64_t)v.ke.unroll * kThreads * v.ke.vec;
+  const int64_t tiles = (c->sw.I + per - 1) / per;
+  const int64_t upb = rope_units_per_block(c->rope.D, 2);
+  const int64_t nB = (s.T * c->rope.NH + upb - 1) / upb, nC = s.T * tiles;
+  if (2 * s.T + nB + nC > 0x7fffffff) return fail(TRIDENT_ERR_INVALID, "layer chain too large for one launch");
+  c->nB = (int32_t)nB;
+  c->nC = (int32_t)nC;
+  c->sw_tiles_per_row = (int32_t)tiles;
+  c->sw_tiles = nC;
+  return TRIDENT_OK;
+}
+
+// Does a chain call write an output over an input? Then the norms keep one CTA per
+// token: with two, a CTA could overwrite row bytes its partner has not read yet.
+bool chain_inplace(const trident_args* a) {
+  const trident_tensor* t = a->t;
+  return t[C_X1].data == t[C_H].data || t[C_R1].data == t[C_R0].data ||
+         t[C_R2].data == t[C_R0].data || t[C_X2].data == t[C_AO].data;
+}
+
+int32_t set_chain_split(ChainParams* c, int64_t T, int32_t split, int64_t* blocks) {
+  c->a_split = split;
+  c->nA = (int32_t)(T * split);
+  *blocks = (int64_t)c->nA + c->nB + c->nC;
+  return TRIDENT_OK;
+}
+
 inline unsigned cap_grid(int64_t n) { return (unsigned)(n < 1 ? 1 : (n > 0x7fffffff ? 0x7fffffff : n)); }
 
 int32_t do_launch(trident_scm* scm, const Version& v, const trident_args* a, const Sig& s,
                   void* stream) {
   const int op = a->op;
   CUlaunchConfig cfg;
-  std::memset(&cfg, 0, sizeof(cfg));
-  cfg.blockDimX = kThreads; cfg.blockDimY = 1; cfg.blockDimZ = 1;
-  cfg.gridDimY = 1; cfg.gridDimZ = 1;
-  cfg.hStream = (CUstream)stream;
-  CUlaunchAttribute attr[2];
-  std::memset(attr, 0, sizeof(attr));
-  cfg.attrs = attr;
-  cfg.numAttrs = 0;
-  if (scm->opt.flags & TRIDENT_OPT_PDL) {
-    attr[cfg.numAttrs].id = CU_LAUNCH_ATTRIBUTE_PROGRAMMATIC_STREAM_SERIALIZATION;
-    attr[cfg.numAttrs].value.programmaticStreamSerializationAllowed = 1;
-    ++cfg.numAttrs;
-  }
+  CUlaunchAttribute attr;
+  base_config(scm, stream, &cfg, &attr);
   union {
     AddNormParams an;
     RmsNormParams rn;
@@ -641,27 +703,16 @@ int32_t do_launch(trident_scm* scm, const Version& v, const trident_args* a, con
     case TRIDENT_OP_LAYER_CHAIN:
     case TRIDENT_OP_LAYER_CHAIN_QKNORM: {
       ChainParams& c = P.ch;
-      pack_addnorm(a, C_H, C_R0, C_GA, C_X1, C_R1, s, K_ACT_H, &c.n1);
-      pack_addnorm(a, C_AO, C_R1, C_GM, C_X2, C_R2, s, K_ACT_H, &c.n2);
-      pack_rope(a, C_Q, op == TRIDENT_OP_LAYER_CHAIN_QKNORM ? C_GQ : -1, v, scm->d_err, &c.rope);
-      pack_swiglu(a, C_G, C_U, C_O, s.T, &c.sw);
-      const int64_t per = (int64_t)v.ke.unroll * kThreads * v.ke.vec;
-      const int64_t tiles = (c.sw.I + per - 1) / per;
-      const int64_t upb = rope_units_per_block(c.rope.D, 2);
+      int32_t st = pack_chain(scm, v, a, s, &c);
+      if (st != TRIDENT_OK) return st;
       // Two CTAs per token for the norms -- so no SM carries a whole token's norm traffic --
       // while the grid still fits in one wave, and unless an output is written over an
       // input the partner CTA still reads (in-place calls keep one CTA per token).
-      const trident_tensor* t = a->t;
-      const bool inplace = t[C_X1].data == t[C_H].data || t[C_R1].data == t[C_R0].data ||
-                           t[C_R2].data == t[C_R0].data || t[C_X2].data == t[C_AO].data;
-      const int64_t nB = (s.T * c.rope.NH + upb - 1) / upb, nC = s.T * tiles;
-      c.a_split = (!inplace && 2 * s.T + nB + nC <= v.wave_blocks) ? 2 : 1;
-      const int64_t nA = s.T * c.a_split;
-      if (nA + nB + nC > 0x7fffffff) return fail(TRIDENT_ERR_INVALID, "layer chain too large for one launch");
-      c.nA = (int32_t)nA; c.nB = (int32_t)nB; c.nC = (int32_t)nC;
-      c.sw_tiles_per_row = (int32_t)tiles;
-      c.sw_tiles = nC;
-      cfg.gridDimX = (unsigned)(nA + nB + nC);
+      const int32_t split = (!chain_inplace(a) && 2 * s.T + c.nB + c.nC <= v.wave_blocks) ? 2 : 1;
+      int64_t blocks = 0;
+      st = set_chain_split(&c, s.T, split, &blocks);
+      if (st != TRIDENT_OK) return st;
+      cfg.gridDimX = (unsigned)blocks;
       break;
     }
     default:
@@ -670,18 +721,60 @@ int32_t do_launch(trident_scm* scm, const Version& v, const trident_args* a, con
   CUfunction fn = v.fn;
   if ((op == TRIDENT_OP_LAYER_CHAIN || op == TRIDENT_OP_LAYER_CHAIN_QKNORM) && P.ch.a_split == 1)
     fn = v.fn_inplace;
-  CUcontext cur = nullptr;
-  g_drv.ctx_get(&cur);
-  const bool swap = cur != scm->ctx;
-  if (swap && g_drv.ctx_push(scm->ctx) != CUDA_SUCCESS)
-    return fail(TRIDENT_ERR_CUDA, "cannot make the SCM's context current");
-  const CUresult rc = g_drv.launch_ex(&cfg, fn, kp, nullptr);
-  if (swap) {
-    CUcontext dummy;
-    g_drv.ctx_pop(&dummy);
+  return launch_on(scm, &cfg, fn, kp);
+}
+
+// Can calls a[0..m-1] run in one launch, as far as their bytes go? Two rules from one
+// sweep over every slot's extent, sorted by start (only pairs whose extents intersect --
+// views into one buffer, in practice -- reach the exact row test):
+//  - within a call, its launch precondition (check_overlap), when check_own is set;
+//  - between calls, independence: no output byte of one call is a byte of another call's
+//    tensor, so running them together equals running them in order.
+bool step_bytes_ok(const trident_args* a, int32_t m, bool check_own) {
+  struct Ext {
+    int64_t base, end, nr, w, rs;
+    int32_t call, slot;
+    bool out;
+  };
+  thread_local std::vector<Ext> ext;
+  ext.clear();
+  for (int32_t c = 0; c < m; ++c) {
+    const OpInfo& oi = g_ops[a[c].op];
+    for (int i = 0; i < oi.nslots; ++i) {
+      const trident_tensor& t = a[c].t[i];
+      const Rows r = rows_of(t, oi.kind[i]);
+      const int es = elem_size(t.dtype);
+      Ext e;
+      e.base = (int64_t)reinterpret_cast<uintptr_t>(t.data);
+      e.nr = r.n;
+      e.w = r.width * es;
+      e.rs = r.stride * es;
+      if (e.nr <= 0 || e.w <= 0) continue;  // no bytes: overlaps nothing
+      e.end = e.base + (e.nr - 1) * e.rs + e.w;
+      e.call = c;
+      e.slot = i;
+      e.out = oi.out[i];
+      ext.push_back(e);
+    }
   }
-  if (rc != CUDA_SUCCESS) return fail(TRIDENT_ERR_CUDA, "cuLaunchKernelEx failed (%d)", (int)rc);
-  return TRIDENT_OK;
+  std::sort(ext.begin(), ext.end(), [](const Ext& x, const Ext& y) { return x.base < y.base; });
+  const size_t n = ext.size();
+  for (size_t x = 0; x < n; ++x) {
+    const Ext& p = ext[x];
+    for (size_t y = x + 1; y < n && ext[y].base < p.end; ++y) {
+      const Ext& q = ext[y];
+      if (!p.out && !q.out) continue;  // inputs may share bytes
+      if (q.call == p.call && !check_own) continue;
+      if (!rows_overlap(p.base, p.nr, p.w, p.rs, q.base, q.nr, q.w, q.rs)) continue;
+      if (q.call != p.call) return false;  // dependent calls
+      const OpInfo& oi = g_ops[a[p.call].op];
+      const trident_tensor* t = a[p.call].t;
+      if (oi.group[p.slot] != 0 && oi.group[p.slot] == oi.group[q.slot] && same_desc(t[p.slot], t[q.slot]))
+        continue;  // an in-place pair
+      return false;  // the call's own precondition fails (reported by the call-by-call path)
+    }
+  }
+  return true;
 }
 
 // Algorithm 1 over the current table snapshot. Returns OK with *sel, MISS, or an error.
@@ -961,11 +1054,19 @@ TRIDENT_API int32_t trident_scm_register_spec(trident_scm_t* scm, const trident_
         if (cudaGetFuncBySymbol(&g, v.ke.fn_inplace) != cudaSuccess || !g)
           return fail(TRIDENT_ERR_CUDA, "cannot resolve the in-place kernel entry");
         v.fn_inplace = reinterpret_cast<CUfunction>(g);
-        int per_sm = 0, sms = 0;
+        cudaFunction_t h = nullptr, k = nullptr;
+        if (cudaGetFuncBySymbol(&h, v.ke.fn_step) != cudaSuccess || !h ||
+            cudaGetFuncBySymbol(&k, v.ke.fn_step_inplace) != cudaSuccess || !k)
+          return fail(TRIDENT_ERR_CUDA, "cannot resolve the multi-call kernel entries");
+        v.step_fn = reinterpret_cast<CUfunction>(h);
+        v.step_fn_inplace = reinterpret_cast<CUfunction>(k);
+        int per_sm = 0, step_per_sm = 0, sms = 0;
         if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, v.ke.fn, kThreads, 0) != cudaSuccess ||
+            cudaOccupancyMaxActiveBlocksPerMultiprocessor(&step_per_sm, v.ke.fn_step, kThreads, 0) != cudaSuccess ||
             cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, scm->device) != cudaSuccess)
           return fail(TRIDENT_ERR_CUDA, "occupancy query failed");
         v.wave_blocks = per_sm * sms;
+        v.step_wave_blocks = step_per_sm * sms;
       }
       if (v.rope) {
         const bool chain = desc->op == TRIDENT_OP_LAYER_CHAIN || desc->op == TRIDENT_OP_LAYER_CHAIN_QKNORM;
@@ -1065,6 +1166,98 @@ TRIDENT_API int32_t trident_scm_invoke_seq(trident_scm_t* scm, const trident_arg
   return result;
 }
 
+namespace {
+
+constexpr int32_t kNotFused = 100;  // step_chunk: run the chunk call by call
+static_assert(kStepMax == TRIDENT_STEP_MAX, "step chunk size");
+static_assert(sizeof(ChainStepParams) <= 32764, "kernel parameter limit");
+
+// One chunk of trident_scm_invoke_step: select every call; if all hit layer-chain
+// versions with one kernel and the calls are independent, pack them into one launch.
+int32_t step_chunk(trident_scm* scm, const trident_args* a, int32_t m, void* stream,
+                   int32_t* out_selected) {
+  if (m < 2) return kNotFused;
+  Sig sig[kStepMax];
+  int32_t sel[kStepMax];
+  const Version* v0 = nullptr;
+  for (int32_t i = 0; i < m; ++i) {  // guards only: the byte rules follow for all calls at once
+    const OpInfo* oi = nullptr;
+    if (dispatch(scm, a + i, &oi, &sig[i], &sel[i], false) != TRIDENT_OK) return kNotFused;
+    const Version& v = scm->versions[sel[i]];
+    if (v.ke.kind != KK_CHAIN) return kNotFused;
+    if (!v0) v0 = &v;
+    else if (v.ke.fn != v0->ke.fn) return kNotFused;
+  }
+  if (!step_bytes_ok(a, m, !(scm->opt.flags & TRIDENT_OPT_NO_ALIAS_CHECK))) return kNotFused;
+  scm->invokes.fetch_add((uint64_t)m, std::memory_order_relaxed);
+  if (out_selected)
+    for (int32_t i = 0; i < m; ++i) out_selected[i] = sel[i];
+  if (scm->opt.flags & TRIDENT_OPT_FAIL_LAUNCHES)
+    return count_error(scm, fail(TRIDENT_ERR_CUDA, "launch failure injected (TRIDENT_OPT_FAIL_LAUNCHES)"));
+  if (!scm->dry) {
+    thread_local ChainStepParams P;
+    bool inplace = false;
+    int64_t two = 0;  // blocks with two CTAs per token
+    for (int32_t i = 0; i < m; ++i) {
+      ChainParams& c = P.c[i];
+      const int32_t st = pack_chain(scm, scm->versions[sel[i]], a + i, sig[i], &c);
+      if (st != TRIDENT_OK) return count_error(scm, st);
+      inplace = inplace || chain_inplace(a + i);
+      two += 2 * sig[i].T + c.nB + c.nC;
+    }
+    const int32_t split = (!inplace && two <= v0->step_wave_blocks) ? 2 : 1;
+    int64_t first = 0;
+    for (int32_t i = 0; i < m; ++i) {
+      int64_t blocks = 0;
+      set_chain_split(&P.c[i], sig[i].T, split, &blocks);
+      P.first[i] = (int32_t)first;
+      first += blocks;
+      if (first > 0x7fffffff)
+        return count_error(scm, fail(TRIDENT_ERR_INVALID, "step too large for one launch"));
+    }
+    P.first[m] = (int32_t)first;
+    P.n = m;
+    CUlaunchConfig cfg;
+    CUlaunchAttribute attr;
+    base_config(scm, stream, &cfg, &attr);
+    cfg.gridDimX = (unsigned)first;
+    void* kp[1] = {&P};
+    const int32_t st = launch_on(scm, &cfg, split == 2 ? v0->step_fn : v0->step_fn_inplace, kp);
+    if (st != TRIDENT_OK) return count_error(scm, st);
+  }
+  uint64_t evals = 0;
+  for (int32_t i = 0; i < m; ++i) {
+    scm->hits_per[sel[i]].fetch_add(1, std::memory_order_relaxed);
+    evals += (uint64_t)sel[i] + 1;
+  }
+  scm->hits.fetch_add((uint64_t)m, std::memory_order_relaxed);
+  scm->guard_evals.fetch_add(evals, std::memory_order_relaxed);
+  scm->fused_launches.fetch_add(1, std::memory_order_relaxed);
+  scm->fused_calls.fetch_add((uint64_t)m, std::memory_order_relaxed);
+  return TRIDENT_OK;
+}
+
+}  // namespace
+
+TRIDENT_API int32_t trident_scm_invoke_step(trident_scm_t* scm, const trident_args* args, int32_t n,
+                                            void* stream, int32_t* out_selected) {
+  if (!scm || (!args && n > 0) || n < 0) return fail(TRIDENT_ERR_INVALID, "bad sequence");
+  int32_t result = TRIDENT_OK;
+  for (int32_t c0 = 0; c0 < n; c0 += kStepMax) {
+    const int32_t m = n - c0 < kStepMax ? n - c0 : kStepMax;
+    int32_t* sel = out_selected ? out_selected + c0 : nullptr;
+    int32_t st = step_chunk(scm, args + c0, m, stream, sel);
+    if (st == kNotFused) st = trident_scm_invoke_seq(scm, args + c0, m, stream, sel);
+    if (st < 0 || st == TRIDENT_MISS) {
+      if (out_selected)
+        for (int32_t j = c0 + m; j < n; ++j) out_selected[j] = TRIDENT_NOT_RUN;
+      return st;
+    }
+    if (st == TRIDENT_MISS_HANDLED) result = TRIDENT_MISS_HANDLED;
+  }
+  return result;
+}
+
 TRIDENT_API int32_t trident_scm_stats(const trident_scm_t* scm, trident_scm_stats_t* out) {
   if (!scm || !out) return fail(TRIDENT_ERR_INVALID, "NULL argument");
   std::memset(out, 0, sizeof(*out));
@@ -1078,6 +1271,8 @@ TRIDENT_API int32_t trident_scm_stats(const trident_scm_t* scm, trident_scm_stat
   out->err_cuda = scm->err_cuda.load();
   out->guard_evals = scm->guard_evals.load();
   out->num_specs = scm->count.load();
+  out->fused_launches = scm->fused_launches.load();
+  out->fused_calls = scm->fused_calls.load();
   return TRIDENT_OK;
 }
 

@@ -24,6 +24,7 @@ VARIANT_AUTO, VARIANT_GENERIC, VARIANT_VECTOR = 0, 1, 2
 OPT_DRY_RUN, OPT_NO_ALIAS_CHECK, OPT_PDL, OPT_TIMING, OPT_FAIL_LAUNCHES = 0x1, 0x2, 0x4, 0x8, 0x10
 DEVERR_POS = 0x1
 MAX_TENSORS, MAX_FIXED = 20, 8
+STEP_MAX = 48  # calls per launch of trident_scm_invoke_step
 OP_NTENSORS = {1: 5, 2: 6, 3: 8, 4: 3, 5: 18, 6: 20, 7: 3, 8: 2, 9: 3, 10: 2, 11: 3}
 
 c_i32, c_i64, c_u32, c_u64, c_dbl, c_vp = (ctypes.c_int32, ctypes.c_int64, ctypes.c_uint32,
@@ -56,7 +57,7 @@ class trident_scm_stats_t(ctypes.Structure):
     _fields_ = [("invokes", c_u64), ("hits", c_u64), ("misses", c_u64), ("hook_calls", c_u64),
                 ("hook_failures", c_u64), ("hook_registered", c_u64), ("err_invalid", c_u64),
                 ("err_cuda", c_u64), ("guard_evals", c_u64), ("num_specs", c_i32),
-                ("reserved", c_i32)]
+                ("reserved", c_i32), ("fused_launches", c_u64), ("fused_calls", c_u64)]
 
 
 HOOK = ctypes.CFUNCTYPE(c_i32, c_vp, c_vp, ctypes.POINTER(trident_args), c_vp, ctypes.POINTER(c_i32))
@@ -78,6 +79,7 @@ def lib():
             "trident_scm_register_spec": (c_i32, [c_vp, P(trident_spec_desc), P(c_i32)]),
             "trident_scm_invoke": (c_i32, [c_vp, P(trident_args), c_vp, P(c_i32)]),
             "trident_scm_invoke_seq": (c_i32, [c_vp, P(trident_args), c_i32, c_vp, P(c_i32)]),
+            "trident_scm_invoke_step": (c_i32, [c_vp, P(trident_args), c_i32, c_vp, P(c_i32)]),
             "trident_scm_select": (c_i32, [c_vp, P(trident_args), P(c_i32)]),
             "trident_scm_stats": (c_i32, [c_vp, P(trident_scm_stats_t)]),
             "trident_scm_spec_hits": (c_i32, [c_vp, P(c_u64), c_i32, P(c_i32)]),
@@ -97,10 +99,10 @@ def lib():
 
 
 def fastcall():
-    """The CPython fast-call shim (`invoke(scm, args_address, stream)` and
-    `invoke_seq(scm, args_address, n, stream)` on raw integer addresses; the default stream
-    is 0), or None if it was not built. Same C calls as trident_scm_invoke / _seq, without
-    ctypes' per-call cost."""
+    """The CPython fast-call shim (`invoke(scm, args_address, stream)`,
+    `invoke_seq(scm, args_address, n, stream)` and `invoke_step(...)`, same arguments, on raw
+    integer addresses; the default stream is 0), or None if it was not built. Same C calls
+    as trident_scm_invoke / _seq / _step, without ctypes' per-call cost."""
     try:
         lib()
         from . import _fastcall
@@ -146,6 +148,14 @@ def trident_scm_invoke_seq(scm, args_array, stream=None):
     n = len(args_array)
     sel = (c_i32 * max(n, 1))()
     st = lib().trident_scm_invoke_seq(scm, args_array, n, stream, sel)
+    return st, list(sel)[:n]
+
+
+def trident_scm_invoke_step(scm, args_array, stream=None):
+    """Like trident_scm_invoke_seq; independent layer-chain calls share one launch."""
+    n = len(args_array)
+    sel = (c_i32 * max(n, 1))()
+    st = lib().trident_scm_invoke_step(scm, args_array, n, stream, sel)
     return st, list(sel)[:n]
 
 
@@ -301,6 +311,12 @@ class Scm:
 
     def invoke(self, args, stream=None):
         return trident_scm_invoke(self.h, args, stream)
+
+    def invoke_seq(self, args_array, stream=None):
+        return trident_scm_invoke_seq(self.h, args_array, stream)
+
+    def invoke_step(self, args_array, stream=None):
+        return trident_scm_invoke_step(self.h, args_array, stream)
 
     def select(self, args):
         return trident_scm_select(self.h, args)

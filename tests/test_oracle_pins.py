@@ -433,6 +433,25 @@ def test_overlap_precondition_brute_force():
     assert not G.launch_precondition(args)
 
 
+def test_calls_independent_hand_cases():
+    """Independence of whole calls: disjoint buffers, shared inputs, a read of another
+    call's output, a write-write clash, and a one-byte overlap at a row edge."""
+    def norm_call(x, r, y, ro, gam=0x90000):
+        return dict(op=1, tensors=[cases.tensor(x, 1, (2, 8)), cases.tensor(r, 1, (2, 8)),
+                                   cases.tensor(gam, 3, (8,)), cases.tensor(y, 1, (2, 8)),
+                                   cases.tensor(ro, 1, (2, 8))], eps=0.0, theta=0.0, flags=0)
+    a = norm_call(0x10000, 0x20000, 0x30000, 0x40000)
+    b = norm_call(0x50000, 0x60000, 0x70000, 0x80000)
+    assert G.calls_independent([a, b])  # disjoint, and both read one gamma
+    assert G.calls_independent([a, norm_call(0x10000, 0x20000, 0x70000, 0x80000)])  # shared inputs
+    assert not G.calls_independent([a, norm_call(0x40000, 0x60000, 0x70000, 0x80000)])  # reads a's r_out
+    assert not G.calls_independent([norm_call(0x50000, 0x60000, 0x30000, 0x80000), a])  # both write y
+    # b's x ends one byte into a's y (rows of 16 bytes; 2 rows = 32 bytes)
+    assert not G.calls_independent([a, norm_call(0x30000 - 31, 0x60000, 0x70000, 0x80000)])
+    assert G.calls_independent([a, norm_call(0x30000 - 32, 0x60000, 0x70000, 0x80000)])
+    assert G.calls_independent([a])
+
+
 def test_bucket_definition():
     assert [G.bucket_of(t) for t in (1, 2, 3, 4, 5, 8, 9, 128, 129)] == [0, 1, 2, 2, 3, 3, 4, 7, 8]
     for b in range(10):

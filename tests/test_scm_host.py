@@ -47,7 +47,16 @@ def test_exports_every_declared_symbol(S):
     exported = set(re.findall(r" T (trident_\w+)", nm))
     assert declared, "no declarations parsed"
     assert declared == exported, (declared ^ exported)
-    assert S.trident_abi_version() == 2
+    assert S.trident_abi_version() == 3
+
+
+def test_binding_constants_match_header_defines(S):
+    header = open(os.path.join(ROOT, "include", "trident_scm.h")).read()
+    defines = dict(re.findall(r"^#define TRIDENT_(\w+) \(?(-?(?:0x)?[0-9a-fA-F]+)u?\)?", header, re.M))
+    defines.pop("ABI_VERSION")
+    assert {"MAX_TENSORS", "MAX_FIXED", "STEP_MAX", "NOT_RUN", "OPT_PDL", "DEVERR_POS"} <= set(defines)
+    for name, val in defines.items():
+        assert getattr(S, name) == int(val, 0), name
 
 
 def test_struct_layout_matches_header(S, tmp_path):
