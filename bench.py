@@ -687,10 +687,37 @@ def bench_motivation(c, warmup=20, rounds=5, repeats=10):
                 e2e.append((h2 - h0) * 1e6)
         return float(np.median(host)), float(np.median(e2e))
 
+    # the same call through the structured-argument entry: rms_norm(x, residual, weight, out,
+    # eps) with two tree versions (residual None -> RMSNORM, a tensor -> ADD_RMSNORM); the
+    # tree prebuilt once, and packed from the Python arguments on every call
+    tscm = S.Scm(device=c.dev.index or 0)
+    tscm.register_tree(S.make_spec(S.OP_RMSNORM, S.BF16, [H], 1, 4096),
+                       S.Recipe(S.Slot(0), None, S.Slot(1), S.Slot(2), S.EPS))
+    tscm.register_tree(S.make_spec(S.OP_ADD_RMSNORM, S.BF16, [H], 1, 4096),
+                       S.Recipe(S.Slot(0), S.Slot(1), S.Slot(2), (S.Slot(3), S.Slot(4)), S.EPS))
+    tree = S.Tree(x, None, w32, y, 1e-6)
+    th, sp = tscm.h.value, c.sp.value or 0
+    if c.fc is not None:
+        tinv = c.fc.invoke_tree
+        t_addr = ctypes.addressof(tree.nodes)
+        ours_tree = lambda: tinv(th, t_addr, tree.nargs, tree.nnodes, sp)
+
+        def ours_tree_packed():
+            tr = S.Tree(x, None, w32, y, 1e-6)
+            return tinv(th, ctypes.addressof(tr.nodes), tr.nargs, tr.nnodes, sp)
+    else:
+        ours_tree = lambda: S.trident_scm_invoke_tree(tscm.h, tree, c.sp)
+        ours_tree_packed = lambda: S.trident_scm_invoke_tree(tscm.h, S.Tree(x, None, w32, y, 1e-6), c.sp)
+
     res = {}
     res["scm"] = dict(zip(("host_us", "e2e_us"), measure(ours)))
     assert_all_hit(scm, "motivation")
     c.launches += warmup + rounds * repeats
+    res["scm_tree_prebuilt"] = dict(zip(("host_us", "e2e_us"), measure(ours_tree)))
+    res["scm_tree_packed_per_call"] = dict(zip(("host_us", "e2e_us"), measure(ours_tree_packed)))
+    assert_all_hit(tscm, "motivation tree")
+    c.launches += 2 * (warmup + rounds * repeats)
+    tscm.close()
     res["torch_eager"] = dict(zip(("host_us", "e2e_us"), measure(eager)))
     try:
         compiled = t.compile(eager)

@@ -214,6 +214,81 @@ typedef struct trident_spec_desc {
   double rope_theta;                /* ROPE ops and chains: guarded constant; else 0     */
 } trident_spec_desc;
 
+struct trident_scm; /* the SCM handle (trident_scm_t below) */
+
+/* ---------------------------------------------------------------- structured arguments
+ * §3.3 of the paper: the boundary sees the source function's structured arguments (tuples
+ * of tensors, scalars, None); each version's recipe binds them to a logical input tree,
+ * guards address values by their path in that tree, and only after the guards hold are the
+ * leaves the version consumes taken out, in the tree's preorder ("exporter order").
+ *
+ * A call's arguments are one array of nodes: nodes[0 .. nargs-1] are the top-level
+ * parameters in source order; a tuple's n children are nodes[first .. first+n-1], and
+ * first > the tuple's own index (children come after their parent, so the tree has no
+ * cycles). At most TRIDENT_TREE_MAX_NODES nodes and depth TRIDENT_TREE_MAX_DEPTH. */
+#define TRIDENT_TREE_MAX_NODES 4096
+#define TRIDENT_TREE_MAX_DEPTH 16
+typedef enum trident_node_kind {
+  TRIDENT_NODE_NONE = 0,      /* Python None                                             */
+  TRIDENT_NODE_TENSOR = 1,    /* t: a tensor descriptor                                  */
+  TRIDENT_NODE_DLTENSOR = 2,  /* dl: a DLPack DLTensor (the layout shared by DLPack 0.6
+                                 to 1.x: data, device {type, id}, ndim, dtype {code,
+                                 bits, lanes}, shape, strides (NULL = compact), byte
+                                 offset). Accepted: CUDA or CPU devices; bf16, fp16,
+                                 fp32, int32, int64, uint8 and bool, one lane.          */
+  TRIDENT_NODE_TUPLE = 3,     /* n children at nodes[first ...]                          */
+  TRIDENT_NODE_INT = 4,       /* i                                                       */
+  TRIDENT_NODE_FLOAT = 5      /* f                                                       */
+} trident_node_kind;
+
+typedef struct trident_node {
+  int32_t kind;       /* trident_node_kind                    */
+  int32_t n;          /* TUPLE: number of children            */
+  int32_t first;      /* TUPLE: index of the first child      */
+  int32_t reserved;   /* 0                                    */
+  int64_t i;          /* INT                                  */
+  double f;           /* FLOAT                                */
+  const void* dl;     /* DLTENSOR: a DLTensor*                */
+  trident_tensor t;   /* TENSOR                               */
+} trident_node;
+
+/* A version's recipe: a pattern over the call's tree, in the same array form. Each
+ * pattern node requires the argument at the same path to have its kind (a TENSOR pattern
+ * accepts TENSOR and DLTENSOR nodes; a TUPLE pattern requires exactly n children) and
+ * says what the version does with it (bind):
+ *   TENSOR: the op slot (0 .. ntensors-1) the leaf fills, or TRIDENT_BIND_UNUSED;
+ *   INT / FLOAT: TRIDENT_BIND_CONST (a guarded constant: the value must equal i / f),
+ *     TRIDENT_BIND_EPS, _THETA or _SCALAR (the value becomes that argument of the op), or
+ *     TRIDENT_BIND_UNUSED (any value);
+ *   NONE, TUPLE: bind is ignored.
+ * Every slot of the version's op is bound by exactly one TENSOR pattern node. eps,
+ * rope_theta and scalar not bound from the tree take the recipe's values. */
+#define TRIDENT_BIND_UNUSED (-1)
+#define TRIDENT_BIND_CONST (-2)
+#define TRIDENT_BIND_EPS (-3)
+#define TRIDENT_BIND_THETA (-4)
+#define TRIDENT_BIND_SCALAR (-5)
+typedef struct trident_recipe_node {
+  int32_t kind;       /* trident_node_kind (not DLTENSOR)      */
+  int32_t n;          /* TUPLE: number of children             */
+  int32_t first;      /* TUPLE: index of the first child       */
+  int32_t bind;       /* see above                             */
+  int64_t i;          /* INT with TRIDENT_BIND_CONST           */
+  double f;           /* FLOAT with TRIDENT_BIND_CONST         */
+} trident_recipe_node;
+
+typedef struct trident_recipe {
+  int32_t nargs;                      /* top-level parameters: nodes[0 .. nargs-1]  */
+  int32_t nnodes;
+  const trident_recipe_node* nodes;   /* copied by register_tree_spec               */
+  double eps, rope_theta, scalar;     /* values not bound from the tree             */
+} trident_recipe;
+
+/* Compile hook of invoke_tree (see trident_scm_set_tree_hook). */
+typedef int32_t (*trident_tree_hook)(void* user, struct trident_scm* scm, const trident_node* nodes,
+                                     int32_t nargs, int32_t nnodes, void* stream,
+                                     int32_t* out_registered);
+
 typedef struct trident_scm_options {
   int32_t device;        /* CUDA ordinal the SCM launches on (ignored for DRY_RUN) */
   int32_t max_specs;     /* capacity of the version table, 1..4096 (0 = 256)       */
@@ -316,6 +391,30 @@ int32_t trident_scm_invoke_seq(trident_scm_t* scm, const trident_args* args, int
 #define TRIDENT_STEP_MAX 48
 int32_t trident_scm_invoke_step(trident_scm_t* scm, const trident_args* args, int32_t n,
                                 void* stream, int32_t* out_selected);
+
+/* Appends a version that invoke_tree can select: desc as for register_spec, plus the
+ * recipe that binds a call's argument tree to desc->op's slots (§3.3). The recipe is
+ * validated (well-formed tree, every slot bound exactly once, bind codes legal for each
+ * kind) and copied. Such versions are also seen by invoke (which ignores recipes); versions
+ * without a recipe are skipped by invoke_tree. Errors: as register_spec. */
+int32_t trident_scm_register_tree_spec(trident_scm_t* scm, const trident_spec_desc* desc,
+                                       const trident_recipe* recipe, int32_t* out_index);
+
+/* Ordered dispatch over structured arguments (§3.3, §3.5). Validates the tree (node kinds,
+ * child ranges after their parent, size and depth limits, DLTensor dtypes and devices;
+ * ERR_INVALID, the hook is not called). Then, for each version with a recipe in creation
+ * order: the recipe's structure and guarded constants are checked against the tree (a
+ * failure is that version's miss); the consumed leaves and bound scalars form the op's
+ * argument tuple, which is validated (ERR_INVALID ends the call: the bound arguments are
+ * malformed) and guarded as in invoke; the first version whose checks all hold is launched
+ * as invoke does. A miss calls the tree hook if one is set (MISS_HANDLED) or returns MISS.
+ * Results are written to the output tensors the tree names; nothing is returned. */
+int32_t trident_scm_invoke_tree(trident_scm_t* scm, const trident_node* nodes, int32_t nargs,
+                                int32_t nnodes, void* stream, int32_t* out_selected);
+
+/* Installs (or with NULL removes) the compile hook of invoke_tree; same rules as the
+ * invoke hook (called only on a miss, never from inside a hook). */
+int32_t trident_scm_set_tree_hook(trident_scm_t* scm, trident_tree_hook hook, void* user);
 
 /* Selection only: validation plus Algorithm 1's guard loop, with no launch, no hook
  * and no statistics. Returns OK (*out_selected = index), MISS (-1) or ERR_INVALID.

@@ -359,6 +359,80 @@ def select(table, args, check_overlap=True):
     return MISS, -1
 
 
+# ----------------------------------------------------------------------------- structured arguments
+def bind_tree(recipe, args_tree):
+    """§3.3: bind a call's structured arguments to a version's recipe, or None.
+
+    args_tree: the top-level parameters, each a tensor dict, None, an int, a float, or a
+    tuple/list of such values. recipe: dict(op, params, eps, theta, scalar) where params
+    holds one pattern per top-level parameter, a pattern being
+      ("tensor", k)          a tensor, filling op slot k (k = -1: not consumed)
+      ("none",)              None
+      ("tuple", [patterns])  a tuple of exactly that many elements
+      ("int" | "float", bind, value)   bind: "const" (must equal value), "eps", "theta",
+                             "scalar" (the value becomes that argument), "unused".
+    A mismatch of structure, kind or guarded constant is this version's miss (None). The
+    consumed tensors fill the op's slots; scalars not bound keep the recipe's values."""
+    params = recipe["params"]
+    if len(args_tree) != len(params):
+        return None
+    slots = [None] * len(SLOTS[recipe["op"]])
+    scal = dict(eps=recipe["eps"], theta=recipe["theta"], scalar=recipe["scalar"])
+
+    def match(p, v):
+        kind = p[0]
+        if kind == "none":
+            return v is None
+        if kind == "tensor":
+            if not isinstance(v, dict):
+                return False
+            if p[1] >= 0:
+                slots[p[1]] = v
+            return True
+        if kind == "tuple":
+            if not isinstance(v, (tuple, list)) or len(v) != len(p[1]):
+                return False
+            for pc, vc in zip(p[1], v):
+                if not match(pc, vc):
+                    return False
+            return True
+        is_int = isinstance(v, int)  # bool counts as int, as in Python
+        if kind == "int" and not is_int:
+            return False
+        if kind == "float" and not isinstance(v, float):
+            return False
+        bind = p[1]
+        if bind == "const":
+            return v == p[2]
+        if bind in scal:
+            scal[bind] = float(v)
+        return True
+
+    for p, v in zip(params, args_tree):
+        if not match(p, v):
+            return None
+    return dict(op=recipe["op"], tensors=slots, eps=scal["eps"], theta=scal["theta"],
+                scalar=scal["scalar"], flags=0)
+
+
+def select_tree(table, args_tree, check_overlap=True):
+    """Algorithm 1 over versions with recipes: table = [(spec, recipe)] in creation order.
+    The first version whose recipe binds and whose guard holds is selected; bound
+    arguments that are malformed are an error, not a miss."""
+    for i, (spec, recipe) in enumerate(table):
+        args = bind_tree(recipe, args_tree)
+        if args is None:
+            continue
+        if not validate(args):
+            return INVALID, -1
+        if not guard(spec, args):
+            continue
+        if check_overlap and not launch_precondition(args):
+            return INVALID, -1
+        return OK, i
+    return MISS, -1
+
+
 def bucket_of(T):
     """Token-count bucket b: b = 0 holds T = 1; b >= 1 holds 2^(b-1) < T <= 2^b."""
     b = 0

@@ -56,10 +56,32 @@ static PyObject* fc_invoke_step(PyObject* self, PyObject* const* args, Py_ssize_
   return call_seq(trident_scm_invoke_step, "invoke_step(scm, args_address, n, stream)", args, nargs);
 }
 
+/* invoke_tree(scm, nodes_address, nargs, nnodes, stream) -> status */
+static PyObject* fc_invoke_tree(PyObject* self, PyObject* const* args, Py_ssize_t nargs) {
+  (void)self;
+  if (nargs != 5) {
+    PyErr_SetString(PyExc_TypeError, "invoke_tree(scm, nodes_address, nargs, nnodes, stream)");
+    return NULL;
+  }
+  void* scm = PyLong_AsVoidPtr(args[0]);
+  void* nodes = PyLong_AsVoidPtr(args[1]);
+  long na = PyLong_AsLong(args[2]);
+  long nn = PyLong_AsLong(args[3]);
+  void* stream = PyLong_AsVoidPtr(args[4]);
+  if (PyErr_Occurred()) return NULL;
+  if (na < 0 || na > INT32_MAX || nn < 0 || nn > INT32_MAX) {
+    PyErr_SetString(PyExc_ValueError, "nargs or nnodes out of range");
+    return NULL;
+  }
+  return PyLong_FromLong(trident_scm_invoke_tree((trident_scm_t*)scm, (const trident_node*)nodes,
+                                                 (int32_t)na, (int32_t)nn, stream, NULL));
+}
+
 static PyMethodDef methods[] = {
     {"invoke", (PyCFunction)(void (*)(void))fc_invoke, METH_FASTCALL, "trident_scm_invoke"},
     {"invoke_seq", (PyCFunction)(void (*)(void))fc_invoke_seq, METH_FASTCALL, "trident_scm_invoke_seq"},
     {"invoke_step", (PyCFunction)(void (*)(void))fc_invoke_step, METH_FASTCALL, "trident_scm_invoke_step"},
+    {"invoke_tree", (PyCFunction)(void (*)(void))fc_invoke_tree, METH_FASTCALL, "trident_scm_invoke_tree"},
     {NULL, NULL, 0, NULL}};
 
 static struct PyModuleDef module = {PyModuleDef_HEAD_INIT, "_fastcall", NULL, -1, methods,

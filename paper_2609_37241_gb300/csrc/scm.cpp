@@ -36,6 +36,7 @@
 #include <vector>
 
 #include "internal.h"
+#include "tree.h"
 #include "trident_scm.h"
 
 #define TRIDENT_API extern "C" __attribute__((visibility("default")))
@@ -379,6 +380,7 @@ struct Version {
   CUfunction step_fn_inplace;   // ... one block per token
   int32_t step_wave_blocks;     // blocks of `step_fn` resident at once
   const float2* inv_freq;
+  Recipe* recipe;               // structured-argument binding (register_tree_spec), or NULL
 };
 
 }  // namespace
@@ -387,6 +389,8 @@ struct trident_scm {
   trident_scm_options opt{};
   trident_compile_hook hook = nullptr;
   void* user = nullptr;
+  trident_tree_hook tree_hook = nullptr;
+  void* tree_user = nullptr;
   bool dry = false;
   Version* versions = nullptr;
   std::atomic<int32_t> count{0};
@@ -1027,14 +1031,13 @@ TRIDENT_API int32_t trident_scm_create(const trident_scm_options* opt, trident_c
   return TRIDENT_OK;
 }
 
-TRIDENT_API int32_t trident_scm_register_spec(trident_scm_t* scm, const trident_spec_desc* desc,
-                                              int32_t* out_index) {
-  if (!scm) return fail(TRIDENT_ERR_INVALID, "scm is NULL");
-  int32_t nfixed = 0;
-  int32_t st = validate_desc(scm, desc, &nfixed);
-  if (st != TRIDENT_OK) return st;
-  Version v;
-  std::memset(&v, 0, sizeof(v));
+namespace {
+
+// Resolves the version's kernels and tables and publishes it (copy, then release the count).
+int32_t append_version(trident_scm_t* scm, const trident_spec_desc* desc, int32_t nfixed, Version* vp,
+                       int32_t* out_index) {
+  Version& v = *vp;
+  int32_t st = TRIDENT_OK;
   v.d = *desc;
   v.nfixed = nfixed;
   v.rope = g_ops[desc->op].rope;
@@ -1085,6 +1088,47 @@ TRIDENT_API int32_t trident_scm_register_spec(trident_scm_t* scm, const trident_
   return TRIDENT_OK;
 }
 
+// Appends a version (with its recipe, or none); shared by register_spec and
+// register_tree_spec. On failure the recipe is freed.
+int32_t register_version(trident_scm_t* scm, const trident_spec_desc* desc, const trident_recipe* recipe,
+                         int32_t* out_index) {
+  if (!scm) return fail(TRIDENT_ERR_INVALID, "scm is NULL");
+  int32_t nfixed = 0;
+  int32_t st = validate_desc(scm, desc, &nfixed);
+  if (st != TRIDENT_OK) return st;
+  Version v;
+  std::memset(&v, 0, sizeof(v));
+  if (recipe) {
+    Recipe* r = new (std::nothrow) Recipe();
+    if (!r) return fail(TRIDENT_ERR_INVALID, "out of host memory");
+    st = make_recipe(recipe, desc->op, g_ops[desc->op].nslots, r);
+    if (st != TRIDENT_OK) {
+      delete r;
+      return st;
+    }
+    v.recipe = r;
+  }
+  st = append_version(scm, desc, nfixed, &v, out_index);
+  if (st != TRIDENT_OK && v.recipe) {
+    free_recipe(v.recipe);
+    delete v.recipe;
+  }
+  return st;
+}
+
+}  // namespace
+
+TRIDENT_API int32_t trident_scm_register_spec(trident_scm_t* scm, const trident_spec_desc* desc,
+                                              int32_t* out_index) {
+  return register_version(scm, desc, nullptr, out_index);
+}
+
+TRIDENT_API int32_t trident_scm_register_tree_spec(trident_scm_t* scm, const trident_spec_desc* desc,
+                                                   const trident_recipe* recipe, int32_t* out_index) {
+  if (!recipe) return fail(TRIDENT_ERR_INVALID, "recipe is NULL");
+  return register_version(scm, desc, recipe, out_index);
+}
+
 TRIDENT_API int32_t trident_scm_select(const trident_scm_t* scm, const trident_args* args,
                                        int32_t* out_selected) {
   if (out_selected) *out_selected = -1;
@@ -1097,48 +1141,42 @@ TRIDENT_API int32_t trident_scm_select(const trident_scm_t* scm, const trident_a
   return st;
 }
 
-TRIDENT_API int32_t trident_scm_invoke(trident_scm_t* scm, const trident_args* args, void* stream,
-                                       int32_t* out_selected) {
-  if (out_selected) *out_selected = -1;
-  if (!scm) return fail(TRIDENT_ERR_INVALID, "scm is NULL");
-  const bool timing = scm->ring != nullptr;
-  const uint64_t t0 = timing ? now_ns() : 0;
-  scm->invokes.fetch_add(1, std::memory_order_relaxed);
-  const OpInfo* oi = nullptr;
-  Sig s;
-  int32_t sel = -1;
-  int32_t st = dispatch(scm, args, &oi, &s, &sel, !(scm->opt.flags & TRIDENT_OPT_NO_ALIAS_CHECK));
-  if (st == TRIDENT_OK) {
-    const Version& v = scm->versions[sel];
-    if (scm->opt.flags & TRIDENT_OPT_FAIL_LAUNCHES) {  // injected failure of P_i
-      if (out_selected) *out_selected = sel;
-      return count_error(scm, fail(TRIDENT_ERR_CUDA, "launch failure injected (TRIDENT_OPT_FAIL_LAUNCHES)"));
-    }
-    if (!scm->dry) {
-      st = do_launch(scm, v, args, s, stream);
-      if (st != TRIDENT_OK) return count_error(scm, st);  // Algorithm 1: raise, no next version
-    }
-    scm->hits.fetch_add(1, std::memory_order_relaxed);
-    scm->hits_per[sel].fetch_add(1, std::memory_order_relaxed);
-    scm->guard_evals.fetch_add((uint64_t)sel + 1, std::memory_order_relaxed);
-    if (timing) {
-      const uint64_t k = scm->ring_n.fetch_add(1, std::memory_order_relaxed);
-      const uint64_t dt = now_ns() - t0;
-      scm->ring[k % (uint64_t)scm->ring_cap] = dt > 0xffffffffull ? 0xffffffffu : (uint32_t)dt;
-    }
-    if (out_selected) *out_selected = sel;
-    return TRIDENT_OK;
+namespace {
+
+// A guard hit on version `sel`: launch (unless dry-run), count, record host time.
+int32_t run_hit(trident_scm* scm, int32_t sel, const trident_args* args, const Sig& s, void* stream,
+                uint64_t t0, int32_t* out_selected) {
+  const Version& v = scm->versions[sel];
+  if (out_selected) *out_selected = sel;
+  if (scm->opt.flags & TRIDENT_OPT_FAIL_LAUNCHES)  // injected failure of P_i
+    return count_error(scm, fail(TRIDENT_ERR_CUDA, "launch failure injected (TRIDENT_OPT_FAIL_LAUNCHES)"));
+  if (!scm->dry) {
+    const int32_t st = do_launch(scm, v, args, s, stream);
+    if (st != TRIDENT_OK) return count_error(scm, st);  // Algorithm 1: raise, no next version
   }
-  if (st != TRIDENT_MISS) return count_error(scm, st);
-  // every guard failed: a specialisation miss (§3.5)
+  scm->hits.fetch_add(1, std::memory_order_relaxed);
+  scm->hits_per[sel].fetch_add(1, std::memory_order_relaxed);
+  scm->guard_evals.fetch_add((uint64_t)sel + 1, std::memory_order_relaxed);
+  if (scm->ring) {
+    const uint64_t k = scm->ring_n.fetch_add(1, std::memory_order_relaxed);
+    const uint64_t dt = now_ns() - t0;
+    scm->ring[k % (uint64_t)scm->ring_cap] = dt > 0xffffffffull ? 0xffffffffu : (uint32_t)dt;
+  }
+  return TRIDENT_OK;
+}
+
+// Every guard failed: a specialisation miss (§3.5). `call_hook` runs the hook (if the
+// call is not already inside one) and returns its status.
+template <class Hook>
+int32_t run_miss(trident_scm* scm, bool have_hook, Hook call_hook, int32_t* out_selected) {
   scm->misses.fetch_add(1, std::memory_order_relaxed);
   scm->guard_evals.fetch_add((uint64_t)scm->count.load(std::memory_order_relaxed),
                              std::memory_order_relaxed);
-  if (!scm->hook || tl_hook_depth > 0) return TRIDENT_MISS;
+  if (!have_hook || tl_hook_depth > 0) return TRIDENT_MISS;
   scm->hook_calls.fetch_add(1, std::memory_order_relaxed);
   int32_t reg = -1;
   ++tl_hook_depth;
-  const int32_t hr = scm->hook(scm->user, scm, args, stream, &reg);
+  const int32_t hr = call_hook(&reg);
   --tl_hook_depth;
   if (hr != 0) {
     scm->hook_failures.fetch_add(1, std::memory_order_relaxed);
@@ -1146,6 +1184,63 @@ TRIDENT_API int32_t trident_scm_invoke(trident_scm_t* scm, const trident_args* a
   }
   if (out_selected) *out_selected = reg;
   return TRIDENT_MISS_HANDLED;
+}
+
+}  // namespace
+
+TRIDENT_API int32_t trident_scm_invoke(trident_scm_t* scm, const trident_args* args, void* stream,
+                                       int32_t* out_selected) {
+  if (out_selected) *out_selected = -1;
+  if (!scm) return fail(TRIDENT_ERR_INVALID, "scm is NULL");
+  const uint64_t t0 = scm->ring ? now_ns() : 0;
+  scm->invokes.fetch_add(1, std::memory_order_relaxed);
+  const OpInfo* oi = nullptr;
+  Sig s;
+  int32_t sel = -1;
+  const int32_t st = dispatch(scm, args, &oi, &s, &sel, !(scm->opt.flags & TRIDENT_OPT_NO_ALIAS_CHECK));
+  if (st == TRIDENT_OK) return run_hit(scm, sel, args, s, stream, t0, out_selected);
+  if (st != TRIDENT_MISS) return count_error(scm, st);
+  return run_miss(scm, scm->hook != nullptr, [&](int32_t* reg) {
+    return scm->hook(scm->user, scm, args, stream, reg);
+  }, out_selected);
+}
+
+TRIDENT_API int32_t trident_scm_invoke_tree(trident_scm_t* scm, const trident_node* nodes, int32_t nargs,
+                                            int32_t nnodes, void* stream, int32_t* out_selected) {
+  if (out_selected) *out_selected = -1;
+  if (!scm) return fail(TRIDENT_ERR_INVALID, "scm is NULL");
+  const uint64_t t0 = scm->ring ? now_ns() : 0;
+  scm->invokes.fetch_add(1, std::memory_order_relaxed);
+  int32_t st = validate_tree(nodes, nargs, nnodes);
+  if (st != TRIDENT_OK) return count_error(scm, st);
+  const bool check_alias = !(scm->opt.flags & TRIDENT_OPT_NO_ALIAS_CHECK);
+  const int32_t n = scm->count.load(std::memory_order_acquire);
+  trident_args a;
+  for (int32_t i = 0; i < n; ++i) {
+    const Version& v = scm->versions[i];
+    if (!v.recipe) continue;
+    if (!bind_tree(*v.recipe, nodes, nargs, &a)) continue;  // structure or a guarded constant differs
+    const OpInfo* oi = nullptr;
+    Sig s;
+    st = analyze(&a, &oi, &s);
+    if (st != TRIDENT_OK) return count_error(scm, st);  // the bound arguments are malformed
+    if (!guard_holds(v, s, &a)) continue;
+    if (check_alias) {
+      st = check_overlap(&a, *oi);
+      if (st != TRIDENT_OK) return count_error(scm, st);
+    }
+    return run_hit(scm, i, &a, s, stream, t0, out_selected);
+  }
+  return run_miss(scm, scm->tree_hook != nullptr, [&](int32_t* reg) {
+    return scm->tree_hook(scm->tree_user, scm, nodes, nargs, nnodes, stream, reg);
+  }, out_selected);
+}
+
+TRIDENT_API int32_t trident_scm_set_tree_hook(trident_scm_t* scm, trident_tree_hook hook, void* user) {
+  if (!scm) return fail(TRIDENT_ERR_INVALID, "scm is NULL");
+  scm->tree_hook = hook;
+  scm->tree_user = user;
+  return TRIDENT_OK;
 }
 
 TRIDENT_API int32_t trident_scm_invoke_seq(trident_scm_t* scm, const trident_args* args, int32_t n,
@@ -1322,6 +1417,14 @@ TRIDENT_API void trident_scm_destroy(trident_scm_t* scm) {
       if (scm->d_err) cudaFree(scm->d_err);
       return TRIDENT_OK;
     });
+  }
+  if (scm->versions) {
+    const int32_t n = scm->count.load();
+    for (int32_t i = 0; i < n; ++i)
+      if (scm->versions[i].recipe) {
+        free_recipe(scm->versions[i].recipe);
+        delete scm->versions[i].recipe;
+      }
   }
   std::free(scm->versions);
   delete[] scm->hits_per;

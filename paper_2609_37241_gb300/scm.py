@@ -25,6 +25,9 @@ OPT_DRY_RUN, OPT_NO_ALIAS_CHECK, OPT_PDL, OPT_TIMING, OPT_FAIL_LAUNCHES = 0x1, 0
 DEVERR_POS = 0x1
 MAX_TENSORS, MAX_FIXED = 20, 8
 STEP_MAX = 48  # calls per launch of trident_scm_invoke_step
+TREE_MAX_NODES, TREE_MAX_DEPTH = 4096, 16
+NODE_NONE, NODE_TENSOR, NODE_DLTENSOR, NODE_TUPLE, NODE_INT, NODE_FLOAT = 0, 1, 2, 3, 4, 5
+BIND_UNUSED, BIND_CONST, BIND_EPS, BIND_THETA, BIND_SCALAR = -1, -2, -3, -4, -5
 OP_NTENSORS = {1: 5, 2: 6, 3: 8, 4: 3, 5: 18, 6: 20, 7: 3, 8: 2, 9: 3, 10: 2, 11: 3}
 
 c_i32, c_i64, c_u32, c_u64, c_dbl, c_vp = (ctypes.c_int32, ctypes.c_int64, ctypes.c_uint32,
@@ -60,7 +63,24 @@ class trident_scm_stats_t(ctypes.Structure):
                 ("reserved", c_i32), ("fused_launches", c_u64), ("fused_calls", c_u64)]
 
 
+class trident_node(ctypes.Structure):
+    _fields_ = [("kind", c_i32), ("n", c_i32), ("first", c_i32), ("reserved", c_i32),
+                ("i", c_i64), ("f", c_dbl), ("dl", c_vp), ("t", trident_tensor)]
+
+
+class trident_recipe_node(ctypes.Structure):
+    _fields_ = [("kind", c_i32), ("n", c_i32), ("first", c_i32), ("bind", c_i32),
+                ("i", c_i64), ("f", c_dbl)]
+
+
+class trident_recipe(ctypes.Structure):
+    _fields_ = [("nargs", c_i32), ("nnodes", c_i32), ("nodes", ctypes.POINTER(trident_recipe_node)),
+                ("eps", c_dbl), ("rope_theta", c_dbl), ("scalar", c_dbl)]
+
+
 HOOK = ctypes.CFUNCTYPE(c_i32, c_vp, c_vp, ctypes.POINTER(trident_args), c_vp, ctypes.POINTER(c_i32))
+TREE_HOOK = ctypes.CFUNCTYPE(c_i32, c_vp, c_vp, ctypes.POINTER(trident_node), c_i32, c_i32, c_vp,
+                             ctypes.POINTER(c_i32))
 
 _lib = None
 
@@ -81,6 +101,10 @@ def lib():
             "trident_scm_invoke_seq": (c_i32, [c_vp, P(trident_args), c_i32, c_vp, P(c_i32)]),
             "trident_scm_invoke_step": (c_i32, [c_vp, P(trident_args), c_i32, c_vp, P(c_i32)]),
             "trident_scm_select": (c_i32, [c_vp, P(trident_args), P(c_i32)]),
+            "trident_scm_register_tree_spec": (c_i32, [c_vp, P(trident_spec_desc), P(trident_recipe),
+                                                       P(c_i32)]),
+            "trident_scm_invoke_tree": (c_i32, [c_vp, P(trident_node), c_i32, c_i32, c_vp, P(c_i32)]),
+            "trident_scm_set_tree_hook": (c_i32, [c_vp, TREE_HOOK, c_vp]),
             "trident_scm_stats": (c_i32, [c_vp, P(trident_scm_stats_t)]),
             "trident_scm_spec_hits": (c_i32, [c_vp, P(c_u64), c_i32, P(c_i32)]),
             "trident_scm_host_times": (c_i32, [c_vp, P(c_u32), c_i32, P(c_i32)]),
@@ -157,6 +181,20 @@ def trident_scm_invoke_step(scm, args_array, stream=None):
     sel = (c_i32 * max(n, 1))()
     st = lib().trident_scm_invoke_step(scm, args_array, n, stream, sel)
     return st, list(sel)[:n]
+
+
+def trident_scm_register_tree_spec(scm, desc, recipe):
+    idx = c_i32(-1)
+    st = lib().trident_scm_register_tree_spec(scm, ctypes.byref(desc), ctypes.byref(recipe.c),
+                                              ctypes.byref(idx))
+    return st, idx.value
+
+
+def trident_scm_invoke_tree(scm, tree, stream=None):
+    sel = c_i32(-1)
+    st = lib().trident_scm_invoke_tree(scm, tree.nodes, tree.nargs, tree.nnodes, stream,
+                                       ctypes.byref(sel))
+    return st, sel.value
 
 
 def trident_scm_select(scm, args):
@@ -280,6 +318,140 @@ def make_spec(op, dtype, fixed, tok_lo, tok_hi, rank=None, layout=LAYOUT_CONTIG,
     return d
 
 
+# ---------------------------------------------------------------- structured arguments
+class DL:
+    """Marks a tensor to be passed through DLPack (a DLTENSOR node) instead of as a
+    descriptor; the capsule is kept alive by the tree."""
+
+    def __init__(self, tensor):
+        self.tensor = tensor
+
+
+_capsule_ptr = None
+
+
+def _dltensor_address(capsule):
+    global _capsule_ptr
+    if _capsule_ptr is None:
+        f = ctypes.pythonapi.PyCapsule_GetPointer
+        f.restype = c_vp
+        f.argtypes = [ctypes.py_object, ctypes.c_char_p]
+        _capsule_ptr = f
+    return _capsule_ptr(capsule, b"dltensor")  # DLManagedTensor: its DLTensor comes first
+
+
+class Tree:
+    """A call's structured arguments as a trident_node array: the top-level parameters
+    first, each tuple's children contiguous after it (breadth-first)."""
+
+    def __init__(self, *args):
+        import torch
+        values = list(args)
+        self._keep = []
+        queue = list(range(len(values)))
+        nodes = [None] * len(values)
+        q = 0
+        while q < len(queue):
+            i = queue[q]
+            q += 1
+            v = values[i]
+            if isinstance(v, (tuple, list)):
+                first = len(values)
+                values.extend(v)
+                nodes.extend([None] * len(v))
+                queue.extend(range(first, first + len(v)))
+                nodes[i] = ("tuple", len(v), first)
+            else:
+                nodes[i] = ("leaf",)
+        arr = (trident_node * max(len(values), 1))()
+        for i, v in enumerate(values):
+            nd = arr[i]
+            if nodes[i][0] == "tuple":
+                nd.kind, nd.n, nd.first = NODE_TUPLE, nodes[i][1], nodes[i][2]
+            elif v is None:
+                nd.kind = NODE_NONE
+            elif isinstance(v, DL):
+                cap = torch.utils.dlpack.to_dlpack(v.tensor)
+                self._keep.append(cap)
+                nd.kind, nd.dl = NODE_DLTENSOR, _dltensor_address(cap)
+            elif isinstance(v, torch.Tensor) or isinstance(v, dict):
+                nd.kind = NODE_TENSOR
+                (fill_tensor_dict if isinstance(v, dict) else fill_tensor)(nd.t, v)
+            elif isinstance(v, bool) or isinstance(v, int):
+                nd.kind, nd.i = NODE_INT, int(v)
+            elif isinstance(v, float):
+                nd.kind, nd.f = NODE_FLOAT, v
+            else:
+                raise TypeError(f"unsupported argument type {type(v).__name__}")
+        self.nodes, self.nargs, self.nnodes = arr, len(args), len(values)
+
+
+class Slot:
+    """Recipe leaf: a tensor that fills op slot k (k = -1: a tensor the version ignores)."""
+
+    def __init__(self, k):
+        self.k = k
+
+
+class Num:
+    """Recipe leaf for an int or float argument: kind 'int' | 'float', bind BIND_*, value
+    for BIND_CONST."""
+
+    def __init__(self, kind, bind, value=0):
+        self.kind, self.bind, self.value = kind, bind, value
+
+
+IGNORED = Slot(-1)
+EPS = Num("float", BIND_EPS)
+THETA = Num("float", BIND_THETA)
+SCALAR_ARG = Num("float", BIND_SCALAR)
+ANY_INT, ANY_FLOAT = Num("int", BIND_UNUSED), Num("float", BIND_UNUSED)
+
+
+def const(v):
+    """A guarded constant (int or float)."""
+    return Num("int" if isinstance(v, int) else "float", BIND_CONST, v)
+
+
+class Recipe:
+    """A version's recipe (trident_recipe) from a pattern over the top-level parameters:
+    Slot / IGNORED for tensors, None, tuples, Num (EPS, THETA, SCALAR_ARG, const(v),
+    ANY_INT, ANY_FLOAT)."""
+
+    def __init__(self, *pattern, eps=0.0, rope_theta=0.0, scalar=0.0):
+        values = list(pattern)
+        spans = [None] * len(values)
+        q = 0
+        while q < len(values):
+            v = values[q]
+            if isinstance(v, (tuple, list)):
+                spans[q] = (len(v), len(values))
+                values.extend(v)
+                spans.extend([None] * len(v))
+            q += 1
+        arr = (trident_recipe_node * max(len(values), 1))()
+        for i, v in enumerate(values):
+            nd = arr[i]
+            if spans[i] is not None:
+                nd.kind, nd.n, nd.first = NODE_TUPLE, spans[i][0], spans[i][1]
+            elif v is None:
+                nd.kind = NODE_NONE
+            elif isinstance(v, Slot):
+                nd.kind, nd.bind = NODE_TENSOR, v.k
+            elif isinstance(v, Num):
+                nd.kind = NODE_INT if v.kind == "int" else NODE_FLOAT
+                nd.bind = v.bind
+                if v.kind == "int":
+                    nd.i = int(v.value)
+                else:
+                    nd.f = float(v.value)
+            else:
+                raise TypeError(f"unsupported recipe element {v!r}")
+        self._arr = arr
+        self.c = trident_recipe(len(pattern), len(values), ctypes.cast(arr, ctypes.POINTER(trident_recipe_node)),
+                                eps, rope_theta, scalar)
+
+
 class Scm:
     """Owning wrapper: create on construction, destroy on close/GC."""
 
@@ -311,6 +483,31 @@ class Scm:
 
     def invoke(self, args, stream=None):
         return trident_scm_invoke(self.h, args, stream)
+
+    def register_tree(self, desc, recipe):
+        st, idx = trident_scm_register_tree_spec(self.h, desc, recipe)
+        if st != OK:
+            raise ScmError(st, "trident_scm_register_tree_spec")
+        return idx
+
+    def invoke_tree(self, tree, stream=None):
+        return trident_scm_invoke_tree(self.h, tree, stream)
+
+    def set_tree_hook(self, fn):
+        """fn(scm, nodes_pointer, nargs, nnodes, stream) -> registered index or None."""
+        def tramp(user, scm, nodes, nargs, nnodes, stream, out_registered):
+            try:
+                reg = fn(self, nodes, nargs, nnodes, stream)
+                out_registered[0] = -1 if reg is None else int(reg)
+                return 0
+            except Exception as e:
+                self.hook_error = e
+                out_registered[0] = -1
+                return 1
+        self._tree_cb = TREE_HOOK(tramp) if fn is not None else TREE_HOOK()
+        st = lib().trident_scm_set_tree_hook(self.h, self._tree_cb, None)
+        if st != OK:
+            raise ScmError(st, "trident_scm_set_tree_hook")
 
     def invoke_seq(self, args_array, stream=None):
         return trident_scm_invoke_seq(self.h, args_array, stream)

@@ -175,3 +175,26 @@ def lib_args(args):
 
 
 STATUS = {0: "OK", 2: "MISS", -1: "INVALID"}
+
+
+def lib_recipe(recipe):
+    """Library recipe (scm.Recipe) from an oracle-style recipe dict (oracle.guards.bind_tree)."""
+    from paper_2609_37241_gb300 import scm
+    binds = {"const": scm.BIND_CONST, "eps": scm.BIND_EPS, "theta": scm.BIND_THETA,
+             "scalar": scm.BIND_SCALAR, "unused": scm.BIND_UNUSED}
+
+    def conv(p):
+        if p[0] == "none":
+            return None
+        if p[0] == "tensor":
+            return scm.Slot(p[1])
+        if p[0] == "tuple":
+            return tuple(conv(c) for c in p[1])
+        return scm.Num(p[0], binds[p[1]], p[2] if len(p) > 2 else 0)
+
+    return scm.Recipe(*[conv(p) for p in recipe["params"]], eps=recipe["eps"],
+                      rope_theta=recipe["theta"], scalar=recipe["scalar"])
+
+
+def recipe(op, *params, eps=0.0, theta=0.0, scalar=0.0):
+    return dict(op=op, params=list(params), eps=eps, theta=theta, scalar=scalar)

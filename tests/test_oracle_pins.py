@@ -452,6 +452,31 @@ def test_calls_independent_hand_cases():
     assert G.calls_independent([a])
 
 
+def test_bind_tree_hand_cases():
+    """The recipe binder on hand-made trees: structure, kinds, guarded constants, bound
+    scalars, ignored leaves and the slot each consumed tensor fills."""
+    a, b, c = (cases.tensor(0x1000 * k, 1, (2, 8)) for k in (1, 2, 3))
+    g = cases.tensor(0x9000, 3, (8,))
+    rec = cases.recipe(1, ("tuple", [("tensor", 1), ("tensor", 0)]), ("tensor", 2), ("none",),
+                       ("tuple", [("tensor", 3), ("tensor", -1), ("tensor", 4)]), ("float", "eps"),
+                       ("int", "const", 2), eps=0.5, theta=7.0)
+    got = G.bind_tree(rec, [(a, b), g, None, (c, a, b), 1e-3, 2])
+    assert [t["addr"] for t in got["tensors"]] == [b["addr"], a["addr"], g["addr"], c["addr"], b["addr"]]
+    assert (got["op"], got["eps"], got["theta"], got["scalar"]) == (1, 1e-3, 7.0, 0.0)
+    assert G.bind_tree(rec, [(a, b), g, None, (c, a, b), 1e-3, 3]) is None      # constant differs
+    assert G.bind_tree(rec, [(a, b), g, None, (c, a, b), 1e-3, 2.0]) is None    # float, not int
+    assert G.bind_tree(rec, [(a, b), g, None, (c, a, b), 1, 2]) is None         # int eps
+    assert G.bind_tree(rec, [(a, b), g, a, (c, a, b), 1e-3, 2]) is None         # tensor for None
+    assert G.bind_tree(rec, [(a, b, c), g, None, (c, a, b), 1e-3, 2]) is None   # tuple arity
+    assert G.bind_tree(rec, [a, g, None, (c, a, b), 1e-3, 2]) is None           # tensor for tuple
+    assert G.bind_tree(rec, [(a, b), g, None, (c, a, b), 1e-3]) is None         # parameter count
+    assert G.bind_tree(rec, [(a, b), g, None, (c, g, b), 1e-3, 2]) is not None  # ignored leaf: any tensor
+    assert G.bind_tree(rec, [(a, b), g, None, (c, 5, b), 1e-3, 2]) is None      # ... but a tensor
+    # True is the int 1 (Python semantics)
+    one = cases.recipe(7, ("tensor", 0), ("tensor", 1), ("tensor", 2), ("int", "const", 1))
+    assert G.bind_tree(one, [a, g, b, True]) is not None
+
+
 def test_bucket_definition():
     assert [G.bucket_of(t) for t in (1, 2, 3, 4, 5, 8, 9, 128, 129)] == [0, 1, 2, 2, 3, 3, 4, 7, 8]
     for b in range(10):

@@ -420,6 +420,17 @@ def test_fastcall_shim_matches_ctypes(S):
     assert (st.hits, st.misses, st.err_invalid) == (3, 2, 1)
     with pytest.raises(TypeError):
         fc.invoke(h, ctypes.addressof(hit), None)
+    # invoke_step and invoke_tree through the shim
+    assert fc.invoke_step(h, ctypes.addressof(arr), 2, 0) == S.OK
+    s.register_tree(S.make_spec(1, 1, [64], 1, 8), S.Recipe(S.Slot(0), S.Slot(1), S.Slot(2),
+                                                             (S.Slot(3), S.Slot(4)), S.EPS))
+    x, r, w, y, ro = cases.make_args({"op": 1, "T": 4, "H": 64})["tensors"]
+    tree = S.Tree(x, r, w, (y, ro), 1e-6)
+    assert fc.invoke_tree(h, ctypes.addressof(tree.nodes), tree.nargs, tree.nnodes, 0) == S.OK
+    assert fc.invoke_tree(h, ctypes.addressof(tree.nodes), tree.nargs, tree.nnodes - 1, 0) == S.ERR_INVALID
+    with pytest.raises(ValueError):
+        fc.invoke_tree(h, ctypes.addressof(tree.nodes), -1, tree.nnodes, 0)
+    assert s.stats().hits == 6
     s.close()
 
 
