@@ -705,18 +705,25 @@ def bench_motivation(c, warmup=20, rounds=5, repeats=10):
         def ours_tree_packed():
             tr = S.Tree(x, None, w32, y, 1e-6)
             return tinv(th, ctypes.addressof(tr.nodes), tr.nargs, tr.nnodes, sp)
+        pinv = c.fc.invoke_py
+        ours_tree_c = lambda: pinv(th, sp, x, None, w32, y, 1e-6)
     else:
         ours_tree = lambda: S.trident_scm_invoke_tree(tscm.h, tree, c.sp)
         ours_tree_packed = lambda: S.trident_scm_invoke_tree(tscm.h, S.Tree(x, None, w32, y, 1e-6), c.sp)
+        ours_tree_c = None
 
     res = {}
     res["scm"] = dict(zip(("host_us", "e2e_us"), measure(ours)))
     assert_all_hit(scm, "motivation")
     c.launches += warmup + rounds * repeats
     res["scm_tree_prebuilt"] = dict(zip(("host_us", "e2e_us"), measure(ours_tree)))
-    res["scm_tree_packed_per_call"] = dict(zip(("host_us", "e2e_us"), measure(ours_tree_packed)))
+    res["scm_tree_packed_python"] = dict(zip(("host_us", "e2e_us"), measure(ours_tree_packed)))
+    n_tree = 2
+    if ours_tree_c is not None:  # the arguments packed per call by the CPython shim
+        res["scm_tree_packed_c"] = dict(zip(("host_us", "e2e_us"), measure(ours_tree_c)))
+        n_tree += 1
     assert_all_hit(tscm, "motivation tree")
-    c.launches += 2 * (warmup + rounds * repeats)
+    c.launches += n_tree * (warmup + rounds * repeats)
     tscm.close()
     res["torch_eager"] = dict(zip(("host_us", "e2e_us"), measure(eager)))
     try:

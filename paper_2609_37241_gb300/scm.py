@@ -493,6 +493,14 @@ class Scm:
     def invoke_tree(self, tree, stream=None):
         return trident_scm_invoke_tree(self.h, tree, stream)
 
+    def call(self, *args, stream=None):
+        """invoke_tree on Python arguments (tensors, tuples, lists, ints, floats, None),
+        packed by the CPython shim when it is built, else by Tree. Returns the status."""
+        fc = fastcall()
+        if fc is not None:
+            return fc.invoke_py(self.h.value, stream or 0, *args)
+        return trident_scm_invoke_tree(self.h, Tree(*args), stream)[0]
+
     def set_tree_hook(self, fn):
         """fn(scm, nodes_pointer, nargs, nnodes, stream) -> registered index or None."""
         def tramp(user, scm, nodes, nargs, nnodes, stream, out_registered):

@@ -85,3 +85,24 @@ def test_layer_chain_as_a_nested_tree(S):
     assert S.trident_scm_device_status(s.h, stream())[1] == 0
     s.close()
     check_chain(ref, out, inp)
+
+
+def test_python_arguments_packed_by_the_shim(S):
+    """Scm.call: the CPython shim packs the Python arguments per call (no prebuilt tree)."""
+    H, T = 4096, 5
+    g = np.random.default_rng(55)
+    x, r, gam = synth.act(g, (T, H), BF16), synth.act(g, (T, H), BF16), synth.gamma(g, H)
+    xd, rd, gd = P.dev(x, BF16), P.dev(r, BF16), torch.from_numpy(gam).cuda()
+    s = rms_scm(S, H, BF16)
+    y, ro = torch.empty_like(xd), torch.empty_like(rd)
+    assert s.call(xd, rd, gd, [y, ro], 1e-6, stream=stream()) == S.OK
+    y1 = torch.empty_like(xd)
+    assert s.call(xd, None, gd, y1, 1e-6, stream=stream()) == S.OK
+    assert s.call(xd, None, gd, y1, 1, stream=stream()) == S.MISS  # an int eps: no version
+    torch.cuda.synchronize()
+    s.close()
+    y_ref, y_bits, ro_bits = L.add_rmsnorm(x, r, gam, 1e-6, BF16)
+    assert np.array_equal(P.host_bits(ro, BF16), ro_bits)
+    P.check_act(P.host_bits(y, BF16), y_ref, y_bits, BF16, "y")
+    y1_ref, y1_bits = L.rmsnorm(x, gam, 1e-6, BF16)
+    P.check_act(P.host_bits(y1, BF16), y1_ref, y1_bits, BF16, "y1")

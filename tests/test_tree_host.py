@@ -316,3 +316,52 @@ def test_torch_dlpack_capsule(S):
     view = DLTensor.from_address(tree.nodes[0].dl)
     assert (view.ndim, view.dtype.code, view.dtype.bits, view.device.device_type) == (2, 4, 16, 1)
     assert view.data + view.byte_offset == t.data_ptr()
+
+
+def _node_fields(nodes, n):
+    out = []
+    for i in range(n):
+        d = nodes[i]
+        t = d.t
+        out.append((d.kind, d.n, d.first, d.i, d.f, (t.data or 0, t.dtype, t.ndim, t.device,
+                                                      tuple(t.shape[:t.ndim]), tuple(t.stride[:t.ndim]))
+                    if d.kind == 1 else None))
+    return out
+
+
+def test_c_packer_builds_the_same_tree_as_the_python_builder(S):
+    torch = pytest.importorskip("torch")
+    fc = S.fastcall()
+    if fc is None:
+        pytest.skip("Python headers not installed: no CPython shim")
+    x = torch.zeros((4, 8), dtype=torch.bfloat16)
+    m = torch.zeros((4, 8), dtype=torch.bool)
+    v = torch.zeros((2, 3, 4), dtype=torch.float16)[:, 1:, ::2]  # a strided view
+    seen = []
+
+    def hook(scm, nodes, nargs, nnodes, stream):
+        seen.append((nargs, _node_fields(nodes, nnodes)))
+        return None
+
+    s = S.Scm(device=0, flags=S.OPT_DRY_RUN)
+    s.set_tree_hook(hook)
+    calls = [
+        (x, None, (m, (v, 3, [True, 2.5])), -7, 1e-6),
+        tuple(range(70)),                 # more nodes than the packer's stack buffer
+        ([x] * 40, [[x, v]] * 20),        # lists, nested, grown past the stack buffer
+        (),
+    ]
+    for args in calls:
+        assert fc.invoke_py(s.h.value, 0, *args) == S.MISS_HANDLED
+        t = S.Tree(*args)
+        assert seen[-1] == (t.nargs, _node_fields(t.nodes, t.nnodes))
+    with pytest.raises(TypeError):
+        fc.invoke_py(s.h.value, 0, x, "a string")
+    with pytest.raises(TypeError):
+        fc.invoke_py(s.h.value, 0, torch.zeros(2, dtype=torch.complex64))
+    with pytest.raises(ValueError):
+        fc.invoke_py(s.h.value, 0, torch.zeros((1, 1, 1, 1, 1)))
+    with pytest.raises(ValueError):
+        fc.invoke_py(s.h.value, 0, tuple(range(5000)))
+    assert len(seen) == len(calls)
+    s.close()
