@@ -818,20 +818,23 @@ def bench_kernels(c, n_calls=30):
     return out
 
 
-def bench_sweep(c, reps=20, quick=False):
+def bench_sweep(c, reps=20, quick=False, tokens=None):
     """HBM bandwidth sweep: add+RMSNorm (H 8192) and SwiGLU (I 28672) at T = 2^0..2^15,
     bf16. Each size: `reps` back-to-back launches from one native call, rotating across
     row windows of arenas sized for 32768 tokens so no launch reads what the previous
-    left in L2 (for T >= 512 the buffers alone exceed L2)."""
+    left in L2 (for T >= 512 the buffers alone exceed L2). With `tokens`, only those sizes,
+    on arenas of four windows of the largest (for profiling a few GB at most)."""
     t, S, synth = c.torch, c.S, c.synth
     H, I, Tmax = 8192, 28672, 32768
+    if tokens:
+        Tmax = 4 * max(tokens)
     peak, _ = measured_peaks()
     s = S.Scm(device=c.dev.index or 0)
     s.register(S.make_spec(S.OP_ADD_RMSNORM, S.BF16, [H], 1, 1 << 20))
     s.register(S.make_spec(S.OP_SWIGLU, S.BF16, [I], 1, 1 << 20))
     out = {"add_rmsnorm": [], "swiglu": []}
     seq = c.L.trident_scm_invoke_seq
-    Ts = [2 ** k for k in range(16)] if not quick else [1, 64, 4096, 32768]
+    Ts = list(tokens) if tokens else ([2 ** k for k in range(16)] if not quick else [1, 64, 4096, 32768])
     # add + RMSNorm
     x = synth.act_device((Tmax, H), S.BF16, 11, c.dev)
     r = synth.act_device((Tmax, H), S.BF16, 12, c.dev)
@@ -945,6 +948,7 @@ def run_ours(a):
 
     extra = {}
     want = (lambda name: True) if a.sections == "all" else (lambda name: name in a.sections.split(","))
+    toks_arg = [int(x) for x in a.tokens.split(",")] if a.tokens else None
     if rank == 0 and want("layers"):
         progress("per-token layer steps")
         per_t = {}
@@ -954,7 +958,7 @@ def run_ours(a):
     if rank == 0 and want("qwen3"):
         progress("qwen3 36-layer steps")
         qw = {}
-        toks = [int(x) for x in a.tokens.split(",")] if a.tokens else (
+        toks = toks_arg or (
             (1, 8, 32, 128) if not a.quick else (1, 128))
         for T in toks:
             qw[str(T)], _ = bench_layer(c, synth.QWEN3, T, K=max(20, min(K, 2000) // 36), W=W,
@@ -974,7 +978,7 @@ def run_ours(a):
         extra["kernel_benchmark"] = bench_kernels(c)
     if rank == 0 and want("sweep"):
         progress("hbm sweep")
-        extra["hbm_sweep"] = bench_sweep(c, quick=a.quick)
+        extra["hbm_sweep"] = bench_sweep(c, quick=a.quick, tokens=toks_arg)
     if rank == 0 and want("roofline"):
         progress("roofline kernel")
         kd = kernel_duration_chain(c, cfg, HEADLINE_T)
@@ -1073,7 +1077,7 @@ def main():
     p.add_argument("--warmup", type=int, default=20)
     p.add_argument("--impl", default="ours", choices=["ours", "reference"])
     p.add_argument("--quick", action="store_true", help="smaller sections (for smoke runs)")
-    p.add_argument("--tokens", default="", help="comma list of token counts for the qwen3 section")
+    p.add_argument("--tokens", default="", help="comma list of token counts for the qwen3 and sweep sections")
     p.add_argument("--sections", default="all",
                    help="comma list of: layers,qwen3,host,stress,motivation,kernels,sweep,roofline,e2e,cpu"
                         " (default all;"
