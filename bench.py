@@ -823,11 +823,11 @@ def bench_sweep(c, reps=20, quick=False, tokens=None):
     bf16. Each size: `reps` back-to-back launches from one native call, rotating across
     row windows of arenas sized for 32768 tokens so no launch reads what the previous
     left in L2 (for T >= 512 the buffers alone exceed L2). With `tokens`, only those sizes,
-    on arenas of four windows of the largest (for profiling a few GB at most)."""
+    on arenas of two windows of the largest (for profiling a few GB at most)."""
     t, S, synth = c.torch, c.S, c.synth
     H, I, Tmax = 8192, 28672, 32768
     if tokens:
-        Tmax = 4 * max(tokens)
+        Tmax = 2 * max(tokens)
     peak, _ = measured_peaks()
     s = S.Scm(device=c.dev.index or 0)
     s.register(S.make_spec(S.OP_ADD_RMSNORM, S.BF16, [H], 1, 1 << 20))
