@@ -395,8 +395,15 @@ def bench_layer(c, cfg, T, K, W, layers=1, min_bytes=2 * L2_BYTES):
 
 def bench_e2e(c, cfg, T, K, W):
     """End to end through the public API: per step, one pinned host -> device copy of the
-    layer's inputs (h, r0, attn_out, qkv, gate|up, pos laid out in one staging arena),
-    one invoke, one device -> host copy of its outputs (x1, x2, r2, o in one arena)."""
+    layer's inputs (h, r0, attn_out, qkv, gate|up, pos laid out in one staging arena), one
+    invoke, one device -> host copy of its outputs (x1, x2, r2, o in one arena).
+
+    Steps are double-buffered over three streams, as a serving engine overlaps transfers:
+    step i+1's input copy (copy-in stream) runs while step i's kernel (the bench stream) and
+    step i's output copy (copy-out stream) run; events order each buffer's reuse. The timed
+    region starts before the first step's input copy and ends after the last step's output
+    copy. The same steps issued serially (copy in, invoke, copy out on one stream) are
+    reported beside it."""
     t, S, synth = c.torch, c.S, c.synth
     H, Hq, Hkv, D, Sl, I = (cfg[k] for k in ("H", "Hq", "Hkv", "D", "S", "I"))
     Wq = (Hq + 2 * Hkv) * D
@@ -412,48 +419,109 @@ def bench_e2e(c, cfg, T, K, W):
     out_parts = [T * H * 2, T * H * 2, T * H * 2, T * I * 2]
     ioffs, itot = layout(in_parts)
     ooffs, otot = layout(out_parts)
-    dev_in = t.empty(itot, dtype=t.uint8, device=c.dev)
-    dev_out = t.empty(otot, dtype=t.uint8, device=c.dev)
-    host_in = t.empty(itot, dtype=t.uint8, pin_memory=True)
-    host_out = t.empty(otot, dtype=t.uint8, pin_memory=True)
     view = lambda buf, o, n, dt, shape: buf[o:o + n].view(dt).view(shape)
     bf = t.bfloat16
-    h = view(dev_in, ioffs[0], in_parts[0], bf, (T, H))
-    r0 = view(dev_in, ioffs[1], in_parts[1], bf, (T, H))
-    ao = view(dev_in, ioffs[2], in_parts[2], bf, (T, H))
-    qkv = view(dev_in, ioffs[3], in_parts[3], bf, (T, Wq))
-    gu = view(dev_in, ioffs[4], in_parts[4], bf, (T, 2 * I))
-    pos = view(dev_in, ioffs[5], in_parts[5], t.int32, (T,))
-    for k, tv in enumerate((h, r0, ao, qkv, gu)):
-        tv.copy_(synth.act_device(tuple(tv.shape), S.BF16, 40 + k, c.dev))
-    pos.copy_(t.from_numpy(synth.positions(np.random.default_rng(1), T, Sl)).to(c.dev))
-    host_in.copy_(dev_in)
-    x1 = view(dev_out, ooffs[0], out_parts[0], bf, (T, H))
-    x2 = view(dev_out, ooffs[1], out_parts[1], bf, (T, H))
-    r2 = view(dev_out, ooffs[2], out_parts[2], bf, (T, H))
-    o = view(dev_out, ooffs[3], out_parts[3], bf, (T, I))
     r1 = t.empty((T, H), dtype=bf, device=c.dev)
     kc = t.zeros((Hkv, Sl, D), dtype=bf, device=c.dev)
     vc = t.zeros((Hkv, Sl, D), dtype=bf, device=c.dev)
     ga, gm = synth.gamma_device(H, 50, c.dev), synth.gamma_device(H, 51, c.dev)
-    ts = [h, r0, ga, x1, r1, qkv[:, :Hq * D].view(T, Hq, D), qkv[:, Hq * D:(Hq + Hkv) * D].view(T, Hkv, D),
-          qkv[:, (Hq + Hkv) * D:].view(T, Hkv, D), pos, kc, vc, ao, gm, x2, r2, gu[:, :I], gu[:, I:], o]
     scm = layer_scm(c, cfg)
-    a = S.make_args(S.OP_LAYER_CHAIN, ts, eps=cfg["eps"], rope_theta=cfg["theta"])
-    addr = ctypes.addressof(a)
+    bufs = []
+    for k in range(2):
+        dev_in = t.empty(itot, dtype=t.uint8, device=c.dev)
+        dev_out = t.empty(otot, dtype=t.uint8, device=c.dev)
+        host_in = t.empty(itot, dtype=t.uint8, pin_memory=True)
+        host_out = t.empty(otot, dtype=t.uint8, pin_memory=True)
+        h = view(dev_in, ioffs[0], in_parts[0], bf, (T, H))
+        r0 = view(dev_in, ioffs[1], in_parts[1], bf, (T, H))
+        ao = view(dev_in, ioffs[2], in_parts[2], bf, (T, H))
+        qkv = view(dev_in, ioffs[3], in_parts[3], bf, (T, Wq))
+        gu = view(dev_in, ioffs[4], in_parts[4], bf, (T, 2 * I))
+        pos = view(dev_in, ioffs[5], in_parts[5], t.int32, (T,))
+        for j, tv in enumerate((h, r0, ao, qkv, gu)):
+            tv.copy_(synth.act_device(tuple(tv.shape), S.BF16, 40 + 10 * k + j, c.dev))
+        pos.copy_(t.from_numpy(synth.positions(np.random.default_rng(1 + k), T, Sl)).to(c.dev))
+        host_in.copy_(dev_in)
+        x1 = view(dev_out, ooffs[0], out_parts[0], bf, (T, H))
+        x2 = view(dev_out, ooffs[1], out_parts[1], bf, (T, H))
+        r2 = view(dev_out, ooffs[2], out_parts[2], bf, (T, H))
+        o = view(dev_out, ooffs[3], out_parts[3], bf, (T, I))
+        ts = [h, r0, ga, x1, r1, qkv[:, :Hq * D].view(T, Hq, D), qkv[:, Hq * D:(Hq + Hkv) * D].view(T, Hkv, D),
+              qkv[:, (Hq + Hkv) * D:].view(T, Hkv, D), pos, kc, vc, ao, gm, x2, r2, gu[:, :I], gu[:, I:], o]
+        a = S.make_args(S.OP_LAYER_CHAIN, ts, eps=cfg["eps"], rope_theta=cfg["theta"])
+        bufs.append(dict(dev_in=dev_in, dev_out=dev_out, host_in=host_in, host_out=host_out, args=a,
+                         addr=ctypes.addressof(a)))
+    t.cuda.synchronize()
     inv = c.invoker(scm)
+    main = c.stream
+    s_in, s_out = t.cuda.Stream(device=c.dev), t.cuda.Stream(device=c.dev)
+    ev = lambda: t.cuda.Event()
+    kdone = [ev(), ev()]    # kernel k finished reading dev_in[k]
+    odone = [ev(), ev()]    # output copy k finished reading dev_out[k]
+    ready = [ev(), ev()]    # input copy k landed
+    made = [ev(), ev()]     # kernel k wrote dev_out[k]
+    started = [False, False]
 
-    def step(i):
-        dev_in.copy_(host_in, non_blocking=True)
-        inv(addr)
-        host_out.copy_(dev_out, non_blocking=True)
+    def pipelined(i):
+        k = i % 2
+        b = bufs[k]
+        with t.cuda.stream(s_in):
+            if started[k]:
+                s_in.wait_event(kdone[k])
+            b["dev_in"].copy_(b["host_in"], non_blocking=True)
+            ready[k].record(s_in)
+        main.wait_event(ready[k])
+        if started[k]:
+            main.wait_event(odone[k])
+        inv(b["addr"])
+        kdone[k].record(main)
+        made[k].record(main)
+        with t.cuda.stream(s_out):
+            s_out.wait_event(made[k])
+            b["host_out"].copy_(b["dev_out"], non_blocking=True)
+            odone[k].record(s_out)
+        started[k] = True
 
-    us, host_us = time_steps(c, step, K, W)
+    def run(fn, n):
+        e0, e1 = c.events()
+        e0.record(main)
+        s_in.wait_event(e0)
+        s_out.wait_event(e0)
+        for i in range(n):
+            fn(i)
+        for k in range(2):
+            if started[k]:
+                main.wait_event(odone[k])
+        e1.record(main)
+        t.cuda.synchronize()
+        return e0.elapsed_time(e1) * 1e3 / max(n, 1)
+
+    run(pipelined, W)
+    us = run(pipelined, K)
+    # each buffer's inputs are the same every step and the kernel is deterministic, so the
+    # pipelined outputs must equal a serial recomputation byte for byte
+    piped = [b["host_out"].clone() for b in bufs]
+
+    def serial(i):
+        b = bufs[i % 2]
+        b["dev_in"].copy_(b["host_in"], non_blocking=True)
+        inv(b["addr"])
+        b["host_out"].copy_(b["dev_out"], non_blocking=True)
+
+    with t.cuda.stream(main):
+        time_steps(c, serial, W, 1)
+        serial_us, _ = time_steps(c, serial, K, W)
+    t.cuda.synchronize()
+    for k, b in enumerate(bufs):
+        if not t.equal(piped[k], b["host_out"]):
+            raise RuntimeError("e2e: pipelined outputs differ from the serial recomputation")
     assert_all_hit(scm, "e2e")
-    c.launches += K
+    c.launches += 3 * W + 2 * K + 1  # pipelined W + K, serial (W + 1) + (W + K)
     scm.close()
     return dict(value=round(us, 3), unit=UNIT, h2d_bytes_per_step=int(sum(in_parts)),
-                d2h_bytes_per_step=int(sum(out_parts)), copies_per_step=2)
+                d2h_bytes_per_step=int(sum(out_parts)), copies_per_step=2,
+                pipeline="double-buffered: input copy of step i+1 overlaps kernel and output copy of step i",
+                serial_us=round(serial_us, 3))
 
 
 def bench_host_hit(c, n=1000):
