@@ -13,6 +13,8 @@
 
 namespace trident {
 
+// The row in registers: x and r as packed 16-byte vectors, gamma and the fp32 sum
+// s = x + r as floats (thread `tid` owns vectors v*256 + tid, v < VPT: coalesced).
 template <int DT, int VPT>
 __global__ void __launch_bounds__(kThreads) addnorm_vec_kernel(const AddNormParams p) {
   pdl_prologue();
@@ -21,12 +23,44 @@ __global__ void __launch_bounds__(kThreads) addnorm_vec_kernel(const AddNormPara
   constexpr int VE = Act<DT>::VE;
   const int tid = threadIdx.x;
   for (int64_t row = blockIdx.x; row < p.T; row += gridDim.x) {
-    AddNormRegs<DT, VPT> R;
-    R.load(row_ptr(p.x, row, p.x_rs, EB), row_ptr(p.r, row, p.r_rs, EB), p.gamma, tid);
-    float s[VPT][VE];
-    const float ss = R.residual(row_ptr(p.r_out, row, p.ro_rs, EB), tid, s);
-    const float tot = block_sum(ss, red);
-    R.normalize(row_ptr(p.y, row, p.y_rs, EB), tid, s, rsqrtf(tot * p.inv_H + p.eps));
+    const uint4* xp = reinterpret_cast<const uint4*>(row_ptr(p.x, row, p.x_rs, EB));
+    const uint4* rp = reinterpret_cast<const uint4*>(row_ptr(p.r, row, p.r_rs, EB));
+    uint4 xv[VPT], rv[VPT];
+    float g[VPT][VE], s[VPT][VE];
+#pragma unroll
+    for (int v = 0; v < VPT; ++v) {
+      const int64_t vi = (int64_t)v * kThreads + tid;
+      xv[v] = ldg16(xp + vi);
+      rv[v] = ldg16(rp + vi);
+#pragma unroll
+      for (int q = 0; q < VE / 4; ++q) {
+        const float4 gg = ldg_f4(p.gamma + vi * VE + 4 * q);
+        g[v][4 * q] = gg.x; g[v][4 * q + 1] = gg.y; g[v][4 * q + 2] = gg.z; g[v][4 * q + 3] = gg.w;
+      }
+    }
+    uint4* rop = reinterpret_cast<uint4*>(row_ptr(p.r_out, row, p.ro_rs, EB));
+    float ss = 0.f;
+#pragma unroll
+    for (int v = 0; v < VPT; ++v) {
+      float xf[VE], rf[VE];
+      unpack<DT>(xv[v], xf);
+      unpack<DT>(rv[v], rf);
+#pragma unroll
+      for (int e = 0; e < VE; ++e) {
+        s[v][e] = xf[e] + rf[e];
+        ss = fmaf(s[v][e], s[v][e], ss);
+      }
+      st16(rop + (int64_t)v * kThreads + tid, pack<DT>(s[v]));
+    }
+    const float inv = rsqrtf(block_sum(ss, red) * p.inv_H + p.eps);
+    uint4* yp = reinterpret_cast<uint4*>(row_ptr(p.y, row, p.y_rs, EB));
+#pragma unroll
+    for (int v = 0; v < VPT; ++v) {
+      float y[VE];
+#pragma unroll
+      for (int e = 0; e < VE; ++e) y[e] = s[v][e] * inv * g[v][e];
+      st16(yp + (int64_t)v * kThreads + tid, pack<DT>(y));
+    }
     __syncthreads();  // `red` is reused by the next row
   }
 }

@@ -140,61 +140,6 @@ __device__ __forceinline__ float block_sum(float v, float* red) {
   return t;
 }
 
-// ---------------------------------------------------------------- add + RMSNorm row
-// One row of H = VPT * kThreads * VE elements held in registers by one block.
-// Thread `tid` owns vectors v*kThreads + tid, v < VPT (coalesced 16-byte accesses).
-template <int DT, int VPT>
-struct AddNormRegs {
-  static constexpr int VE = Act<DT>::VE;
-  uint4 xv[VPT], rv[VPT];
-  float g[VPT][VE];
-
-  __device__ __forceinline__ void load(const void* x_row, const void* r_row, const float* gamma,
-                                       int tid) {
-#pragma unroll
-    for (int v = 0; v < VPT; ++v) {
-      const int64_t vi = (int64_t)v * kThreads + tid;
-      xv[v] = ldg16(reinterpret_cast<const uint4*>(x_row) + vi);
-      rv[v] = ldg16(reinterpret_cast<const uint4*>(r_row) + vi);
-#pragma unroll
-      for (int q = 0; q < VE / 4; ++q) {
-        float4 gg = ldg_f4(gamma + vi * VE + 4 * q);
-        g[v][4 * q] = gg.x; g[v][4 * q + 1] = gg.y; g[v][4 * q + 2] = gg.z; g[v][4 * q + 3] = gg.w;
-      }
-    }
-  }
-  // s = x + r (fp32); stores round(s) to r_out (and leaves it in rv); returns sum(s^2)
-  // of this thread; s is left in `s`.
-  __device__ __forceinline__ float residual(void* ro_row, int tid, float (&s)[VPT][VE]) {
-    float ss = 0.f;
-#pragma unroll
-    for (int v = 0; v < VPT; ++v) {
-      float xf[VE], rf[VE];
-      unpack<DT>(xv[v], xf);
-      unpack<DT>(rv[v], rf);
-#pragma unroll
-      for (int e = 0; e < VE; ++e) {
-        s[v][e] = xf[e] + rf[e];
-        ss = fmaf(s[v][e], s[v][e], ss);
-      }
-      rv[v] = pack<DT>(s[v]);
-      st16(reinterpret_cast<uint4*>(ro_row) + (int64_t)v * kThreads + tid, rv[v]);
-    }
-    return ss;
-  }
-
-  __device__ __forceinline__ void normalize(void* y_row, int tid, const float (&s)[VPT][VE],
-                                            float inv) {
-#pragma unroll
-    for (int v = 0; v < VPT; ++v) {
-      float y[VE];
-#pragma unroll
-      for (int e = 0; e < VE; ++e) y[e] = s[v][e] * inv * g[v][e];
-      st16(reinterpret_cast<uint4*>(y_row) + (int64_t)v * kThreads + tid, pack<DT>(y));
-    }
-  }
-};
-
 // ---------------------------------------------------------------- RoPE angles
 // sin and cos of the angle pos * f, with f = fhi + flo (a double-float split of
 // theta^(-2i/D) made in fp64 on the host). The product is kept as ah + al (al holds the

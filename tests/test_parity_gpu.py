@@ -43,6 +43,8 @@ ADDNORM_CASES = [
     (BF16, 4096, 13, "strided", 0, "row-strided views"),
     (BF16, 4096, 21, "rank3", 0, "[3, 7, H] flattened"),
     (BF16, 8192, 19, "contig", 0, "register row, H 8192"),
+    (BF16, 8192, 1500, "contig", 0, "H 8192 persistent grid: several rows per block"),
+    (FP16, 8192, 700, "strided", 0, "fp16 H 8192 persistent, row-strided"),
     (BF16, 2048, 5, "contig", 0, "register row, H 2048"),
     (BF16, 1000, 5, "contig", 0, "two-pass vector loop, ragged H"),
     (BF16, 100, 6, "contig", 0, "H*2 not a multiple of 16: generic"),
@@ -116,9 +118,10 @@ def test_add_rmsnorm_unaligned_rows_miss_an_aligned_version(S):
     s.close()
 
 
-@pytest.mark.parametrize("H,variant", [(4096, 0), (1000, 0), (100, 0), (4096, 1)])
-def test_add_rmsnorm_in_place(S, H, variant):
-    got_y, got_r, y_ref, y_bits, ro_bits = run_addnorm(S, BF16, H, 7, "contig", variant, inplace=True)
+@pytest.mark.parametrize("H,variant,T", [(4096, 0, 7), (1000, 0, 7), (100, 0, 7), (4096, 1, 7),
+                                         (8192, 0, 1300)])
+def test_add_rmsnorm_in_place(S, H, variant, T):
+    got_y, got_r, y_ref, y_bits, ro_bits = run_addnorm(S, BF16, H, T, "contig", variant, inplace=True)
     assert np.array_equal(got_r, ro_bits)
     P.check_act(got_y, y_ref, y_bits, BF16, "y in place")
 
