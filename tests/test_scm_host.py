@@ -67,14 +67,20 @@ def test_struct_layout_matches_header(S, tmp_path):
         "int main(void){printf(\"%zu %zu %zu %zu %zu %zu %zu %zu\\n\", sizeof(trident_tensor),"
         " sizeof(trident_args), offsetof(trident_args, t), sizeof(trident_spec_desc),"
         " offsetof(trident_spec_desc, rope_theta), sizeof(trident_scm_options),"
-        " sizeof(trident_scm_stats_t), offsetof(trident_tensor, dtype)); return 0;}\n")
+        " sizeof(trident_scm_stats_t), offsetof(trident_tensor, dtype)); "
+        "printf(\"%zu %zu %zu %zu %zu %zu %zu\\n\", sizeof(trident_node), offsetof(trident_node, dl),"
+        " offsetof(trident_node, t), sizeof(trident_recipe_node), offsetof(trident_recipe_node, f),"
+        " sizeof(trident_recipe), offsetof(trident_recipe, eps)); return 0;}\n")
     exe = tmp_path / "layout"
     subprocess.run(["gcc", "-I", os.path.join(ROOT, "include"), str(src), "-o", str(exe)], check=True)
     got = [int(v) for v in subprocess.run([str(exe)], capture_output=True, text=True).stdout.split()]
     want = [ctypes.sizeof(S.trident_tensor), ctypes.sizeof(S.trident_args),
             S.trident_args.t.offset, ctypes.sizeof(S.trident_spec_desc),
             S.trident_spec_desc.rope_theta.offset, ctypes.sizeof(S.trident_scm_options),
-            ctypes.sizeof(S.trident_scm_stats_t), S.trident_tensor.dtype.offset]
+            ctypes.sizeof(S.trident_scm_stats_t), S.trident_tensor.dtype.offset,
+            ctypes.sizeof(S.trident_node), S.trident_node.dl.offset, S.trident_node.t.offset,
+            ctypes.sizeof(S.trident_recipe_node), S.trident_recipe_node.f.offset,
+            ctypes.sizeof(S.trident_recipe), S.trident_recipe.eps.offset]
     assert got == want
 
 
