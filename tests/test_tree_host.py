@@ -365,3 +365,61 @@ def test_c_packer_builds_the_same_tree_as_the_python_builder(S):
         fc.invoke_py(s.h.value, 0, tuple(range(5000)))
     assert len(seen) == len(calls)
     s.close()
+
+
+def test_tree_execution_error_is_raised_not_retried(S):
+    """As for invoke: a failed launch of the selected version (injected on the host) returns
+    ERR_CUDA at once -- no later version, no hook."""
+    x, r, w, y, ro = rms_inputs()
+    called = []
+    s = S.Scm(device=0, flags=S.OPT_DRY_RUN | S.OPT_FAIL_LAUNCHES)
+    s.set_tree_hook(lambda *a: called.append(1))
+    spec_a, rec_a = rms_table()[1]
+    for _ in range(2):
+        s.register_tree(cases.lib_spec(spec_a), cases.lib_recipe(rec_a))
+    assert s.invoke_tree(S.Tree(x, r, w, (y, ro), 1e-6)) == (S.ERR_CUDA, 0)
+    assert "injected" in S.trident_scm_last_error()
+    st = s.stats()
+    assert (st.hits, st.misses, st.err_cuda, st.hook_calls) == (0, 0, 1, 0) and not called
+    s.close()
+
+
+def test_concurrent_tree_and_step_calls_with_growth(S):
+    """Several threads call invoke_tree and invoke_step while another registers versions:
+    every call sees a consistent table (first match stays version 0) and no error."""
+    import threading
+    s = S.Scm(device=0, flags=S.OPT_DRY_RUN, max_specs=400)
+    spec_a, rec_a = rms_table()[1]
+    s.register_tree(cases.lib_spec(spec_a), cases.lib_recipe(rec_a))
+    x, r, w, y, ro = rms_inputs()
+    tree = S.Tree(x, r, w, (y, ro), 1e-6)
+    from tests.test_step_host import chain_call, chain_spec
+    s.register(cases.lib_spec(chain_spec()))
+    calls = (S.trident_args * 3)(*[cases.lib_args(chain_call(k)) for k in range(3)])
+    stop = threading.Event()
+    errors = []
+
+    def tree_reader():
+        while not stop.is_set():
+            got = S.trident_scm_invoke_tree(s.h, tree)
+            if got != (S.OK, 0):
+                errors.append(("tree", got))
+
+    def step_reader():
+        while not stop.is_set():
+            got = S.trident_scm_invoke_step(s.h, calls)
+            if got != (S.OK, [1, 1, 1]):
+                errors.append(("step", got))
+
+    th = [threading.Thread(target=f) for f in (tree_reader, tree_reader, step_reader, step_reader)]
+    for t in th:
+        t.start()
+    for _ in range(300):
+        s.register_tree(cases.lib_spec(spec_a), cases.lib_recipe(rec_a))
+    stop.set()
+    for t in th:
+        t.join()
+    assert not errors, errors[:3]
+    st = s.stats()
+    assert st.num_specs == 302 and st.fused_launches > 0 and st.hits == st.invokes
+    s.close()
