@@ -138,3 +138,39 @@ def test_step_fp16_longer_than_one_chunk(S):
     s.close()
     for inp, (_, out) in zip(inps, outs):
         check_chain(L.layer_chain(inp, cfg["theta"], cfg["eps"], FP16), out, inp, FP16)
+
+
+@pytest.mark.parametrize("entry", ["invoke", "step"])
+def test_dependent_layers_back_to_back_with_pdl(S, entry):
+    """Six Llama layers at 64 tokens where layer l+1's residual input is layer l's second
+    residual output, launched back to back with programmatic dependent launch (one invoke
+    each through the fast-call shim, or one invoke_step that must fall back to call-by-call
+    order). Each kernel's memory accesses wait for the previous kernel, so every layer equals
+    the oracle run in sequence."""
+    import ctypes
+    cfg = synth.LLAMA
+    T, n = 64, 6
+    s, op = step_scm(S, cfg, BF16, S.LAYOUT_ROWSTRIDED)
+    inps, outs, args = build_layers(S, cfg, T, n, seed=606)
+    for l in range(1, n):
+        ts = outs[l][0]
+        ts[1] = outs[l - 1][1]["r2"]
+        args[l] = S.make_args(op, ts, eps=cfg["eps"], rope_theta=cfg["theta"])
+    st = stream()
+    if entry == "invoke":
+        fc = S.fastcall()
+        for a in args:
+            rc = fc.invoke(s.h.value, ctypes.addressof(a), st) if fc else S.trident_scm_invoke(s.h, a, st)[0]
+            assert rc == S.OK, S.trident_scm_last_error()
+    else:
+        run_step(S, s, args)
+        assert s.stats().fused_launches == 0
+    torch.cuda.synchronize()
+    assert S.trident_scm_device_status(s.h, st)[1] == 0
+    s.close()
+    r0 = inps[0]["r0"]
+    for l in range(n):
+        inp = dict(inps[l], r0=r0)
+        ref = L.layer_chain(inp, cfg["theta"], cfg["eps"], BF16)
+        check_chain(ref, outs[l][1], inp)
+        r0 = ref["r2"]
