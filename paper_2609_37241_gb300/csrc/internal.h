@@ -87,6 +87,7 @@ struct ChainParams {
   SwigluParams sw;
   int32_t nA, nB, nC, sw_tiles_per_row;
   int32_t a_split;   // CTAs per token for the norms (2, or 1 for in-place calls)
+  int32_t prefetch;  // 1: each block prefetches its input lines into L2 before the PDL wait
   int64_t sw_tiles;  // T * sw_tiles_per_row (valid SwiGLU tiles)
 };
 

@@ -379,6 +379,7 @@ struct Version {
   CUfunction step_fn;           // layer chain: several calls per launch (two blocks per token)
   CUfunction step_fn_inplace;   // ... one block per token
   int32_t step_wave_blocks;     // blocks of `step_fn` resident at once
+  int32_t sm_count;             // layer chain: SMs of the device (grids up to this prefetch)
   const float2* inv_freq;
   Recipe* recipe;               // structured-argument binding (register_tree_spec), or NULL
 };
@@ -629,6 +630,7 @@ int32_t pack_chain(trident_scm* scm, const Version& v, const trident_args* a, co
   c->nC = (int32_t)nC;
   c->sw_tiles_per_row = (int32_t)tiles;
   c->sw_tiles = nC;
+  c->prefetch = 0;
   return TRIDENT_OK;
 }
 
@@ -717,6 +719,10 @@ int32_t do_launch(trident_scm* scm, const Version& v, const trident_args* a, con
       st = set_chain_split(&c, s.T, split, &blocks);
       if (st != TRIDENT_OK) return st;
       cfg.gridDimX = (unsigned)blocks;
+      // prefetch before the PDL wait only when the grid is at most one block per SM and
+      // the launch overlaps a previous kernel (measured: ~10% faster at 1-4 tokens, slower
+      // once the grid fills the GPU)
+      c.prefetch = (scm->opt.flags & TRIDENT_OPT_PDL) && blocks <= v.sm_count ? 1 : 0;
       break;
     }
     default:
@@ -1070,6 +1076,7 @@ int32_t append_version(trident_scm_t* scm, const trident_spec_desc* desc, int32_
           return fail(TRIDENT_ERR_CUDA, "occupancy query failed");
         v.wave_blocks = per_sm * sms;
         v.step_wave_blocks = step_per_sm * sms;
+        v.sm_count = sms;
       }
       if (v.rope) {
         const bool chain = desc->op == TRIDENT_OP_LAYER_CHAIN || desc->op == TRIDENT_OP_LAYER_CHAIN_QKNORM;
