@@ -17,11 +17,20 @@ namespace trident {
 // s = x + r as floats (thread `tid` owns vectors v*256 + tid, v < VPT: coalesced).
 template <int DT, int VPT>
 __global__ void __launch_bounds__(kThreads) addnorm_vec_kernel(const AddNormParams p) {
-  pdl_prologue();
+  pdl_trigger();
   __shared__ float red[kThreads / 32];
   constexpr int EB = Act<DT>::BYTES;
   constexpr int VE = Act<DT>::VE;
   const int tid = threadIdx.x;
+  if (p.prefetch && (tid & 7) == 0 && blockIdx.x < p.T) {  // the first row's lines (prefetch_l2)
+#pragma unroll
+    for (int v = 0; v < VPT; ++v) {
+      const int64_t vi = (int64_t)v * kThreads + tid;
+      prefetch_l2(reinterpret_cast<const uint4*>(row_ptr(p.x, blockIdx.x, p.x_rs, EB)) + vi);
+      prefetch_l2(reinterpret_cast<const uint4*>(row_ptr(p.r, blockIdx.x, p.r_rs, EB)) + vi);
+    }
+  }
+  pdl_wait();
   for (int64_t row = blockIdx.x; row < p.T; row += gridDim.x) {
     const uint4* xp = reinterpret_cast<const uint4*>(row_ptr(p.x, row, p.x_rs, EB));
     const uint4* rp = reinterpret_cast<const uint4*>(row_ptr(p.r, row, p.r_rs, EB));

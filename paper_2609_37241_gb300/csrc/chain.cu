@@ -142,23 +142,16 @@ __device__ __forceinline__ void chain_block(const ChainParams& c, const int b) {
   }
 }
 
-// L2 prefetch of the lines block b will read first -- the norm rows, the RoPE head-rows and
-// positions, the SwiGLU tile -- one prefetch per 128-byte line. It is issued between the
-// programmatic launch trigger and griddepcontrol.wait, while the previous kernel of the
-// stream may still run: a prefetch has no effect on the values later loads return (the
-// loads themselves come after the wait), it only lets the DRAM fetch overlap the previous
-// kernel's tail and the launch handoff. The host enables it only for grids of at most one
-// block per SM: a grid that fills the GPU becomes resident only as the previous kernel's
-// blocks retire, and its prefetches then compete with that kernel for DRAM.
-__device__ __forceinline__ void prefetch_l2(const void* p) { asm volatile("prefetch.L2 [%0];" :: "l"(p)); }
-
+// L2 prefetch of the lines block b reads first -- the norm rows, the RoPE head-rows and
+// positions, the SwiGLU tile -- one prefetch per 128-byte line, between the launch trigger
+// and the PDL wait (see prefetch_l2).
 template <int DT, int VPT, int SPLIT, int D>
 __device__ __forceinline__ void chain_prefetch(const ChainParams& c, const int b) {
   constexpr int EB = Act<DT>::BYTES;
   constexpr int VE = Act<DT>::VE;
   const int tid = threadIdx.x;
-  if ((tid & 7) != 0) return;  // 8 threads x 16 bytes = one line
   if (b < c.nA) {
+    if ((tid & 7) != 0) return;  // 8 threads x 16 bytes = one line
     const int64_t row = b / SPLIT;
     const uint4* hp = reinterpret_cast<const uint4*>(row_ptr(c.n1.x, row, c.n1.x_rs, EB));
     const uint4* rp = reinterpret_cast<const uint4*>(row_ptr(c.n1.r, row, c.n1.r_rs, EB));
@@ -172,35 +165,13 @@ __device__ __forceinline__ void chain_prefetch(const ChainParams& c, const int b
     }
   } else if (b < c.nA + c.nB) {
     constexpr int LPH = D / VE;
-    const RopeParams& p = c.rope;
-    const int64_t unit = (int64_t)(b - c.nA) * (kThreads / LPH) + tid / LPH;
-    if (unit >= p.T * p.NH) return;
-    const int lane = tid % LPH;
-    const int64_t t = unit / p.NH;
-    const int hh = (int)(unit - t * p.NH);
-    const bool is_q = hh < p.Hq, is_v = hh >= p.Hq + p.Hkv;
-    const int h = is_q ? hh : (is_v ? hh - p.Hq - p.Hkv : hh - p.Hq);
-    const char* src = is_q ? row_ptr(p.q, t, p.q_rs, EB) : is_v ? row_ptr(p.v, t, p.v_rs, EB)
-                                                               : row_ptr(p.k, t, p.k_rs, EB);
-    prefetch_l2(src + ((int64_t)h * D + lane * VE) * EB);
-    if (lane == 0) prefetch_l2(p.pos + t);
+    rope_prefetch<DT, D>(c.rope, (int64_t)(b - c.nA) * (kThreads / LPH) + tid / LPH, tid % LPH);
   } else {
     const int64_t tile = b - c.nA - c.nB;
     if (tile >= c.sw_tiles) return;
-    const SwigluParams& p = c.sw;
     const int64_t row = tile / c.sw_tiles_per_row;
-    const int64_t v0 = (tile - row * c.sw_tiles_per_row) * kChainSwigluUnroll * kThreads;
-    const int64_t nvec = p.I / VE;
-    const uint4* g = reinterpret_cast<const uint4*>(row_ptr(p.g, row, p.g_rs, EB));
-    const uint4* u = reinterpret_cast<const uint4*>(row_ptr(p.u, row, p.u_rs, EB));
-#pragma unroll
-    for (int k = 0; k < kChainSwigluUnroll; ++k) {
-      const int64_t vi = v0 + (int64_t)k * kThreads + tid;
-      if (vi < nvec) {
-        prefetch_l2(g + vi);
-        prefetch_l2(u + vi);
-      }
-    }
+    swiglu_prefetch<DT, kChainSwigluUnroll>(
+        c.sw, row, (tile - row * c.sw_tiles_per_row) * kChainSwigluUnroll * kThreads, tid);
   }
 }
 
@@ -209,9 +180,9 @@ __device__ __forceinline__ void chain_prefetch(const ChainParams& c, const int b
 template <int DT, int VPT, int SPLIT, int D, bool QKNORM>
 __global__ void __launch_bounds__(kThreads, VPT == 2 ? 4 : 2)
     chain_kernel(const __grid_constant__ ChainParams c) {
-  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+  pdl_trigger();
   if (c.prefetch) chain_prefetch<DT, VPT, SPLIT, D>(c, blockIdx.x);
-  asm volatile("griddepcontrol.wait;" ::: "memory");
+  pdl_wait();
   chain_block<DT, VPT, SPLIT, D, QKNORM>(c, blockIdx.x);
 }
 

@@ -17,10 +17,23 @@ namespace trident {
 
 constexpr uint32_t kErrPos = 0x1u;  // TRIDENT_DEVERR_POS
 
-__device__ __forceinline__ void pdl_prologue() {
+__device__ __forceinline__ void pdl_trigger() {
   asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
-  asm volatile("griddepcontrol.wait;" ::: "memory");
 }
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_prologue() {
+  pdl_trigger();
+  pdl_wait();
+}
+
+// L2 prefetch of one line. Kernels issue prefetches of the lines they read first between
+// pdl_trigger and pdl_wait, while the previous kernel of the stream may still run: a
+// prefetch changes no value that a later load returns (the loads come after the wait), it
+// only lets the DRAM fetch overlap the previous kernel's tail and the launch handoff. The
+// host enables it (params.prefetch) for grids of at most one block per SM launched with
+// programmatic stream serialisation: a grid that fills the GPU becomes resident only as the
+// previous kernel's blocks retire, and its prefetches then compete with that kernel.
+__device__ __forceinline__ void prefetch_l2(const void* p) { asm volatile("prefetch.L2 [%0];" :: "l"(p)); }
 
 template <int DT> struct Act;
 template <> struct Act<DT_BF16> { static constexpr int VE = 8; static constexpr int BYTES = 2; };
@@ -164,6 +177,22 @@ __device__ __forceinline__ void rope_sincos(float pos, float fhi, float flo, flo
 }
 
 // ---------------------------------------------------------------- RoPE head-row
+// L2 prefetch of head-row `unit`'s source line(s) and position (lanes on a line boundary).
+template <int DT, int D>
+__device__ __forceinline__ void rope_prefetch(const RopeParams& p, int64_t unit, int lane) {
+  constexpr int VE = Act<DT>::VE;
+  constexpr int EB = Act<DT>::BYTES;
+  if (unit >= p.T * p.NH || (lane * VE * EB) % 128 != 0) return;
+  const int64_t t = unit / p.NH;
+  const int hh = (int)(unit - t * p.NH);
+  const bool is_q = hh < p.Hq, is_v = hh >= p.Hq + p.Hkv;
+  const int h = is_q ? hh : (is_v ? hh - p.Hq - p.Hkv : hh - p.Hq);
+  const char* src = is_q ? row_ptr(p.q, t, p.q_rs, EB) : is_v ? row_ptr(p.v, t, p.v_rs, EB)
+                                                             : row_ptr(p.k, t, p.k_rs, EB);
+  prefetch_l2(src + ((int64_t)h * D + lane * VE) * EB);
+  if (lane == 0) prefetch_l2(p.pos + t);
+}
+
 // One head-row (token t, head hh) handled by LPH = D / VE consecutive lanes, each lane
 // owning VE consecutive elements. Rotate-half pairs element i with i + D/2, i.e. lane
 // l with lane l ^ (LPH/2). hh < Hq: q head (rotated in place); hh < Hq + Hkv: k head
@@ -262,6 +291,26 @@ template <> __device__ __forceinline__ float silu_mul<DT_FP16>(float g, float u)
 // fp32 outputs: full-precision exp and IEEE division.
 template <> __device__ __forceinline__ float silu_mul<DT_FP32>(float g, float u) {
   return g / (1.0f + expf(-g)) * u;
+}
+
+// L2 prefetch of the gate and up lines of one SwiGLU tile (threads on a line boundary).
+template <int DT, int UNROLL>
+__device__ __forceinline__ void swiglu_prefetch(const SwigluParams& p, int64_t row, int64_t v0,
+                                                int tid) {
+  constexpr int VE = Act<DT>::VE;
+  constexpr int EB = Act<DT>::BYTES;
+  if ((tid & 7) != 0 || row >= p.T) return;
+  const int64_t nvec = p.I / VE;
+  const uint4* g = reinterpret_cast<const uint4*>(row_ptr(p.g, row, p.g_rs, EB));
+  const uint4* u = reinterpret_cast<const uint4*>(row_ptr(p.u, row, p.u_rs, EB));
+#pragma unroll
+  for (int k = 0; k < UNROLL; ++k) {
+    const int64_t vi = v0 + (int64_t)k * kThreads + tid;
+    if (vi < nvec) {
+      prefetch_l2(g + vi);
+      prefetch_l2(u + vi);
+    }
+  }
 }
 
 // One tile of UNROLL * kThreads vectors of one row, starting at vector index v0.

@@ -24,6 +24,7 @@ struct AddNormParams {
   int64_t T, H;
   int64_t x_rs, r_rs, y_rs, ro_rs;
   float eps, inv_H;
+  int32_t prefetch;  // 1: prefetch this block's first lines into L2 before the PDL wait
 };
 
 // RMSNorm over T rows of H elements (no residual). Row strides in elements.
@@ -34,6 +35,7 @@ struct RmsNormParams {
   int64_t T, H;
   int64_t x_rs, y_rs;
   float eps, inv_H;
+  int32_t prefetch;
 };
 
 // Pointwise operators over T rows of W elements (a: x or the first addend; b: the second
@@ -47,6 +49,7 @@ struct PointwiseParams {
   int64_t T, W;
   int64_t a_rs, b_rs, m_rs, y_rs;
   float scalar;
+  int32_t prefetch;
 };
 
 // RoPE on q/k (optionally after per-head RMSNorm) plus KV-cache append.
@@ -67,6 +70,7 @@ struct RopeParams {
   int64_t q_rs, k_rs, v_rs;
   int32_t Hq, Hkv, D, NH;  // NH = Hq + 2 Hkv head-rows per token
   float eps, inv_D;
+  int32_t prefetch;
 };
 
 // out = silu(g) * u over T rows of I elements.
@@ -76,6 +80,7 @@ struct SwigluParams {
   void* out;
   int64_t T, I;
   int64_t g_rs, u_rs, o_rs;
+  int32_t prefetch;
 };
 
 // One decoder layer's chain in one launch. Blocks [0, nA) run the two add+RMSNorm steps

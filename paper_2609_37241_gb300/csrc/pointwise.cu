@@ -21,11 +21,22 @@ __device__ __forceinline__ float pw_apply(float a, float b, uint8_t m, float sca
 
 template <int DT, int OP, int UNROLL>
 __global__ void __launch_bounds__(kThreads) pointwise_vec_kernel(const PointwiseParams p) {
-  pdl_prologue();
+  pdl_trigger();
   constexpr int VE = Act<DT>::VE;
   constexpr int EB = Act<DT>::BYTES;
   const int64_t nvec = p.W / VE;
   const int64_t v0 = (int64_t)blockIdx.x * UNROLL * kThreads;
+  if (p.prefetch && (threadIdx.x & 7) == 0 && blockIdx.y < p.T) {  // the first row's tile (prefetch_l2)
+#pragma unroll
+    for (int k = 0; k < UNROLL; ++k) {
+      const int64_t vi = v0 + (int64_t)k * kThreads + threadIdx.x;
+      if (vi < nvec) {
+        prefetch_l2(reinterpret_cast<const uint4*>(row_ptr(p.a, blockIdx.y, p.a_rs, EB)) + vi);
+        if (OP == PW_ADD) prefetch_l2(reinterpret_cast<const uint4*>(row_ptr(p.b, blockIdx.y, p.b_rs, EB)) + vi);
+      }
+    }
+  }
+  pdl_wait();
   for (int64_t row = blockIdx.y; row < p.T; row += gridDim.y) {
     const uint4* a = reinterpret_cast<const uint4*>(row_ptr(p.a, row, p.a_rs, EB));
     const uint4* b = reinterpret_cast<const uint4*>(row_ptr(p.b, row, p.b_rs, EB));

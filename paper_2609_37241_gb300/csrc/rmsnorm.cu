@@ -15,11 +15,16 @@ namespace trident {
 
 template <int DT, int LPR>
 __global__ void __launch_bounds__(kThreads) rmsnorm_rows_kernel(const RmsNormParams p) {
-  pdl_prologue();
+  pdl_trigger();
   constexpr int VE = Act<DT>::VE;
   constexpr int EB = Act<DT>::BYTES;
   constexpr int RPB = kThreads / LPR;
   const int lane = threadIdx.x % LPR;
+  if (p.prefetch && (lane & 7) == 0) {  // the first row's lines (prefetch_l2)
+    const int64_t row0 = (int64_t)blockIdx.x * RPB + threadIdx.x / LPR;
+    if (row0 < p.T) prefetch_l2(row_ptr(p.x, row0, p.x_rs, EB) + (int64_t)lane * 16);
+  }
+  pdl_wait();
   const unsigned mask =
       (LPR == 32) ? 0xffffffffu : (((1u << LPR) - 1u) << ((threadIdx.x & 31) & ~(LPR - 1)));
   for (int64_t row = (int64_t)blockIdx.x * RPB + threadIdx.x / LPR; row < p.T;
@@ -47,11 +52,18 @@ __global__ void __launch_bounds__(kThreads) rmsnorm_rows_kernel(const RmsNormPar
 
 template <int DT, int VPT>
 __global__ void __launch_bounds__(kThreads) rmsnorm_vec_kernel(const RmsNormParams p) {
-  pdl_prologue();
+  pdl_trigger();
   __shared__ float red[kThreads / 32];
   constexpr int VE = Act<DT>::VE;
   constexpr int EB = Act<DT>::BYTES;
   const int tid = threadIdx.x;
+  if (p.prefetch && (tid & 7) == 0 && blockIdx.x < p.T) {  // the first row's lines (prefetch_l2)
+#pragma unroll
+    for (int v = 0; v < VPT; ++v)
+      prefetch_l2(reinterpret_cast<const uint4*>(row_ptr(p.x, blockIdx.x, p.x_rs, EB)) +
+                  (int64_t)v * kThreads + tid);
+  }
+  pdl_wait();
   for (int64_t row = blockIdx.x; row < p.T; row += gridDim.x) {
     const uint4* xr = reinterpret_cast<const uint4*>(row_ptr(p.x, row, p.x_rs, EB));
     uint4 xv[VPT];

@@ -13,11 +13,13 @@ namespace trident {
 
 template <int DT, int D, bool QKNORM>
 __global__ void __launch_bounds__(kThreads) rope_vec_kernel(const RopeParams p) {
-  pdl_prologue();
+  pdl_trigger();
   constexpr int LPH = D / Act<DT>::VE;
   constexpr int UPB = kThreads / LPH;
   const int64_t total = p.T * p.NH;
   const int lane = threadIdx.x % LPH;
+  if (p.prefetch) rope_prefetch<DT, D>(p, (int64_t)blockIdx.x * UPB + threadIdx.x / LPH, lane);
+  pdl_wait();
   for (int64_t unit = (int64_t)blockIdx.x * UPB + threadIdx.x / LPH; unit < total;
        unit += (int64_t)gridDim.x * UPB) {
     rope_head_row<DT, D, QKNORM>(p, unit, lane);

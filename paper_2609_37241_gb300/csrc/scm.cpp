@@ -379,7 +379,6 @@ struct Version {
   CUfunction step_fn;           // layer chain: several calls per launch (two blocks per token)
   CUfunction step_fn_inplace;   // ... one block per token
   int32_t step_wave_blocks;     // blocks of `step_fn` resident at once
-  int32_t sm_count;             // layer chain: SMs of the device (grids up to this prefetch)
   const float2* inv_freq;
   Recipe* recipe;               // structured-argument binding (register_tree_spec), or NULL
 };
@@ -404,6 +403,7 @@ struct trident_scm {
   int32_t device = 0;
   CUcontext ctx = nullptr;
   uint32_t* d_err = nullptr;
+  int32_t sm_count = 0;  // grids of at most this many blocks prefetch before the PDL wait
   std::vector<RopeTable> tables;
   // host timing of hits
   uint32_t* ring = nullptr;
@@ -521,6 +521,7 @@ void pack_addnorm(const trident_args* a, int x, int r, int g, int y, int ro, con
   p->y_rs = row_stride(t[y], kind); p->ro_rs = row_stride(t[ro], kind);
   p->eps = (float)a->eps;
   p->inv_H = (float)(1.0 / (double)p->H);
+  p->prefetch = 0;
 }
 
 void pack_rmsnorm(const trident_args* a, const Sig& s, RmsNormParams* p) {
@@ -531,6 +532,7 @@ void pack_rmsnorm(const trident_args* a, const Sig& s, RmsNormParams* p) {
   p->x_rs = row_stride(t[0], K_ACT_H); p->y_rs = row_stride(t[2], K_ACT_H);
   p->eps = (float)a->eps;
   p->inv_H = (float)(1.0 / (double)p->H);
+  p->prefetch = 0;
 }
 
 void pack_pointwise(const trident_args* a, const Sig& s, PointwiseParams* p) {
@@ -548,6 +550,7 @@ void pack_pointwise(const trident_args* a, const Sig& s, PointwiseParams* p) {
   p->m_rs = op == TRIDENT_OP_MASKED_FILL ? row_stride(t[1], K_MASK_H) : 0;
   p->y_rs = row_stride(t[yi], K_ACT_H);
   p->scalar = (float)a->scalar;
+  p->prefetch = 0;
 }
 
 void pack_rope(const trident_args* a, int base, int gq, const Version& v, uint32_t* err,
@@ -569,6 +572,7 @@ void pack_rope(const trident_args* a, int base, int gq, const Version& v, uint32
   p->NH = p->Hq + 2 * p->Hkv;
   p->eps = (float)a->eps;
   p->inv_D = (float)(1.0 / (double)p->D);
+  p->prefetch = 0;
 }
 
 void pack_swiglu(const trident_args* a, int g, int u, int o, int64_t T, SwigluParams* p) {
@@ -578,6 +582,7 @@ void pack_swiglu(const trident_args* a, int g, int u, int o, int64_t T, SwigluPa
   p->I = t[g].shape[t[g].ndim - 1];
   p->g_rs = row_stride(t[g], K_ACT_I); p->u_rs = row_stride(t[u], K_ACT_I);
   p->o_rs = row_stride(t[o], K_ACT_I);
+  p->prefetch = 0;
 }
 
 // Launches fn with the SCM's context current on this thread.
@@ -719,14 +724,25 @@ int32_t do_launch(trident_scm* scm, const Version& v, const trident_args* a, con
       st = set_chain_split(&c, s.T, split, &blocks);
       if (st != TRIDENT_OK) return st;
       cfg.gridDimX = (unsigned)blocks;
-      // prefetch before the PDL wait only when the grid is at most one block per SM and
-      // the launch overlaps a previous kernel (measured: ~10% faster at 1-4 tokens, slower
-      // once the grid fills the GPU)
-      c.prefetch = (scm->opt.flags & TRIDENT_OPT_PDL) && blocks <= v.sm_count ? 1 : 0;
       break;
     }
     default:
       return fail(TRIDENT_ERR_INVALID, "op");
+  }
+  // L2 prefetch before the PDL wait (prefetch_l2 in device_common.cuh): only for grids of
+  // at most one block per SM launched with programmatic serialisation (measured: ~10%
+  // faster layer steps at 1-4 tokens; slower once the grid fills the GPU)
+  const int32_t pf = (scm->opt.flags & TRIDENT_OPT_PDL) &&
+                     (int64_t)cfg.gridDimX * cfg.gridDimY <= scm->sm_count ? 1 : 0;
+  switch (op) {
+    case TRIDENT_OP_ADD_RMSNORM: P.an.prefetch = pf; break;
+    case TRIDENT_OP_RMSNORM: P.rn.prefetch = pf; break;
+    case TRIDENT_OP_ROPE_KV:
+    case TRIDENT_OP_QKNORM_ROPE_KV: P.rp.prefetch = pf; break;
+    case TRIDENT_OP_SWIGLU: P.sw.prefetch = pf; break;
+    case TRIDENT_OP_LAYER_CHAIN:
+    case TRIDENT_OP_LAYER_CHAIN_QKNORM: P.ch.prefetch = pf; break;
+    default: P.pw.prefetch = pf; break;
   }
   CUfunction fn = v.fn;
   if ((op == TRIDENT_OP_LAYER_CHAIN || op == TRIDENT_OP_LAYER_CHAIN_QKNORM) && P.ch.a_split == 1)
@@ -1022,6 +1038,8 @@ TRIDENT_API int32_t trident_scm_create(const trident_scm_options* opt, trident_c
       if (cudaFree(nullptr) != cudaSuccess) return fail(TRIDENT_ERR_CUDA, "CUDA init failed");
       if (g_drv.ctx_get(&s->ctx) != CUDA_SUCCESS || !s->ctx)
         return fail(TRIDENT_ERR_CUDA, "no current CUDA context");
+      if (cudaDeviceGetAttribute(&s->sm_count, cudaDevAttrMultiProcessorCount, s->device) != cudaSuccess)
+        return fail(TRIDENT_ERR_CUDA, "cannot read the SM count");
       if (cudaMalloc(&s->d_err, sizeof(uint32_t)) != cudaSuccess)
         return fail(TRIDENT_ERR_CUDA, "cudaMalloc of the status word failed");
       if (cudaMemset(s->d_err, 0, sizeof(uint32_t)) != cudaSuccess)
@@ -1076,7 +1094,6 @@ int32_t append_version(trident_scm_t* scm, const trident_spec_desc* desc, int32_
           return fail(TRIDENT_ERR_CUDA, "occupancy query failed");
         v.wave_blocks = per_sm * sms;
         v.step_wave_blocks = step_per_sm * sms;
-        v.sm_count = sms;
       }
       if (v.rope) {
         const bool chain = desc->op == TRIDENT_OP_LAYER_CHAIN || desc->op == TRIDENT_OP_LAYER_CHAIN_QKNORM;

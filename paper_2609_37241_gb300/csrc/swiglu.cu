@@ -13,8 +13,10 @@ constexpr int kSwigluUnroll = 2;
 
 template <int DT, int UNROLL>
 __global__ void __launch_bounds__(kThreads) swiglu_vec_kernel(const SwigluParams p) {
-  pdl_prologue();
+  pdl_trigger();
   const int64_t v0 = (int64_t)blockIdx.x * UNROLL * kThreads;
+  if (p.prefetch) swiglu_prefetch<DT, UNROLL>(p, blockIdx.y, v0, threadIdx.x);
+  pdl_wait();
   for (int64_t row = blockIdx.y; row < p.T; row += gridDim.y)
     swiglu_tile<DT, UNROLL>(p, row, v0, threadIdx.x);
 }
