@@ -19,13 +19,13 @@ namespace trident {
 
 constexpr int kChainSwigluUnroll = 2;
 
-// Block b of one call's grid (b < nA + nB + nC).
-template <int DT, int VPT, int SPLIT, int D, bool QKNORM>
-__device__ __forceinline__ void chain_block(const ChainParams& c, const int b) {
+// Norm role: part `part` (< SPLIT) of token `row`'s two add+RMSNorm steps.
+template <int DT, int VPT, int SPLIT>
+__device__ __forceinline__ void chain_norm(const ChainParams& c, const int64_t row, const int part) {
   constexpr int EB = Act<DT>::BYTES;
   constexpr int VE = Act<DT>::VE;
   const int tid = threadIdx.x;
-  if (b < c.nA) {
+  {
     // Both norms of one token. The second residual sum s2 = attn_out + round(s1) is
     // elementwise, so both sums of squares are formed before any reduction and reduced
     // together: one barrier. With a_split = 2 two CTAs share a token: each reads the whole
@@ -35,8 +35,6 @@ __device__ __forceinline__ void chain_block(const ChainParams& c, const int b) {
     __shared__ float2 red[kThreads / 32];
     constexpr int PP = VPT / SPLIT;  // vectors per thread this CTA writes
     static_assert(VPT % SPLIT == 0, "split");
-    const int64_t row = b / SPLIT;
-    const int part = b - (int)row * SPLIT;
     const AddNormParams& n1 = c.n1;
     const AddNormParams& n2 = c.n2;
     uint4 hv[VPT], rv[VPT], av[VPT];
@@ -128,43 +126,85 @@ __device__ __forceinline__ void chain_block(const ChainParams& c, const int b) {
       st16(x1p + vi, pack<DT>(y1));
       st16(x2p + vi, pack<DT>(y2));
     }
+  }
+}
+
+// RoPE role: RoPE block rb (< nB), i.e. head-rows [rb * UPB, (rb + 1) * UPB).
+template <int DT, int D, bool QKNORM>
+__device__ __forceinline__ void chain_rope(const ChainParams& c, const int64_t rb) {
+  constexpr int LPH = D / Act<DT>::VE;
+  const int64_t unit = rb * (kThreads / LPH) + threadIdx.x / LPH;
+  if (unit < c.rope.T * c.rope.NH) rope_head_row<DT, D, QKNORM>(c.rope, unit, threadIdx.x % LPH);
+}
+
+// SwiGLU role: column tile `col_tile` of row `row`.
+template <int DT>
+__device__ __forceinline__ void chain_swiglu(const ChainParams& c, const int64_t row, const int64_t col_tile) {
+  swiglu_tile<DT, kChainSwigluUnroll>(c.sw, row, col_tile * kChainSwigluUnroll * kThreads, threadIdx.x);
+}
+
+// Block b of one call's role-major grid (b < nA + nB + nC): [norms | RoPE | SwiGLU].
+template <int DT, int VPT, int SPLIT, int D, bool QKNORM>
+__device__ __forceinline__ void chain_block(const ChainParams& c, const int b) {
+  if (b < c.nA) {
+    const int64_t row = b / SPLIT;
+    chain_norm<DT, VPT, SPLIT>(c, row, b - (int)row * SPLIT);
   } else if (b < c.nA + c.nB) {
-    constexpr int LPH = D / VE;
-    constexpr int UPB = kThreads / LPH;
-    const int64_t unit = (int64_t)(b - c.nA) * UPB + tid / LPH;
-    if (unit < c.rope.T * c.rope.NH) rope_head_row<DT, D, QKNORM>(c.rope, unit, tid % LPH);
+    chain_rope<DT, D, QKNORM>(c, b - c.nA);
   } else {
     const int64_t tile = b - c.nA - c.nB;
     if (tile >= c.sw_tiles) return;
     const int64_t row = tile / c.sw_tiles_per_row;
-    const int64_t col_tile = tile - row * c.sw_tiles_per_row;
-    swiglu_tile<DT, kChainSwigluUnroll>(c.sw, row, col_tile * kChainSwigluUnroll * kThreads, tid);
+    chain_swiglu<DT>(c, row, tile - row * c.sw_tiles_per_row);
   }
 }
 
-// L2 prefetch of the lines block b reads first -- the norm rows, the RoPE head-rows and
+// Token-major grid (SPLIT + rope_per_tok + sw_tiles_per_row, T): block (q, t) is token t's
+// q-th block -- its norm parts, then its RoPE blocks, then its SwiGLU tiles. Blocks are
+// dispatched x first, so consecutive blocks belong to one token and any few of them carry a
+// mix of roles: under programmatic launch the blocks of a grid land on SMs as the previous
+// kernel's blocks retire, several consecutive blocks on one SM, and a role-major order can
+// give one SM four norm blocks (160 KB) while another gets 24 KB. Both indices come from
+// special registers, so no remapped index stays live in a register through the body.
+template <int DT, int VPT, int SPLIT, int D, bool QKNORM>
+__device__ __forceinline__ void chain_block_tok(const ChainParams& c) {
+  const int q = blockIdx.x;
+  if (q < SPLIT) {
+    chain_norm<DT, VPT, SPLIT>(c, blockIdx.y, q);
+  } else if (q < SPLIT + c.rope_per_tok) {
+    chain_rope<DT, D, QKNORM>(c, (int64_t)blockIdx.y * c.rope_per_tok + (q - SPLIT));
+  } else {
+    chain_swiglu<DT>(c, blockIdx.y, q - SPLIT - c.rope_per_tok);
+  }
+}
+
+// L2 prefetch of the lines a block reads first -- the norm rows, the RoPE head-rows and
 // positions, the SwiGLU tile -- one prefetch per 128-byte line, between the launch trigger
 // and the PDL wait (see prefetch_l2).
+template <int DT, int VPT>
+__device__ __forceinline__ void norm_prefetch(const ChainParams& c, const int64_t row) {
+  constexpr int EB = Act<DT>::BYTES;
+  const int tid = threadIdx.x;
+  if ((tid & 7) != 0) return;  // 8 threads x 16 bytes = one line
+  const uint4* hp = reinterpret_cast<const uint4*>(row_ptr(c.n1.x, row, c.n1.x_rs, EB));
+  const uint4* rp = reinterpret_cast<const uint4*>(row_ptr(c.n1.r, row, c.n1.r_rs, EB));
+  const uint4* ap = reinterpret_cast<const uint4*>(row_ptr(c.n2.x, row, c.n2.x_rs, EB));
+#pragma unroll
+  for (int v = 0; v < VPT; ++v) {
+    const int64_t vi = (int64_t)v * kThreads + tid;
+    prefetch_l2(hp + vi);
+    prefetch_l2(rp + vi);
+    prefetch_l2(ap + vi);
+  }
+}
+
 template <int DT, int VPT, int SPLIT, int D>
 __device__ __forceinline__ void chain_prefetch(const ChainParams& c, const int b) {
-  constexpr int EB = Act<DT>::BYTES;
-  constexpr int VE = Act<DT>::VE;
+  constexpr int LPH = D / Act<DT>::VE;
   const int tid = threadIdx.x;
   if (b < c.nA) {
-    if ((tid & 7) != 0) return;  // 8 threads x 16 bytes = one line
-    const int64_t row = b / SPLIT;
-    const uint4* hp = reinterpret_cast<const uint4*>(row_ptr(c.n1.x, row, c.n1.x_rs, EB));
-    const uint4* rp = reinterpret_cast<const uint4*>(row_ptr(c.n1.r, row, c.n1.r_rs, EB));
-    const uint4* ap = reinterpret_cast<const uint4*>(row_ptr(c.n2.x, row, c.n2.x_rs, EB));
-#pragma unroll
-    for (int v = 0; v < VPT; ++v) {
-      const int64_t vi = (int64_t)v * kThreads + tid;
-      prefetch_l2(hp + vi);
-      prefetch_l2(rp + vi);
-      prefetch_l2(ap + vi);
-    }
+    norm_prefetch<DT, VPT>(c, b / SPLIT);
   } else if (b < c.nA + c.nB) {
-    constexpr int LPH = D / VE;
     rope_prefetch<DT, D>(c.rope, (int64_t)(b - c.nA) * (kThreads / LPH) + tid / LPH, tid % LPH);
   } else {
     const int64_t tile = b - c.nA - c.nB;
@@ -175,15 +215,36 @@ __device__ __forceinline__ void chain_prefetch(const ChainParams& c, const int b
   }
 }
 
+template <int DT, int VPT, int SPLIT, int D>
+__device__ __forceinline__ void chain_prefetch_tok(const ChainParams& c) {
+  constexpr int LPH = D / Act<DT>::VE;
+  const int tid = threadIdx.x, q = blockIdx.x;
+  if (q < SPLIT) {
+    norm_prefetch<DT, VPT>(c, blockIdx.y);
+  } else if (q < SPLIT + c.rope_per_tok) {
+    const int64_t rb = (int64_t)blockIdx.y * c.rope_per_tok + (q - SPLIT);
+    rope_prefetch<DT, D>(c.rope, rb * (kThreads / LPH) + tid / LPH, tid % LPH);
+  } else {
+    swiglu_prefetch<DT, kChainSwigluUnroll>(
+        c.sw, blockIdx.y, (int64_t)(q - SPLIT - c.rope_per_tok) * kChainSwigluUnroll * kThreads, tid);
+  }
+}
+
 // Four resident blocks per SM for H 4096 (64 registers): the 64-token grid (576 blocks)
 // then fits one wave on 152 SMs; a fifth register would drop it to three blocks per SM.
 template <int DT, int VPT, int SPLIT, int D, bool QKNORM>
 __global__ void __launch_bounds__(kThreads, VPT == 2 ? 4 : 2)
     chain_kernel(const __grid_constant__ ChainParams c) {
   pdl_trigger();
-  if (c.prefetch) chain_prefetch<DT, VPT, SPLIT, D>(c, blockIdx.x);
-  pdl_wait();
-  chain_block<DT, VPT, SPLIT, D, QKNORM>(c, blockIdx.x);
+  if (c.tok_grid) {
+    if (c.prefetch) chain_prefetch_tok<DT, VPT, SPLIT, D>(c);
+    pdl_wait();
+    chain_block_tok<DT, VPT, SPLIT, D, QKNORM>(c);
+  } else {
+    if (c.prefetch) chain_prefetch<DT, VPT, SPLIT, D>(c, blockIdx.x);
+    pdl_wait();
+    chain_block<DT, VPT, SPLIT, D, QKNORM>(c, blockIdx.x);
+  }
 }
 
 // Several independent calls in one launch: a block finds its call by binary search over

@@ -636,6 +636,8 @@ int32_t pack_chain(trident_scm* scm, const Version& v, const trident_args* a, co
   c->sw_tiles_per_row = (int32_t)tiles;
   c->sw_tiles = nC;
   c->prefetch = 0;
+  c->tok_grid = 0;
+  c->rope_per_tok = 0;
   return TRIDENT_OK;
 }
 
@@ -724,6 +726,18 @@ int32_t do_launch(trident_scm* scm, const Version& v, const trident_args* a, con
       st = set_chain_split(&c, s.T, split, &blocks);
       if (st != TRIDENT_OK) return st;
       cfg.gridDimX = (unsigned)blocks;
+      // Token-major grid (chain_block_tok) for grids of at most one block per SM, when every
+      // token has the same number of RoPE blocks: consecutive blocks then mix roles (measured:
+      // 16 tokens 3.55 -> 2.85 us per layer step, 1 token 2.20 -> 2.04 us). A grid that fills
+      // the GPU keeps the role-major order, which starts the longest (norm) blocks first
+      // (64 tokens: 3.98 us role-major, 4.05 us token-major).
+      const int64_t upb = rope_units_per_block(c.rope.D, 2);
+      if (c.rope.NH % upb == 0 && s.T >= 1 && s.T <= 65535 && blocks <= scm->sm_count) {
+        c.tok_grid = 1;
+        c.rope_per_tok = (int32_t)(c.rope.NH / upb);
+        cfg.gridDimX = (unsigned)(split + c.rope_per_tok + c.sw_tiles_per_row);
+        cfg.gridDimY = (unsigned)s.T;
+      }
       break;
     }
     default:
