@@ -776,15 +776,25 @@ bool step_bytes_ok(const trident_args* a, int32_t m, bool check_own) {
     int32_t call, slot;
     bool out;
   };
-  thread_local std::vector<Ext> ext;
-  ext.clear();
-  for (int32_t c = 0; c < m; ++c) {
-    const OpInfo& oi = g_ops[a[c].op];
-    for (int i = 0; i < oi.nslots; ++i) {
+  constexpr int kMaxExt = kStepMax * TRIDENT_MAX_TENSORS;  // on the stack: no allocation
+  Ext ext[kMaxExt];
+  uint64_t keys[kMaxExt], keys2[kMaxExt];
+  uint32_t order[kMaxExt];
+  size_t n = 0;
+  int64_t lo = INT64_MAX, hi = INT64_MIN;
+  // Slot-major: one slot of every call, then the next slot. When each slot's tensors sit in
+  // one arena in call order (a serving engine's per-layer buffers, or views into one
+  // buffer), every slot then contributes an ascending run of starts.
+  int32_t nslots = 0;
+  for (int32_t c = 0; c < m; ++c) nslots = g_ops[a[c].op].nslots > nslots ? g_ops[a[c].op].nslots : nslots;
+  for (int i = 0; i < nslots; ++i) {
+    for (int32_t c = 0; c < m; ++c) {
+      const OpInfo& oi = g_ops[a[c].op];
+      if (i >= oi.nslots) continue;
       const trident_tensor& t = a[c].t[i];
       const Rows r = rows_of(t, oi.kind[i]);
       const int es = elem_size(t.dtype);
-      Ext e;
+      Ext& e = ext[n];
       e.base = (int64_t)reinterpret_cast<uintptr_t>(t.data);
       e.nr = r.n;
       e.w = r.width * es;
@@ -794,15 +804,55 @@ bool step_bytes_ok(const trident_args* a, int32_t m, bool check_own) {
       e.call = c;
       e.slot = i;
       e.out = oi.out[i];
-      ext.push_back(e);
+      lo = e.base < lo ? e.base : lo;
+      hi = e.base > hi ? e.base : hi;
+      ++n;
     }
   }
-  std::sort(ext.begin(), ext.end(), [](const Ext& x, const Ext& y) { return x.base < y.base; });
-  const size_t n = ext.size();
+  // Sort by start. One 64-bit key per extent -- the start relative to the lowest one,
+  // shifted past an 11-bit extent index. With few ascending runs (see above) a natural
+  // merge sort merges them pairwise in a few linear passes (on the Grace host: 0.3 us for
+  // sorted input, 3.0 us for 20 interleaved runs, against 2.9 and 3.6 us for std::sort);
+  // otherwise std::sort (random layouts: 3.6 us against 6.9). Spans beyond 2^53 bytes fall
+  // back to sorting indices by start.
+  if (n > 0 && (uint64_t)(hi - lo) < (1ull << 53)) {
+    uint64_t* src = keys;
+    uint64_t* dst = keys2;
+    size_t runs = 1;
+    for (size_t i = 0; i < n; ++i) {
+      src[i] = ((uint64_t)(ext[i].base - lo) << 11) | (uint64_t)i;
+      runs += i > 0 && src[i] < src[i - 1];
+    }
+    if (runs > 24) {  // little run structure to use: an ordinary sort
+      std::sort(src, src + n);
+      runs = 1;
+    }
+    while (runs > 1) {  // one pass merges each pair of consecutive ascending runs of src into dst
+      size_t merged = 0, i = 0;
+      while (i < n) {
+        size_t j = i + 1;
+        while (j < n && src[j - 1] < src[j]) ++j;  // first run [i, j)
+        size_t k = j;
+        if (j < n) {
+          k = j + 1;
+          while (k < n && src[k - 1] < src[k]) ++k;  // second run [j, k)
+        }
+        std::merge(src + i, src + j, src + j, src + k, dst + i);
+        ++merged;
+        i = k;
+      }
+      std::swap(src, dst);
+      if (merged == 1) break;  // the whole array was at most two runs: now sorted
+    }
+    for (size_t i = 0; i < n; ++i) order[i] = (uint32_t)(src[i] & 2047u);
+  } else {
+    for (size_t i = 0; i < n; ++i) order[i] = (uint32_t)i;
+    std::sort(order, order + n, [&](uint32_t x, uint32_t y) { return ext[x].base < ext[y].base; });
+  }
   for (size_t x = 0; x < n; ++x) {
-    const Ext& p = ext[x];
-    for (size_t y = x + 1; y < n && ext[y].base < p.end; ++y) {
-      const Ext& q = ext[y];
+    const Ext& p = ext[order[x]];
+    for (size_t y = x + 1; y < n && ext[order[y]].base < p.end; ++y) {
+      const Ext& q = ext[order[y]];
       if (!p.out && !q.out) continue;  // inputs may share bytes
       if (q.call == p.call && !check_own) continue;
       if (!rows_overlap(p.base, p.nr, p.w, p.rs, q.base, q.nr, q.w, q.rs)) continue;
@@ -1303,6 +1353,7 @@ namespace {
 
 constexpr int32_t kNotFused = 100;  // step_chunk: run the chunk call by call
 static_assert(kStepMax == TRIDENT_STEP_MAX, "step chunk size");
+static_assert(kStepMax * TRIDENT_MAX_TENSORS <= 2048, "extent index fits the sort key");
 static_assert(sizeof(ChainStepParams) <= 32764, "kernel parameter limit");
 
 // One chunk of trident_scm_invoke_step: select every call; if all hit layer-chain
