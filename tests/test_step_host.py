@@ -180,3 +180,24 @@ def test_non_chain_ops_take_the_sequential_path(S):
         t["addr"] += 1 << 40
     st, sel, stats = run_step(S, [norm], [a, b])
     assert (st, sel, stats.fused_launches, stats.hits) == (S.OK, [0, 0], 0, 2)
+
+
+def test_scattered_layouts_take_the_sorting_path(S):
+    """30 calls whose tensors sit at addresses permuted independently per slot (more than
+    24 ascending runs, so the extents are sorted rather than merged): independent calls
+    fuse; one call reading another's output makes the step run call by call."""
+    rng = random.Random(7)
+    table = [chain_spec()]
+    n = 30
+    calls = [chain_call(0) for _ in range(n)]
+    for slot in range(18):
+        perm = list(range(n))
+        rng.shuffle(perm)
+        for k in range(n):
+            calls[k]["tensors"][slot]["addr"] += perm[k] << 40
+    assert len({(t["addr"]) for c in calls for t in c["tensors"]}) == n * 18
+    st, sel, stats = run_step(S, table, calls)
+    assert (st, stats.fused_launches, stats.fused_calls) == (S.OK, 1, n)
+    calls[17]["tensors"][1] = dict(calls[4]["tensors"][14])  # r0 of call 17 = r2 of call 4
+    st, sel, stats = run_step(S, table, calls)
+    assert (st, sel, stats.fused_launches, stats.hits) == (S.OK, [0] * n, 0, n)
