@@ -6,13 +6,16 @@
 // The only data dependency inside the chain is r1 feeding the second norm, and it is
 // row-local: the block that produces row t of r1 keeps it in registers and runs the
 // second norm of row t itself. So no grid-wide barrier is needed; the launch is a
-// horizontal fusion where block ranges take different roles:
-//   [0, nA)            two add+RMSNorm steps, one or two blocks per token (the longest
-//                      per-block work, so these blocks are scheduled first)
-//   [nA, nA + nB)      RoPE/KV head-rows, (256 / (D/8)) per block
-//   [nA + nB, end)     SwiGLU tiles of one row each
-// One launch replaces four, which is what matters at decode sizes, where each step
-// moves well under a microsecond of HBM traffic.
+// horizontal fusion where blocks take different roles:
+//   norm     two add+RMSNorm steps, one or two blocks per token (the longest per-block
+//            work)
+//   RoPE     RoPE/KV head-rows, (256 / (D/8)) per block
+//   SwiGLU   tiles of one row each
+// A grid that fills the GPU is role-major ([norms | RoPE | SwiGLU], so the longest blocks
+// start first); a grid of at most one block per SM is token-major (chain_block_tok), so
+// consecutive blocks mix roles. One launch replaces four, which is what matters at decode
+// sizes, where each step moves well under a microsecond of HBM traffic. chain_step_kernel
+// runs several independent calls' grids in one launch.
 #include "device_common.cuh"
 
 namespace trident {

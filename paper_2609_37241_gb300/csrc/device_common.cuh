@@ -5,7 +5,8 @@
 // warp-shuffle reductions. Each kernel starts with the programmatic-dependent-launch
 // pair (trigger, then wait) so that, when launched with programmatic stream
 // serialisation, the next kernel's launch overlaps this one while every global memory
-// access still waits for the previous kernel to finish.
+// access still waits for the previous kernel to finish; between the two, small grids
+// prefetch their first lines into L2 (prefetch_l2).
 #pragma once
 #include <cuda_bf16.h>
 #include <cuda_fp16.h>
