@@ -140,16 +140,17 @@ def test_step_fp16_longer_than_one_chunk(S):
         check_chain(L.layer_chain(inp, cfg["theta"], cfg["eps"], FP16), out, inp, FP16)
 
 
-@pytest.mark.parametrize("entry", ["invoke", "step"])
-def test_dependent_layers_back_to_back_with_pdl(S, entry):
-    """Six Llama layers at 64 tokens where layer l+1's residual input is layer l's second
-    residual output, launched back to back with programmatic dependent launch (one invoke
-    each through the fast-call shim, or one invoke_step that must fall back to call-by-call
+@pytest.mark.parametrize("entry,T", [("invoke", 64), ("step", 64), ("invoke", 4), ("step", 4)])
+def test_dependent_layers_back_to_back_with_pdl(S, entry, T):
+    """Six Llama layers where layer l+1's residual input is layer l's second residual
+    output, launched back to back with programmatic dependent launch (one invoke each
+    through the fast-call shim, or one invoke_step that must fall back to call-by-call
     order). Each kernel's memory accesses wait for the previous kernel, so every layer equals
-    the oracle run in sequence."""
+    the oracle run in sequence. At 4 tokens the grid is small: it is token-major and
+    prefetches its rows into L2 before the wait, while the previous layer still writes them."""
     import ctypes
     cfg = synth.LLAMA
-    T, n = 64, 6
+    n = 6
     s, op = step_scm(S, cfg, BF16, S.LAYOUT_ROWSTRIDED)
     inps, outs, args = build_layers(S, cfg, T, n, seed=606)
     for l in range(1, n):
