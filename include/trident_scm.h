@@ -156,6 +156,8 @@ typedef enum trident_variant {
 
 /* Bits of the device status word. */
 #define TRIDENT_DEVERR_POS 0x1u   /* a RoPE/KV position was outside [0, S) */
+#define TRIDENT_DEVERR_TIMEOUT 0x2u /* a kernel's bounded wait for its own bulk copies ran
+                                       out; that block's outputs were not written */
 
 /* Option flags of trident_scm_create. */
 #define TRIDENT_OPT_DRY_RUN 0x1        /* no CUDA at all: invoke selects and calls the hook,

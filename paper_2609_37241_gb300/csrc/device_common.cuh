@@ -17,6 +17,7 @@
 namespace trident {
 
 constexpr uint32_t kErrPos = 0x1u;  // TRIDENT_DEVERR_POS
+constexpr uint32_t kErrTimeout = 0x2u;  // TRIDENT_DEVERR_TIMEOUT
 
 __device__ __forceinline__ void pdl_trigger() {
   asm volatile("griddepcontrol.launch_dependents;" ::: "memory");

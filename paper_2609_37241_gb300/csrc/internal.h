@@ -25,6 +25,7 @@ struct AddNormParams {
   int64_t x_rs, r_rs, y_rs, ro_rs;
   float eps, inv_H;
   int32_t prefetch;  // 1: prefetch this block's first lines into L2 before the PDL wait
+  uint32_t* err;     // device status word (the bulk-copy kernel reports a timed-out wait)
 };
 
 // RMSNorm over T rows of H elements (no residual). Row strides in elements.
@@ -115,6 +116,8 @@ struct KernelEntry {
   const void* fn_inplace = nullptr;  // chain only: the entry for calls that write in place
   const void* fn_step = nullptr;          // chain only: several calls per launch (ChainStepParams)
   const void* fn_step_inplace = nullptr;  // ... one block per token for the norms
+  const void* fn_large = nullptr;  // add+RMSNorm: the entry for calls of >= large_rows rows
+  int32_t large_rows = 0;
   int32_t kind = 0;      // which grid rule the host applies (KernelKind)
   int32_t vec = 0;       // elements per vector (VE), or tile width for SwiGLU
   int32_t unroll = 1;    // vectors per thread per tile (SwiGLU, chain)

@@ -376,6 +376,7 @@ struct Version {
   CUfunction fn;
   CUfunction fn_inplace;  // layer chain: one block per token when outputs alias inputs
   int32_t wave_blocks;    // layer chain: blocks of `fn` resident at once on the whole GPU
+  CUfunction fn_large;          // add+RMSNorm: entry for calls of >= ke.large_rows rows
   CUfunction step_fn;           // layer chain: several calls per launch (two blocks per token)
   CUfunction step_fn_inplace;   // ... one block per token
   int32_t step_wave_blocks;     // blocks of `step_fn` resident at once
@@ -522,6 +523,7 @@ void pack_addnorm(const trident_args* a, int x, int r, int g, int y, int ro, con
   p->eps = (float)a->eps;
   p->inv_H = (float)(1.0 / (double)p->H);
   p->prefetch = 0;
+  p->err = nullptr;
 }
 
 void pack_rmsnorm(const trident_args* a, const Sig& s, RmsNormParams* p) {
@@ -676,6 +678,7 @@ int32_t do_launch(trident_scm* scm, const Version& v, const trident_args* a, con
   switch (op) {
     case TRIDENT_OP_ADD_RMSNORM:
       pack_addnorm(a, 0, 1, 2, 3, 4, s, K_ACT_H, &P.an);
+      P.an.err = scm->d_err;
       cfg.gridDimX = cap_grid(s.T);
       break;
     case TRIDENT_OP_RMSNORM:
@@ -761,6 +764,7 @@ int32_t do_launch(trident_scm* scm, const Version& v, const trident_args* a, con
   CUfunction fn = v.fn;
   if ((op == TRIDENT_OP_LAYER_CHAIN || op == TRIDENT_OP_LAYER_CHAIN_QKNORM) && P.ch.a_split == 1)
     fn = v.fn_inplace;
+  if (v.fn_large && s.T >= v.ke.large_rows) fn = v.fn_large;  // many rows: the bulk-copy kernel
   return launch_on(scm, &cfg, fn, kp);
 }
 
@@ -1140,6 +1144,12 @@ int32_t append_version(trident_scm_t* scm, const trident_spec_desc* desc, int32_
       if (cudaGetFuncBySymbol(&f, v.ke.fn) != cudaSuccess || !f)
         return fail(TRIDENT_ERR_CUDA, "cannot resolve the kernel entry");
       v.fn = reinterpret_cast<CUfunction>(f);
+      if (v.ke.fn_large) {
+        cudaFunction_t h = nullptr;
+        if (cudaGetFuncBySymbol(&h, v.ke.fn_large) != cudaSuccess || !h)
+          return fail(TRIDENT_ERR_CUDA, "cannot resolve the large-call kernel entry");
+        v.fn_large = reinterpret_cast<CUfunction>(h);
+      }
       if (v.ke.fn_inplace) {
         cudaFunction_t g = nullptr;
         if (cudaGetFuncBySymbol(&g, v.ke.fn_inplace) != cudaSuccess || !g)

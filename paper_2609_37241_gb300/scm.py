@@ -22,7 +22,7 @@ OP_SILU, OP_ADD, OP_NEG, OP_MASKED_FILL = 8, 9, 10, 11
 LAYOUT_CONTIG, LAYOUT_ROWSTRIDED, LAYOUT_ANY = 0, 1, 2
 VARIANT_AUTO, VARIANT_GENERIC, VARIANT_VECTOR = 0, 1, 2
 OPT_DRY_RUN, OPT_NO_ALIAS_CHECK, OPT_PDL, OPT_TIMING, OPT_FAIL_LAUNCHES = 0x1, 0x2, 0x4, 0x8, 0x10
-DEVERR_POS = 0x1
+DEVERR_POS, DEVERR_TIMEOUT = 0x1, 0x2
 MAX_TENSORS, MAX_FIXED = 20, 8
 STEP_MAX = 48  # calls per launch of trident_scm_invoke_step
 TREE_MAX_NODES, TREE_MAX_DEPTH = 4096, 16

@@ -53,7 +53,7 @@ def test_fuzz_add_rmsnorm_and_rmsnorm(S, seed):
     g = np.random.default_rng(seed)
     dtype = rng.choice([BF16, BF16, FP16, FP32])
     H = rng.choice([64, 128, 256, 1000, 2048, 4096, 8192] + ([520] if dtype != FP32 else []))
-    T = rng.choice([1, 2, 7, 37, 150, 153, 300])
+    T = rng.choice([1, 2, 7, 37, 150, 153, 300, 1024, 1100])
     es = ES[dtype]
     vec_ok = (H * es) % 16 == 0
     pad = rng.choice([0, 0, 8 * (16 // es)]) if vec_ok else 0
@@ -83,6 +83,28 @@ def test_fuzz_add_rmsnorm_and_rmsnorm(S, seed):
     run_one(S, desc, S.OP_RMSNORM, [xd, gd, yd], pdl, eps=eps)
     y_ref, y_bits = L.rmsnorm(x, gam, eps, dtype)
     P.check_act(P.host_bits(yd, dtype), y_ref, y_bits, dtype, f"rmsnorm {dtype} {H} {T}")
+
+
+@pytest.mark.parametrize("seed", range(6))
+def test_fuzz_add_rmsnorm_bulk_rows(S, seed):
+    """H 8192 with at least 1024 rows: the kernel that stages rows by bulk copies."""
+    rng = random.Random(50 + seed)
+    g = np.random.default_rng(50 + seed)
+    dtype = rng.choice([BF16, FP16])
+    T = rng.choice([1024, 1100, 2048])
+    H = 8192
+    pad = rng.choice([0, 64])
+    pdl = rng.random() < 0.5
+    inplace = rng.random() < 0.4
+    x, r = synth.act(g, (T, H), dtype), synth.act(g, (T, H), dtype)
+    gam = synth.gamma(g, H)
+    xd, rd = rows(x, dtype, pad), rows(r, dtype, pad)
+    yd, rod = (xd, rd) if inplace else (rows(np.zeros_like(x), dtype, pad), rows(np.zeros_like(r), dtype, pad))
+    desc = S.make_spec(S.OP_ADD_RMSNORM, dtype, [H], 1, 1 << 20, layout=layout_of(S, T, pad))
+    run_one(S, desc, S.OP_ADD_RMSNORM, [xd, rd, torch.from_numpy(gam).cuda(), yd, rod], pdl, eps=1e-6)
+    y_ref, y_bits, ro_bits = L.add_rmsnorm(x, r, gam, 1e-6, dtype)
+    assert np.array_equal(P.host_bits(rod, dtype), ro_bits)
+    P.check_act(P.host_bits(yd, dtype), y_ref, y_bits, dtype, f"add_rmsnorm bulk {dtype} {T}")
 
 
 @pytest.mark.parametrize("seed", range(12))
