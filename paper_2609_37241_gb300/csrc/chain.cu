@@ -255,7 +255,7 @@ __global__ void __launch_bounds__(kThreads, VPT == 2 ? 4 : 2)
 template <int DT, int VPT, int SPLIT, int D, bool QKNORM>
 __global__ void __launch_bounds__(kThreads, VPT == 2 ? 4 : 2)
     chain_step_kernel(const __grid_constant__ ChainStepParams p) {
-  pdl_prologue();
+  pdl_trigger();
   const int b = blockIdx.x;
   int lo = 0, hi = p.n - 1;
   while (lo < hi) {
@@ -263,6 +263,8 @@ __global__ void __launch_bounds__(kThreads, VPT == 2 ? 4 : 2)
     if (b >= p.first[mid]) lo = mid;
     else hi = mid - 1;
   }
+  if (p.c[lo].prefetch) chain_prefetch<DT, VPT, SPLIT, D>(p.c[lo], b - p.first[lo]);
+  pdl_wait();
   chain_block<DT, VPT, SPLIT, D, QKNORM>(p.c[lo], b - p.first[lo]);
 }
 

@@ -1411,6 +1411,9 @@ int32_t step_chunk(trident_scm* scm, const trident_args* a, int32_t m, void* str
     }
     P.first[m] = (int32_t)first;
     P.n = m;
+    // L2 prefetch before the PDL wait under the same rule as single calls (do_launch)
+    const int32_t pf = (scm->opt.flags & TRIDENT_OPT_PDL) && first <= scm->sm_count ? 1 : 0;
+    for (int32_t i = 0; i < m; ++i) P.c[i].prefetch = pf;
     CUlaunchConfig cfg;
     CUlaunchAttribute attr;
     base_config(scm, stream, &cfg, &attr);
