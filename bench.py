@@ -269,11 +269,13 @@ class ChainSets:
                 S.make_args(S.OP_SWIGLU, [g, u, o])]
 
 
-def layer_scm(c, cfg, pdl=True, timing=False):
+def layer_scm(c, cfg, pdl=True, timing=False, replay=False):
     """One SCM holding the layer's versions: the fused chain (index 0), then the four
-    single-step versions, all for token buckets 1..4096 and row-strided q/k/v and g/u."""
+    single-step versions, all for token buckets 1..4096 and row-strided q/k/v and g/u.
+    invoke_step's replay cache is off unless `replay`: the rotating-set lines measure the
+    full path (selection, byte rules and packing on every step)."""
     S = c.S
-    flags = (S.OPT_PDL if pdl else 0) | (S.OPT_TIMING if timing else 0)
+    flags = (S.OPT_PDL if pdl else 0) | (S.OPT_TIMING if timing else 0) | (0 if replay else S.OPT_NO_STEP_REPLAY)
     s = S.Scm(device=c.dev.index or 0, flags=flags)
     qk = cfg.get("qknorm", False)
     fixed = [cfg[k] for k in ("H", "Hq", "Hkv", "D", "S", "I")]
@@ -368,6 +370,23 @@ def bench_layer(c, cfg, T, K, W, layers=1, min_bytes=2 * L2_BYTES):
         assert fused_n == (K + W) * per_step, ("step launches not fused", fused_n)
         c.launches += K * per_step
         step = dict(us=round(step_dev, 3), host_us=round(step_host, 3), launches_per_step=per_step)
+        # A decode loop with static buffers passes the same argument arrays every step:
+        # invoke_step relaunches them from its replay cache (no selection, byte rules or
+        # packing). As many rotating arrays as the cache keeps (4); working set reported.
+        rs = layer_scm(c, cfg, replay=True)
+        rstp = c.step_invoker(rs)
+        nrep = min(groups, 4)
+        for i in range(2 * nrep):  # seen, then stored
+            rstp(fa[i % nrep], layers)
+        before = rs.stats().step_replays
+        rep_dev, rep_host = time_steps(c, lambda i: rstp(fa[i % nrep], layers), K, W)
+        replayed = rs.stats().step_replays - before
+        assert replayed == (K + W) * layers, ("steps not replayed", replayed)
+        assert_all_hit(rs, "replayed step T=%d" % T)
+        rs.close()
+        c.launches += K * per_step
+        step["replayed"] = dict(us=round(rep_dev, 3), host_us=round(rep_host, 3), arrays=nrep,
+                                working_set_mb=round(nrep * layers * chain_bytes_per_token(cfg) * T / 2 ** 20, 1))
     # device throughput floor: the same launches issued from one native call
     nat = min(K, R if layers == 1 else R)
     if layers == 1:

@@ -34,7 +34,7 @@
 extern "C" {
 #endif
 
-#define TRIDENT_ABI_VERSION 3
+#define TRIDENT_ABI_VERSION 4
 #define TRIDENT_MAX_TENSORS 20
 #define TRIDENT_MAX_FIXED 8
 /* out_selected value for a sequence element that was not run (trident_scm_invoke_seq). */
@@ -167,6 +167,7 @@ typedef enum trident_variant {
 #define TRIDENT_OPT_TIMING 0x8         /* record host ns per hit (trident_scm_host_times) */
 #define TRIDENT_OPT_FAIL_LAUNCHES 0x10 /* fault injection on the host, for tests: every launch
                                           step of a hit reports ERR_CUDA without launching */
+#define TRIDENT_OPT_NO_STEP_REPLAY 0x20 /* invoke_step never replays a stored chunk */
 
 /* ---------------------------------------------------------------- structs */
 /* Caller-owned tensor descriptor (DLPack-like, §3.4: tensors cross the boundary as
@@ -312,6 +313,9 @@ typedef struct trident_scm_stats_t {
   int32_t reserved;
   uint64_t fused_launches;  /* invoke_step launches that ran several calls at once   */
   uint64_t fused_calls;     /* calls run by those launches                           */
+  uint64_t step_replays;    /* calls of fused chunks relaunched from the replay cache
+                               (counted in invokes, hits and fused_calls as well; no
+                               guard is evaluated for them)                          */
 } trident_scm_stats_t;
 
 typedef struct trident_scm trident_scm_t; /* opaque; owns the table, kernels and device state */
@@ -389,7 +393,18 @@ int32_t trident_scm_invoke_seq(trident_scm_t* scm, const trident_args* args, int
  * statistics; no host time is recorded for it. If its launch fails, the call returns
  * ERR_CUDA with the chunk's out_selected set to the versions it selected and the calls
  * after the chunk set to TRIDENT_NOT_RUN. Host cost of the independence test: one sort of
- * the chunk's tensor extents (about 20 per call). */
+ * the chunk's tensor extents (about 20 per call).
+ * Replay: a fused chunk's outcome depends on nothing but its argument bytes (selection reads
+ * them and a table that only grows, so a call's first match cannot change; the byte rules
+ * and the packed kernel parameters read only them and state fixed when the SCM and its
+ * versions were created). The SCM therefore keeps the last few fused chunks whose
+ * fingerprint it had seen before (4 entries, about 110 KB each, allocated on the first
+ * store); a chunk whose argument bytes equal a kept one is relaunched from the stored
+ * parameter block, with the same statuses, out_selected and statistics as the full path
+ * (plus step_replays; guard_evals does not grow). A decode loop that passes the same
+ * buffers every step takes this path from its third step on. Device data may change freely
+ * between steps: only the argument bytes are compared. TRIDENT_OPT_NO_STEP_REPLAY turns it
+ * off. Thread-safe: a thread that finds the cache in use by another takes the full path. */
 #define TRIDENT_STEP_MAX 48
 int32_t trident_scm_invoke_step(trident_scm_t* scm, const trident_args* args, int32_t n,
                                 void* stream, int32_t* out_selected);

@@ -384,6 +384,29 @@ struct Version {
   Recipe* recipe;               // structured-argument binding (register_tree_spec), or NULL
 };
 
+// Step replay cache of invoke_step. A fused chunk's outcome is a function of its argument
+// bytes alone: selection reads the arguments and a table that only grows (a call's first
+// match stays its first match), the byte rules read only the arguments, and the packed
+// parameter block reads the arguments, the selected versions and state fixed at creation.
+// So a chunk whose argument bytes equal a stored one relaunches the stored block. Entries
+// are stored only for chunks whose fingerprint was seen before (a decode loop passing the
+// same buffers step after step), so chunks that never repeat pay one fingerprint.
+constexpr int kMemoEntries = 4;
+constexpr int kSeenRing = 8;
+
+struct StepMemo {
+  uint64_t fp;     // fingerprint; 0 marks an empty entry
+  uint64_t used;   // clock of the last store or replay (least recently used is replaced)
+  int32_t m;       // calls
+  int32_t ndist;   // distinct selected versions
+  unsigned grid;
+  CUfunction fn;
+  int32_t sel[kStepMax];
+  int32_t dist_idx[kStepMax], dist_cnt[kStepMax];
+  trident_args args[kStepMax];
+  ChainStepParams P;
+};
+
 }  // namespace
 
 struct trident_scm {
@@ -410,6 +433,14 @@ struct trident_scm {
   uint32_t* ring = nullptr;
   int32_t ring_cap = 0;
   std::atomic<uint64_t> ring_n{0};
+  // step replay cache (invoke_step); memo, seen and memo_clock are used only while
+  // memo_lock is held (a thread that finds it held takes the full path)
+  StepMemo* memo = nullptr;  // kMemoEntries entries, allocated by the first store
+  uint64_t seen[kSeenRing] = {};
+  uint32_t seen_next = 0;
+  uint64_t memo_clock = 0;
+  std::atomic_flag memo_lock = ATOMIC_FLAG_INIT;
+  std::atomic<uint64_t> step_replays{0};
 };
 
 namespace {
@@ -1076,7 +1107,7 @@ TRIDENT_API int32_t trident_scm_create(const trident_scm_options* opt, trident_c
   if (o.timing_ring == 0) o.timing_ring = 65536;
   if (o.timing_ring < 1 || o.timing_ring > (1 << 24)) return fail(TRIDENT_ERR_INVALID, "timing_ring");
   if (o.flags & ~(TRIDENT_OPT_DRY_RUN | TRIDENT_OPT_NO_ALIAS_CHECK | TRIDENT_OPT_PDL | TRIDENT_OPT_TIMING |
-                  TRIDENT_OPT_FAIL_LAUNCHES))
+                  TRIDENT_OPT_FAIL_LAUNCHES | TRIDENT_OPT_NO_STEP_REPLAY))
     return fail(TRIDENT_ERR_INVALID, "unknown option flags");
   if (o.device < 0) return fail(TRIDENT_ERR_INVALID, "device");
   trident_scm* s = new (std::nothrow) trident_scm();
@@ -1366,11 +1397,114 @@ static_assert(kStepMax == TRIDENT_STEP_MAX, "step chunk size");
 static_assert(kStepMax * TRIDENT_MAX_TENSORS <= 2048, "extent index fits the sort key");
 static_assert(sizeof(ChainStepParams) <= 32764, "kernel parameter limit");
 
+// Fingerprint of a chunk for the replay cache: a few words from its first, middle and last
+// calls (collisions only cost a failed byte comparison or one unneeded store).
+uint64_t step_fingerprint(const trident_args* a, int32_t m) {
+  uint64_t h = 0x9e3779b97f4a7c15ull ^ (uint64_t)m;
+  auto mix = [&h](uint64_t v) {
+    h ^= v + 0x9e3779b97f4a7c15ull + (h << 6) + (h >> 2);
+    h *= 0xff51afd7ed558ccdull;
+  };
+  const int32_t pick[3] = {0, m / 2, m - 1};
+  for (int32_t k : pick) {
+    const trident_args& c = a[k];
+    mix((uint64_t)(uint32_t)c.op | ((uint64_t)(uint32_t)c.ntensors << 32));
+    mix((uint64_t)reinterpret_cast<uintptr_t>(c.t[0].data));
+    mix((uint64_t)reinterpret_cast<uintptr_t>(c.t[1].data));
+    mix((uint64_t)c.t[0].shape[0]);
+  }
+  return h | 1;  // never 0 (the empty-entry mark)
+}
+
+// Under memo_lock. Looks the chunk up; on a match relaunches it (or, in a dry run, only
+// counts it) and returns its status. Otherwise returns kNotFused and sets *repeat when
+// the fingerprint was seen before (the full path then stores the chunk).
+int32_t replay_chunk(trident_scm* scm, const trident_args* a, int32_t m, uint64_t fp, void* stream,
+                     int32_t* out_selected, bool* repeat) {
+  StepMemo* e = nullptr;
+  if (scm->memo)
+    for (int k = 0; k < kMemoEntries && !e; ++k) {
+      StepMemo& x = scm->memo[k];
+      if (x.fp == fp && x.m == m && std::memcmp(x.args, a, (size_t)m * sizeof(trident_args)) == 0) e = &x;
+    }
+  if (!e) {
+    for (int k = 0; k < kSeenRing; ++k)
+      if (scm->seen[k] == fp) *repeat = true;
+    if (!*repeat) scm->seen[scm->seen_next++ % kSeenRing] = fp;
+    return kNotFused;
+  }
+  e->used = ++scm->memo_clock;
+  scm->invokes.fetch_add((uint64_t)m, std::memory_order_relaxed);
+  if (out_selected)
+    for (int32_t i = 0; i < m; ++i) out_selected[i] = e->sel[i];
+  if (scm->opt.flags & TRIDENT_OPT_FAIL_LAUNCHES)
+    return count_error(scm, fail(TRIDENT_ERR_CUDA, "launch failure injected (TRIDENT_OPT_FAIL_LAUNCHES)"));
+  if (!scm->dry) {
+    CUlaunchConfig cfg;
+    CUlaunchAttribute attr;
+    base_config(scm, stream, &cfg, &attr);
+    cfg.gridDimX = e->grid;
+    void* kp[1] = {&e->P};
+    const int32_t st = launch_on(scm, &cfg, e->fn, kp);
+    if (st != TRIDENT_OK) return count_error(scm, st);
+  }
+  for (int32_t k = 0; k < e->ndist; ++k)
+    scm->hits_per[e->dist_idx[k]].fetch_add((uint64_t)e->dist_cnt[k], std::memory_order_relaxed);
+  scm->hits.fetch_add((uint64_t)m, std::memory_order_relaxed);
+  scm->fused_launches.fetch_add(1, std::memory_order_relaxed);
+  scm->fused_calls.fetch_add((uint64_t)m, std::memory_order_relaxed);
+  scm->step_replays.fetch_add((uint64_t)m, std::memory_order_relaxed);
+  return TRIDENT_OK;
+}
+
+// Under memo_lock: stores a fused chunk over the least recently used entry.
+void store_chunk(trident_scm* scm, const trident_args* a, int32_t m, uint64_t fp, const int32_t* sel,
+                 const ChainStepParams* P, unsigned grid, CUfunction fn) {
+  if (!scm->memo) {
+    scm->memo = static_cast<StepMemo*>(std::calloc(kMemoEntries, sizeof(StepMemo)));
+    if (!scm->memo) return;  // no cache: every chunk takes the full path
+  }
+  StepMemo* e = &scm->memo[0];
+  for (int k = 1; k < kMemoEntries; ++k)
+    if (scm->memo[k].used < e->used) e = &scm->memo[k];
+  e->fp = fp;
+  e->used = ++scm->memo_clock;
+  e->m = m;
+  e->grid = grid;
+  e->fn = fn;
+  e->ndist = 0;
+  for (int32_t i = 0; i < m; ++i) {
+    e->sel[i] = sel[i];
+    int32_t k = 0;
+    while (k < e->ndist && e->dist_idx[k] != sel[i]) ++k;
+    if (k == e->ndist) {
+      e->dist_idx[k] = sel[i];
+      e->dist_cnt[k] = 0;
+      ++e->ndist;
+    }
+    ++e->dist_cnt[k];
+  }
+  std::memcpy(e->args, a, (size_t)m * sizeof(trident_args));
+  if (P) std::memcpy(&e->P, P, sizeof(ChainStepParams));
+}
+
 // One chunk of trident_scm_invoke_step: select every call; if all hit layer-chain
 // versions with one kernel and the calls are independent, pack them into one launch.
+// A chunk stored in the replay cache is relaunched without re-running these steps.
 int32_t step_chunk(trident_scm* scm, const trident_args* a, int32_t m, void* stream,
                    int32_t* out_selected) {
   if (m < 2) return kNotFused;
+  const bool memo_on = !(scm->opt.flags & TRIDENT_OPT_NO_STEP_REPLAY);
+  uint64_t fp = 0;
+  bool repeat = false;
+  if (memo_on) {
+    fp = step_fingerprint(a, m);
+    if (!scm->memo_lock.test_and_set(std::memory_order_acquire)) {
+      const int32_t st = replay_chunk(scm, a, m, fp, stream, out_selected, &repeat);
+      scm->memo_lock.clear(std::memory_order_release);
+      if (st != kNotFused) return st;
+    }
+  }
   Sig sig[kStepMax];
   int32_t sel[kStepMax];
   const Version* v0 = nullptr;
@@ -1388,8 +1522,10 @@ int32_t step_chunk(trident_scm* scm, const trident_args* a, int32_t m, void* str
     for (int32_t i = 0; i < m; ++i) out_selected[i] = sel[i];
   if (scm->opt.flags & TRIDENT_OPT_FAIL_LAUNCHES)
     return count_error(scm, fail(TRIDENT_ERR_CUDA, "launch failure injected (TRIDENT_OPT_FAIL_LAUNCHES)"));
+  thread_local ChainStepParams P;
+  unsigned grid = 0;
+  CUfunction fn = nullptr;
   if (!scm->dry) {
-    thread_local ChainStepParams P;
     bool inplace = false;
     int64_t two = 0;  // blocks with two CTAs per token
     for (int32_t i = 0; i < m; ++i) {
@@ -1417,9 +1553,11 @@ int32_t step_chunk(trident_scm* scm, const trident_args* a, int32_t m, void* str
     CUlaunchConfig cfg;
     CUlaunchAttribute attr;
     base_config(scm, stream, &cfg, &attr);
-    cfg.gridDimX = (unsigned)first;
+    grid = (unsigned)first;
+    fn = split == 2 ? v0->step_fn : v0->step_fn_inplace;
+    cfg.gridDimX = grid;
     void* kp[1] = {&P};
-    const int32_t st = launch_on(scm, &cfg, split == 2 ? v0->step_fn : v0->step_fn_inplace, kp);
+    const int32_t st = launch_on(scm, &cfg, fn, kp);
     if (st != TRIDENT_OK) return count_error(scm, st);
   }
   uint64_t evals = 0;
@@ -1431,6 +1569,10 @@ int32_t step_chunk(trident_scm* scm, const trident_args* a, int32_t m, void* str
   scm->guard_evals.fetch_add(evals, std::memory_order_relaxed);
   scm->fused_launches.fetch_add(1, std::memory_order_relaxed);
   scm->fused_calls.fetch_add((uint64_t)m, std::memory_order_relaxed);
+  if (repeat && !scm->memo_lock.test_and_set(std::memory_order_acquire)) {
+    store_chunk(scm, a, m, fp, sel, scm->dry ? nullptr : &P, grid, fn);
+    scm->memo_lock.clear(std::memory_order_release);
+  }
   return TRIDENT_OK;
 }
 
@@ -1470,6 +1612,7 @@ TRIDENT_API int32_t trident_scm_stats(const trident_scm_t* scm, trident_scm_stat
   out->num_specs = scm->count.load();
   out->fused_launches = scm->fused_launches.load();
   out->fused_calls = scm->fused_calls.load();
+  out->step_replays = scm->step_replays.load();
   return TRIDENT_OK;
 }
 
@@ -1531,5 +1674,6 @@ TRIDENT_API void trident_scm_destroy(trident_scm_t* scm) {
   std::free(scm->versions);
   delete[] scm->hits_per;
   std::free(scm->ring);
+  std::free(scm->memo);
   delete scm;
 }

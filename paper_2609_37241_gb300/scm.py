@@ -22,6 +22,7 @@ OP_SILU, OP_ADD, OP_NEG, OP_MASKED_FILL = 8, 9, 10, 11
 LAYOUT_CONTIG, LAYOUT_ROWSTRIDED, LAYOUT_ANY = 0, 1, 2
 VARIANT_AUTO, VARIANT_GENERIC, VARIANT_VECTOR = 0, 1, 2
 OPT_DRY_RUN, OPT_NO_ALIAS_CHECK, OPT_PDL, OPT_TIMING, OPT_FAIL_LAUNCHES = 0x1, 0x2, 0x4, 0x8, 0x10
+OPT_NO_STEP_REPLAY = 0x20
 DEVERR_POS, DEVERR_TIMEOUT = 0x1, 0x2
 MAX_TENSORS, MAX_FIXED = 20, 8
 STEP_MAX = 48  # calls per launch of trident_scm_invoke_step
@@ -60,7 +61,8 @@ class trident_scm_stats_t(ctypes.Structure):
     _fields_ = [("invokes", c_u64), ("hits", c_u64), ("misses", c_u64), ("hook_calls", c_u64),
                 ("hook_failures", c_u64), ("hook_registered", c_u64), ("err_invalid", c_u64),
                 ("err_cuda", c_u64), ("guard_evals", c_u64), ("num_specs", c_i32),
-                ("reserved", c_i32), ("fused_launches", c_u64), ("fused_calls", c_u64)]
+                ("reserved", c_i32), ("fused_launches", c_u64), ("fused_calls", c_u64),
+                ("step_replays", c_u64)]
 
 
 class trident_node(ctypes.Structure):

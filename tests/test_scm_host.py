@@ -47,7 +47,7 @@ def test_exports_every_declared_symbol(S):
     exported = set(re.findall(r" T (trident_\w+)", nm))
     assert declared, "no declarations parsed"
     assert declared == exported, (declared ^ exported)
-    assert S.trident_abi_version() == 3
+    assert S.trident_abi_version() == 4
 
 
 def test_binding_constants_match_header_defines(S):

@@ -175,3 +175,28 @@ def test_dependent_layers_back_to_back_with_pdl(S, entry, T):
         ref = L.layer_chain(inp, cfg["theta"], cfg["eps"], BF16)
         check_chain(ref, outs[l][1], inp)
         r0 = ref["r2"]
+
+
+def test_step_replays_follow_new_data(S):
+    """A decode loop's pattern: the same buffers every step with new data in them. From the
+    third step on the chunk is relaunched from the replay cache (only argument bytes are
+    compared); each step's outputs equal the oracle on that step's data."""
+    cfg = synth.QWEN3
+    T, n = 4, 6
+    s, _ = step_scm(S, cfg, BF16, S.LAYOUT_ROWSTRIDED)
+    inps, outs, args = build_layers(S, cfg, T, n, seed=70)
+    for step in range(4):
+        if step:
+            g = np.random.default_rng(700 + step)
+            for l in range(n):
+                inps[l] = synth.layer_inputs(g, T, cfg)
+                fresh, _ = chain_device(inps[l], BF16, True)
+                for dst, src in zip(outs[l][0], fresh):
+                    dst.copy_(src)
+        assert run_step(S, s, args) == [0] * n
+        torch.cuda.synchronize()
+        for inp, (_, out) in zip(inps, outs):
+            check_chain(L.layer_chain(inp, cfg["theta"], cfg["eps"], BF16, qknorm=True), out, inp)
+    st = s.stats()
+    assert (st.step_replays, st.fused_launches, st.hits) == (2 * n, 4, 4 * n)
+    s.close()
