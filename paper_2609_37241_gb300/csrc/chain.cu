@@ -184,8 +184,9 @@ __device__ __forceinline__ void chain_block_tok(const ChainParams& c) {
 // L2 prefetch of the lines a block reads first -- the norm rows, the RoPE head-rows and
 // positions, the SwiGLU tile -- one prefetch per 128-byte line, between the launch trigger
 // and the PDL wait (see prefetch_l2).
-template <int DT, int VPT>
-__device__ __forceinline__ void norm_prefetch(const ChainParams& c, const int64_t row) {
+// A token's SPLIT norm blocks share its rows' lines: part p prefetches vectors v = p mod SPLIT.
+template <int DT, int VPT, int SPLIT>
+__device__ __forceinline__ void norm_prefetch(const ChainParams& c, const int64_t row, const int part) {
   constexpr int EB = Act<DT>::BYTES;
   const int tid = threadIdx.x;
   if ((tid & 7) != 0) return;  // 8 threads x 16 bytes = one line
@@ -194,6 +195,7 @@ __device__ __forceinline__ void norm_prefetch(const ChainParams& c, const int64_
   const uint4* ap = reinterpret_cast<const uint4*>(row_ptr(c.n2.x, row, c.n2.x_rs, EB));
 #pragma unroll
   for (int v = 0; v < VPT; ++v) {
+    if (v % SPLIT != part) continue;
     const int64_t vi = (int64_t)v * kThreads + tid;
     prefetch_l2(hp + vi);
     prefetch_l2(rp + vi);
@@ -201,12 +203,16 @@ __device__ __forceinline__ void norm_prefetch(const ChainParams& c, const int64_
   }
 }
 
+// prefetch == 1: every block; prefetch == 2: only the norm blocks (their rows are the first
+// loads of the longest blocks; the other roles' lines would compete with them for DRAM).
 template <int DT, int VPT, int SPLIT, int D>
 __device__ __forceinline__ void chain_prefetch(const ChainParams& c, const int b) {
   constexpr int LPH = D / Act<DT>::VE;
   const int tid = threadIdx.x;
   if (b < c.nA) {
-    norm_prefetch<DT, VPT>(c, b / SPLIT);
+    norm_prefetch<DT, VPT, SPLIT>(c, b / SPLIT, b % SPLIT);
+  } else if (c.prefetch == 2) {
+    return;
   } else if (b < c.nA + c.nB) {
     rope_prefetch<DT, D>(c.rope, (int64_t)(b - c.nA) * (kThreads / LPH) + tid / LPH, tid % LPH);
   } else {
@@ -223,7 +229,7 @@ __device__ __forceinline__ void chain_prefetch_tok(const ChainParams& c) {
   constexpr int LPH = D / Act<DT>::VE;
   const int tid = threadIdx.x, q = blockIdx.x;
   if (q < SPLIT) {
-    norm_prefetch<DT, VPT>(c, blockIdx.y);
+    norm_prefetch<DT, VPT, SPLIT>(c, blockIdx.y, q);
   } else if (q < SPLIT + c.rope_per_tok) {
     const int64_t rb = (int64_t)blockIdx.y * c.rope_per_tok + (q - SPLIT);
     rope_prefetch<DT, D>(c.rope, rb * (kThreads / LPH) + tid / LPH, tid % LPH);

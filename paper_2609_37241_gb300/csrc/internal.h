@@ -93,7 +93,8 @@ struct ChainParams {
   SwigluParams sw;
   int32_t nA, nB, nC, sw_tiles_per_row;
   int32_t a_split;   // CTAs per token for the norms (2, or 1 for in-place calls)
-  int32_t prefetch;  // 1: each block prefetches its input lines into L2 before the PDL wait
+  int32_t prefetch;  // before the PDL wait, into L2: 1 every block's first input lines,
+                     // 2 only the norm blocks' rows, 0 none
   int32_t tok_grid;  // 1: grid (a_split + rope_per_tok + sw_tiles_per_row, T), token-major
   int32_t rope_per_tok;  // RoPE blocks per token (token-major grid: nB = T * rope_per_tok)
   int64_t sw_tiles;  // T * sw_tiles_per_row (valid SwiGLU tiles)

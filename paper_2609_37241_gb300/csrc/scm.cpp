@@ -689,6 +689,17 @@ int32_t set_chain_split(ChainParams* c, int64_t T, int32_t split, int64_t* block
   return TRIDENT_OK;
 }
 
+// Layer-chain prefetch before the PDL wait: every block's first lines for grids of at most
+// one block per SM (small_grid); otherwise, while the grid still fits one wave (two norm
+// CTAs per token), only the norm blocks' rows -- the first loads of the longest blocks, which
+// then come from L2 while every other block's loads stream from DRAM (64 tokens: 4.32 ->
+// 3.98 us per launch back to back in a per-block timeline probe; prefetching every block's
+// lines there was slower, 4.26 -> 4.68 us).
+inline int32_t chain_prefetch_mode(bool pdl, int32_t small_grid, int32_t split) {
+  if (!pdl) return 0;
+  return small_grid ? 1 : (split == 2 ? 2 : 0);
+}
+
 inline unsigned cap_grid(int64_t n) { return (unsigned)(n < 1 ? 1 : (n > 0x7fffffff ? 0x7fffffff : n)); }
 
 int32_t do_launch(trident_scm* scm, const Version& v, const trident_args* a, const Sig& s,
@@ -779,9 +790,10 @@ int32_t do_launch(trident_scm* scm, const Version& v, const trident_args* a, con
   }
   // L2 prefetch before the PDL wait (prefetch_l2 in device_common.cuh): only for grids of
   // at most one block per SM launched with programmatic serialisation (measured: ~10%
-  // faster layer steps at 1-4 tokens; slower once the grid fills the GPU)
-  const int32_t pf = (scm->opt.flags & TRIDENT_OPT_PDL) &&
-                     (int64_t)cfg.gridDimX * cfg.gridDimY <= scm->sm_count ? 1 : 0;
+  // faster layer steps at 1-4 tokens; slower once the grid fills the GPU, where a layer
+  // chain prefetches only its norm rows -- see chain_prefetch_mode)
+  const bool pdl = (scm->opt.flags & TRIDENT_OPT_PDL) != 0;
+  const int32_t pf = pdl && (int64_t)cfg.gridDimX * cfg.gridDimY <= scm->sm_count ? 1 : 0;
   switch (op) {
     case TRIDENT_OP_ADD_RMSNORM: P.an.prefetch = pf; break;
     case TRIDENT_OP_RMSNORM: P.rn.prefetch = pf; break;
@@ -789,7 +801,7 @@ int32_t do_launch(trident_scm* scm, const Version& v, const trident_args* a, con
     case TRIDENT_OP_QKNORM_ROPE_KV: P.rp.prefetch = pf; break;
     case TRIDENT_OP_SWIGLU: P.sw.prefetch = pf; break;
     case TRIDENT_OP_LAYER_CHAIN:
-    case TRIDENT_OP_LAYER_CHAIN_QKNORM: P.ch.prefetch = pf; break;
+    case TRIDENT_OP_LAYER_CHAIN_QKNORM: P.ch.prefetch = chain_prefetch_mode(pdl, pf, P.ch.a_split); break;
     default: P.pw.prefetch = pf; break;
   }
   CUfunction fn = v.fn;
@@ -1548,7 +1560,8 @@ int32_t step_chunk(trident_scm* scm, const trident_args* a, int32_t m, void* str
     P.first[m] = (int32_t)first;
     P.n = m;
     // L2 prefetch before the PDL wait under the same rule as single calls (do_launch)
-    const int32_t pf = (scm->opt.flags & TRIDENT_OPT_PDL) && first <= scm->sm_count ? 1 : 0;
+    const int32_t pf = chain_prefetch_mode((scm->opt.flags & TRIDENT_OPT_PDL) != 0,
+                                           first <= scm->sm_count ? 1 : 0, split);
     for (int32_t i = 0; i < m; ++i) P.c[i].prefetch = pf;
     CUlaunchConfig cfg;
     CUlaunchAttribute attr;
