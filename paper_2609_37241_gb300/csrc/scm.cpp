@@ -690,14 +690,15 @@ int32_t set_chain_split(ChainParams* c, int64_t T, int32_t split, int64_t* block
 }
 
 // Layer-chain prefetch before the PDL wait: every block's first lines for grids of at most
-// one block per SM (small_grid); otherwise, while the grid still fits one wave (two norm
-// CTAs per token), only the norm blocks' rows -- the first loads of the longest blocks, which
-// then come from L2 while every other block's loads stream from DRAM (64 tokens: 4.32 ->
-// 3.98 us per launch back to back in a per-block timeline probe; prefetching every block's
-// lines there was slower, 4.26 -> 4.68 us).
-inline int32_t chain_prefetch_mode(bool pdl, int32_t small_grid, int32_t split) {
+// one block per SM (small_grid); otherwise, when norm_rows, only the norm blocks' rows --
+// the first loads of the longest blocks, which then come from L2 while every other block's
+// loads stream from DRAM. Measured: one call at 64 tokens (one wave) 3.80 -> 3.53 us per
+// layer step and at 128 tokens (two waves) 6.1 -> 5.8 us; prefetching every block's lines
+// there was slower (4.26 -> 4.68 us at 64 tokens). Whole-step launches take it only with two
+// norm CTAs per token (one wave): on multi-wave steps it measured 1-2 % slower.
+inline int32_t chain_prefetch_mode(bool pdl, bool small_grid, bool norm_rows) {
   if (!pdl) return 0;
-  return small_grid ? 1 : (split == 2 ? 2 : 0);
+  return small_grid ? 1 : (norm_rows ? 2 : 0);
 }
 
 inline unsigned cap_grid(int64_t n) { return (unsigned)(n < 1 ? 1 : (n > 0x7fffffff ? 0x7fffffff : n)); }
@@ -801,7 +802,7 @@ int32_t do_launch(trident_scm* scm, const Version& v, const trident_args* a, con
     case TRIDENT_OP_QKNORM_ROPE_KV: P.rp.prefetch = pf; break;
     case TRIDENT_OP_SWIGLU: P.sw.prefetch = pf; break;
     case TRIDENT_OP_LAYER_CHAIN:
-    case TRIDENT_OP_LAYER_CHAIN_QKNORM: P.ch.prefetch = chain_prefetch_mode(pdl, pf, P.ch.a_split); break;
+    case TRIDENT_OP_LAYER_CHAIN_QKNORM: P.ch.prefetch = chain_prefetch_mode(pdl, pf != 0, true); break;
     default: P.pw.prefetch = pf; break;
   }
   CUfunction fn = v.fn;
@@ -1561,7 +1562,7 @@ int32_t step_chunk(trident_scm* scm, const trident_args* a, int32_t m, void* str
     P.n = m;
     // L2 prefetch before the PDL wait under the same rule as single calls (do_launch)
     const int32_t pf = chain_prefetch_mode((scm->opt.flags & TRIDENT_OPT_PDL) != 0,
-                                           first <= scm->sm_count ? 1 : 0, split);
+                                           first <= scm->sm_count, split == 2);
     for (int32_t i = 0; i < m; ++i) P.c[i].prefetch = pf;
     CUlaunchConfig cfg;
     CUlaunchAttribute attr;
