@@ -193,3 +193,67 @@ def test_fuzz_layer_chain(S, seed):
     desc = S.make_spec(op, dtype, fixed, 1, 4096, layout=lay, rope_theta=cfg["theta"])
     run_one(S, desc, op, ts, pdl, eps=cfg["eps"], rope_theta=cfg["theta"])
     check_chain(ref, out, inp, dtype)
+
+
+@pytest.mark.parametrize("seed", range(6))
+def test_fuzz_step_replay(S, seed):
+    """invoke_step over several independent layers, four steps on the same buffers with new
+    data each time (steps 3 and 4 replay the stored chunk), then a fifth step in which one layer
+    reads another's output (never replayed: it runs call by call). Every step's outputs are
+    checked against the oracle on that step's data."""
+    rng = random.Random(400 + seed)
+    base = rng.choice([synth.LLAMA, synth.QWEN3])
+    dtype = rng.choice([BF16, FP16])
+    T = rng.choice([1, 3, 8, 17])
+    n = rng.choice([2, 3, 5])
+    cfg = dict(base, S=rng.choice([128, 8192]))
+    qk = cfg["qknorm"]
+    layout = rng.choice(["fused", "separate"])
+    op = S.OP_LAYER_CHAIN_QKNORM if qk else S.OP_LAYER_CHAIN
+    fixed = [cfg["H"], cfg["Hq"], cfg["Hkv"], cfg["D"], cfg["S"], cfg["I"]]
+    lay = S.LAYOUT_ROWSTRIDED if (layout == "fused" and T > 1) else S.LAYOUT_CONTIG
+    s = S.Scm(device=0, flags=S.OPT_PDL if rng.random() < 0.7 else 0)
+    s.register(S.make_spec(op, dtype, fixed, 1, 4096, layout=lay, rope_theta=cfg["theta"]))
+    g = np.random.default_rng(400 + seed)
+    inps = [synth.layer_inputs(g, T, cfg, dtype=dtype) for _ in range(n)]
+    dev = [chain_device(inp, dtype, qk, layout=layout) for inp in inps]
+    args = [S.make_args(op, ts, eps=cfg["eps"], rope_theta=cfg["theta"]) for ts, _ in dev]
+
+    def step(a):
+        st, sel = s.invoke_step((S.trident_args * n)(*a), stream())
+        assert st == S.OK and sel == [0] * n, S.trident_scm_last_error()
+        torch.cuda.synchronize()
+        assert S.trident_scm_device_status(s.h, stream())[1] == 0
+
+    for k in range(4):
+        if k:
+            for l in range(n):
+                inps[l] = synth.layer_inputs(g, T, cfg, dtype=dtype)
+                fresh, _ = chain_device(inps[l], dtype, qk, layout=layout)
+                for dst, src in zip(dev[l][0], fresh):
+                    dst.copy_(src)
+        step(args)
+        for inp, (_, out) in zip(inps, dev):
+            check_chain(L.layer_chain(inp, cfg["theta"], cfg["eps"], dtype, qknorm=qk), out, inp, dtype)
+    st = s.stats()
+    assert (st.step_replays, st.fused_launches) == (2 * n, 4)
+    # layer 1 now reads layer 0's second residual output: dependent, run in order
+    for l in range(n):
+        inps[l] = synth.layer_inputs(g, T, cfg, dtype=dtype)
+        fresh, _ = chain_device(inps[l], dtype, qk, layout=layout)
+        for dst, src in zip(dev[l][0], fresh):
+            dst.copy_(src)
+    ts1 = list(dev[1][0])
+    ts1[1] = dev[0][1]["r2"]
+    dep = list(args)
+    dep[1] = S.make_args(op, ts1, eps=cfg["eps"], rope_theta=cfg["theta"])
+    step(dep)
+    st = s.stats()
+    assert (st.step_replays, st.fused_launches) == (2 * n, 4)
+    s.close()
+    ref0 = L.layer_chain(inps[0], cfg["theta"], cfg["eps"], dtype, qknorm=qk)
+    inp1 = dict(inps[1], r0=ref0["r2"])
+    check_chain(ref0, dev[0][1], inps[0], dtype)
+    check_chain(L.layer_chain(inp1, cfg["theta"], cfg["eps"], dtype, qknorm=qk), dev[1][1], inp1, dtype)
+    for l in range(2, n):
+        check_chain(L.layer_chain(inps[l], cfg["theta"], cfg["eps"], dtype, qknorm=qk), dev[l][1], inps[l], dtype)
