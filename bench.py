@@ -412,6 +412,47 @@ def bench_layer(c, cfg, T, K, W, layers=1, min_bytes=2 * L2_BYTES):
     return res, sets
 
 
+def bench_launch_floor(c, n=2000):
+    """Single-launch latency floor: an empty kernel launched back to back through the
+    library's own launch path (trident_launch_floor: same context, driver entry point and
+    launch attributes as a hit), with and without programmatic dependent launch. Device us
+    per launch from CUDA events around one native call of n launches; host us per launch
+    from the host clock around the same call."""
+    S, t = c.S, c.torch
+    res = {}
+    for name, flags in (("pdl", S.OPT_PDL), ("no_pdl", 0)):
+        s = S.Scm(device=c.dev.index or 0, flags=flags)
+        assert S.trident_launch_floor(s.h, c.sp.value, 20) == S.OK, S.trident_scm_last_error()
+        t.cuda.synchronize()
+        e0, e1 = c.events()
+        h0 = time.perf_counter()
+        e0.record(c.stream)
+        st = S.trident_launch_floor(s.h, c.sp.value, n)
+        e1.record(c.stream)
+        h1 = time.perf_counter()
+        t.cuda.synchronize()
+        assert st == S.OK, S.trident_scm_last_error()
+        res[name] = dict(device_us=round(e0.elapsed_time(e1) * 1e3 / n, 3),
+                         host_us=round((h1 - h0) * 1e6 / n, 3))
+        s.close()
+    c.launches += 2 * (n + 20)
+    return res
+
+
+def add_floor_fractions(per_t, floor_us, layers=1):
+    """Fraction of the single-launch latency floor (n_launches x the empty-kernel launch
+    time) that each decode-size step reaches: 1.0 would be a step as fast as its launches."""
+    for v in per_t.values():
+        n_fused, n_unf = v["launches_per_step"]
+        v["floor_frac"] = dict(fused=round(n_fused * floor_us / v["fused_us"], 3),
+                               unfused=round(n_unf * floor_us / v["unfused_us"], 3))
+        o = v.get("one_launch_step")
+        if o:
+            v["floor_frac"]["one_launch_step"] = round(o["launches_per_step"] * floor_us / o["us"], 3)
+            if "replayed" in o:
+                v["floor_frac"]["replayed"] = round(o["launches_per_step"] * floor_us / o["replayed"]["us"], 3)
+
+
 def bench_e2e(c, cfg, T, K, W):
     """End to end through the public API: per step, one pinned host -> device copy of the
     layer's inputs (h, r0, attn_out, qkv, gate|up, pos laid out in one staging arena), one
@@ -1036,11 +1077,17 @@ def run_ours(a):
     extra = {}
     want = (lambda name: True) if a.sections == "all" else (lambda name: name in a.sections.split(","))
     toks_arg = [int(x) for x in a.tokens.split(",")] if a.tokens else None
+    floor_us = None
+    if rank == 0 and (want("floor") or want("layers") or want("qwen3")):
+        progress("launch floor")
+        extra["latency_floor"] = bench_launch_floor(c)
+        floor_us = extra["latency_floor"]["pdl"]["device_us"]
     if rank == 0 and want("layers"):
         progress("per-token layer steps")
         per_t = {}
         for T in (1, 4, 16, 64):
             per_t[str(T)], _ = bench_layer(c, cfg, T, K=min(K, 2000), W=W)
+        add_floor_fractions(per_t, floor_us)
         extra["llama_per_tokens"] = per_t
     if rank == 0 and want("qwen3"):
         progress("qwen3 36-layer steps")
@@ -1050,6 +1097,7 @@ def run_ours(a):
         for T in toks:
             qw[str(T)], _ = bench_layer(c, synth.QWEN3, T, K=max(20, min(K, 2000) // 36), W=W,
                                         layers=36)
+        add_floor_fractions(qw, floor_us)
         extra["qwen3_36layer_step"] = qw
     if rank == 0 and want("host"):
         progress("host dispatch")
@@ -1166,7 +1214,7 @@ def main():
     p.add_argument("--quick", action="store_true", help="smaller sections (for smoke runs)")
     p.add_argument("--tokens", default="", help="comma list of token counts for the qwen3 and sweep sections")
     p.add_argument("--sections", default="all",
-                   help="comma list of: layers,qwen3,host,stress,motivation,kernels,sweep,roofline,e2e,cpu"
+                   help="comma list of: floor,layers,qwen3,host,stress,motivation,kernels,sweep,roofline,e2e,cpu"
                         " (default all;"
                         " the headline always runs)")
     a = p.parse_args()

@@ -450,6 +450,15 @@ int32_t trident_scm_spec_hits(const trident_scm_t* scm, uint64_t* out, int32_t c
  * count. Samples are recorded per hit, so concurrent invokers may interleave. */
 int32_t trident_scm_host_times(const trident_scm_t* scm, uint32_t* out, int32_t cap, int32_t* n);
 
+/* Latency-floor probe (measurement, not part of the dispatch path): launches n empty
+ * kernels (one block of 32 threads; the kernel only takes part in programmatic dependent
+ * launch) back to back on `stream`, with the SCM's launch configuration (its context, and
+ * programmatic stream serialisation when TRIDENT_OPT_PDL is set) through the same driver
+ * entry point as a hit. The time per launch is the single-launch floor against which
+ * decode-size steps are reported. Reads and writes no memory. Errors: ERR_INVALID (scm
+ * NULL or n < 0), ERR_STATE (dry-run SCM), ERR_CUDA. */
+int32_t trident_launch_floor(trident_scm_t* scm, void* stream, int32_t n);
+
 /* Reads the device status word (TRIDENT_DEVERR_* bits) after synchronising `stream`;
  * clears it when clear != 0. Errors: ERR_STATE in dry-run mode, ERR_CUDA. */
 int32_t trident_scm_device_status(trident_scm_t* scm, void* stream, uint32_t* out_bits,

@@ -145,6 +145,7 @@ bool rope_kernel(int32_t dtype, int32_t variant, int32_t D, bool qknorm, KernelE
 bool swiglu_kernel(int32_t dtype, int32_t variant, int64_t I, KernelEntry* out, const char** why);
 bool chain_kernel(int32_t dtype, int64_t H, int32_t D, bool qknorm, KernelEntry* out,
                   const char** why);
+const void* empty_kernel_entry();  // the latency-floor probe's kernel (does nothing)
 
 // Validation, guard-equivalent checks (sizes, layouts, 16-byte alignment, overlap) and
 // parameter packing of a ROPE_KV / QKNORM_ROPE_KV argument tuple without an SCM. Leaves

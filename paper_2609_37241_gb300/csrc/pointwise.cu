@@ -130,6 +130,15 @@ static const void* pick(int32_t op, bool vec) {
   return nullptr;
 }
 
+// Latency-floor probe (trident_launch_floor): a kernel that does nothing but take part in
+// programmatic dependent launch like every kernel of the library.
+__global__ void empty_kernel() {
+  pdl_trigger();
+  pdl_wait();
+}
+
+const void* empty_kernel_entry() { return (const void*)empty_kernel; }
+
 bool pointwise_kernel(int32_t op, int32_t dtype, int32_t variant, int64_t W, KernelEntry* out,
                       const char** why) {
   if (dtype != DT_BF16 && dtype != DT_FP16 && dtype != DT_FP32) { *why = "dtype"; return false; }

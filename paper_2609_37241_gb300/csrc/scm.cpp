@@ -1668,6 +1668,28 @@ TRIDENT_API int32_t trident_scm_device_status(trident_scm_t* scm, void* stream, 
   });
 }
 
+TRIDENT_API int32_t trident_launch_floor(trident_scm_t* scm, void* stream, int32_t n) {
+  if (!scm || n < 0) return fail(TRIDENT_ERR_INVALID, "bad arguments");
+  if (scm->dry) return fail(TRIDENT_ERR_STATE, "dry-run SCM launches nothing");
+  static std::once_flag once;
+  static CUfunction fn = nullptr;
+  std::call_once(once, [] {
+    cudaFunction_t f = nullptr;
+    if (cudaGetFuncBySymbol(&f, empty_kernel_entry()) == cudaSuccess) fn = reinterpret_cast<CUfunction>(f);
+  });
+  if (!fn) return fail(TRIDENT_ERR_CUDA, "cannot resolve the empty kernel");
+  CUlaunchConfig cfg;
+  CUlaunchAttribute attr;
+  base_config(scm, stream, &cfg, &attr);
+  cfg.blockDimX = 32;
+  cfg.gridDimX = 1;
+  for (int32_t i = 0; i < n; ++i) {
+    const int32_t st = launch_on(scm, &cfg, fn, nullptr);
+    if (st != TRIDENT_OK) return st;
+  }
+  return TRIDENT_OK;
+}
+
 TRIDENT_API void trident_scm_destroy(trident_scm_t* scm) {
   if (!scm) return;
   if (!scm->dry && (scm->d_err || !scm->tables.empty())) {

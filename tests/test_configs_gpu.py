@@ -184,3 +184,16 @@ def test_qwen3_36_layers_through_one_table(S):
         P.check_act(hb(o["o"]), ref["o_ref"], ref["o"], BF16, f"layer {l} o")
         assert np.array_equal(hb(o["v_cache"]), ref["v_cache"])
     s.close()
+
+
+@pytest.mark.parametrize("pdl", [False, True])
+def test_launch_floor_probe_runs(S, pdl):
+    """The latency-floor probe launches its empty kernels through the hit path's launch code
+    (with and without programmatic dependent launch) and leaves the stream usable."""
+    s = S.Scm(device=0, flags=S.OPT_PDL if pdl else 0)
+    st = torch.cuda.current_stream().cuda_stream
+    assert S.trident_launch_floor(s.h, st, 100) == S.OK, S.trident_scm_last_error()
+    assert S.trident_launch_floor(s.h, st, 0) == S.OK
+    torch.cuda.synchronize()
+    assert S.trident_scm_device_status(s.h, st)[1] == 0
+    s.close()

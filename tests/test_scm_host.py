@@ -462,3 +462,11 @@ def test_execution_error_is_raised_not_retried(S):
     st, sels = S.trident_scm_invoke_seq(s.h, arr)
     assert st == S.ERR_CUDA and sels == [-1, 0, S.NOT_RUN] and len(calls) == 2
     s.close()
+
+
+def test_launch_floor_probe_rejects_dry_runs_and_bad_counts(S):
+    s = S.Scm(device=0, flags=S.OPT_DRY_RUN)
+    assert S.trident_launch_floor(s.h, None, 1) == S.ERR_STATE
+    assert S.trident_launch_floor(s.h, None, -1) == S.ERR_INVALID
+    assert S.trident_launch_floor(None, None, 1) == S.ERR_INVALID
+    s.close()
