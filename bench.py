@@ -632,9 +632,24 @@ def bench_host_hit(c, n=1000):
     d.close()
     st, ns = S.trident_scm_host_times(s.h, n)
     hits = S.trident_scm_spec_hits(s.h)[1]
+    # one call at a time (after the samples above were read): device us from an event
+    # recorded before the call to one after it, and host us from the call to the return of
+    # that event's synchronise (launch to completion)
+    e0, e1 = c.events()
+    ev_us, wall_us = [], []
+    for _ in range(200):
+        t.cuda.synchronize()
+        w0 = time.perf_counter()
+        e0.record(c.stream)
+        inv(s.h, ar, c.sp, ctypes.byref(sel))
+        e1.record(c.stream)
+        e1.synchronize()
+        w1 = time.perf_counter()
+        ev_us.append(e0.elapsed_time(e1) * 1e3)
+        wall_us.append((w1 - w0) * 1e6)
     assert_all_hit(s, "host dispatch")
     ns = np.array(ns[-n:], np.float64)
-    c.launches += n
+    c.launches += n + 200
     s.close()
     # the fused layer chain (18 tensors, 64 tokens): host ns per hit with the launch, and alone
     cfg = synth.LLAMA
@@ -658,6 +673,9 @@ def bench_host_hit(c, n=1000):
         cs.close()
     del sets
     return dict(hits_on_bf16_contig=int(hits[3]), calls=n, selected=sel.value, layer_chain=chain_ns,
+                isolated_call=dict(event_us_median=round(float(np.median(ev_us)), 3),
+                                   launch_to_completion_us_median=round(float(np.median(wall_us)), 3),
+                                   calls=len(ev_us)),
                 median_ns=float(np.median(ns)), p99_ns=float(np.percentile(ns, 99)),
                 min_ns=float(ns.min()), guards_only_median_ns=float(np.median(dns)),
                 python_call_us_ctypes=round((h1 - h0) * 1e6 / n, 3), python_call_us_fastcall=fast_us)
