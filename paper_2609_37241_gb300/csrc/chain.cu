@@ -20,7 +20,6 @@
 
 namespace trident {
 
-constexpr int kChainSwigluUnroll = 2;
 
 // Norm role: part `part` (< SPLIT) of token `row`'s two add+RMSNorm steps.
 template <int DT, int VPT, int SPLIT>
@@ -140,14 +139,15 @@ __device__ __forceinline__ void chain_rope(const ChainParams& c, const int64_t r
   if (unit < c.rope.T * c.rope.NH) rope_head_row<DT, D, QKNORM>(c.rope, unit, threadIdx.x % LPH);
 }
 
-// SwiGLU role: column tile `col_tile` of row `row`.
-template <int DT>
+// SwiGLU role: column tile `col_tile` of row `row`, SWU x 256 16-byte vectors of g and of u
+// (kChainSwigluUnroll for one call's grid, kChainStepSwigluUnroll for a whole step's).
+template <int DT, int SWU>
 __device__ __forceinline__ void chain_swiglu(const ChainParams& c, const int64_t row, const int64_t col_tile) {
-  swiglu_tile<DT, kChainSwigluUnroll>(c.sw, row, col_tile * kChainSwigluUnroll * kThreads, threadIdx.x);
+  swiglu_tile<DT, SWU>(c.sw, row, col_tile * SWU * kThreads, threadIdx.x);
 }
 
 // Block b of one call's role-major grid (b < nA + nB + nC): [norms | RoPE | SwiGLU].
-template <int DT, int VPT, int SPLIT, int D, bool QKNORM>
+template <int DT, int VPT, int SPLIT, int D, bool QKNORM, int SWU>
 __device__ __forceinline__ void chain_block(const ChainParams& c, const int b) {
   if (b < c.nA) {
     const int64_t row = b / SPLIT;
@@ -158,7 +158,7 @@ __device__ __forceinline__ void chain_block(const ChainParams& c, const int b) {
     const int64_t tile = b - c.nA - c.nB;
     if (tile >= c.sw_tiles) return;
     const int64_t row = tile / c.sw_tiles_per_row;
-    chain_swiglu<DT>(c, row, tile - row * c.sw_tiles_per_row);
+    chain_swiglu<DT, SWU>(c, row, tile - row * c.sw_tiles_per_row);
   }
 }
 
@@ -177,7 +177,7 @@ __device__ __forceinline__ void chain_block_tok(const ChainParams& c) {
   } else if (q < SPLIT + c.rope_per_tok) {
     chain_rope<DT, D, QKNORM>(c, (int64_t)blockIdx.y * c.rope_per_tok + (q - SPLIT));
   } else {
-    chain_swiglu<DT>(c, blockIdx.y, q - SPLIT - c.rope_per_tok);
+    chain_swiglu<DT, kChainSwigluUnroll>(c, blockIdx.y, q - SPLIT - c.rope_per_tok);
   }
 }
 
@@ -205,7 +205,7 @@ __device__ __forceinline__ void norm_prefetch(const ChainParams& c, const int64_
 
 // prefetch == 1: every block; prefetch == 2: only the norm blocks (their rows are the first
 // loads of the longest blocks; the other roles' lines would compete with them for DRAM).
-template <int DT, int VPT, int SPLIT, int D>
+template <int DT, int VPT, int SPLIT, int D, int SWU>
 __device__ __forceinline__ void chain_prefetch(const ChainParams& c, const int b) {
   constexpr int LPH = D / Act<DT>::VE;
   const int tid = threadIdx.x;
@@ -219,8 +219,7 @@ __device__ __forceinline__ void chain_prefetch(const ChainParams& c, const int b
     const int64_t tile = b - c.nA - c.nB;
     if (tile >= c.sw_tiles) return;
     const int64_t row = tile / c.sw_tiles_per_row;
-    swiglu_prefetch<DT, kChainSwigluUnroll>(
-        c.sw, row, (tile - row * c.sw_tiles_per_row) * kChainSwigluUnroll * kThreads, tid);
+    swiglu_prefetch<DT, SWU>(c.sw, row, (tile - row * c.sw_tiles_per_row) * SWU * kThreads, tid);
   }
 }
 
@@ -250,9 +249,9 @@ __global__ void __launch_bounds__(kThreads, VPT == 2 ? 4 : 2)
     pdl_wait();
     chain_block_tok<DT, VPT, SPLIT, D, QKNORM>(c);
   } else {
-    if (c.prefetch) chain_prefetch<DT, VPT, SPLIT, D>(c, blockIdx.x);
+    if (c.prefetch) chain_prefetch<DT, VPT, SPLIT, D, kChainSwigluUnroll>(c, blockIdx.x);
     pdl_wait();
-    chain_block<DT, VPT, SPLIT, D, QKNORM>(c, blockIdx.x);
+    chain_block<DT, VPT, SPLIT, D, QKNORM, kChainSwigluUnroll>(c, blockIdx.x);
   }
 }
 
@@ -269,9 +268,9 @@ __global__ void __launch_bounds__(kThreads, VPT == 2 ? 4 : 2)
     if (b >= p.first[mid]) lo = mid;
     else hi = mid - 1;
   }
-  if (p.c[lo].prefetch) chain_prefetch<DT, VPT, SPLIT, D>(p.c[lo], b - p.first[lo]);
+  if (p.c[lo].prefetch) chain_prefetch<DT, VPT, SPLIT, D, kChainStepSwigluUnroll>(p.c[lo], b - p.first[lo]);
   pdl_wait();
-  chain_block<DT, VPT, SPLIT, D, QKNORM>(p.c[lo], b - p.first[lo]);
+  chain_block<DT, VPT, SPLIT, D, QKNORM, kChainStepSwigluUnroll>(p.c[lo], b - p.first[lo]);
 }
 
 template <int DT, int SPLIT, bool QK>

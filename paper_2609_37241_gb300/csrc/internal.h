@@ -105,6 +105,13 @@ struct ChainParams {
 // the single-call kernel. The struct is passed as the kernel parameter (about 21 KB, under
 // the 32 KB parameter limit), so no device buffer is written before the launch.
 constexpr int kStepMax = 48;
+// SwiGLU tile width of the layer chain's blocks, in 256-thread rounds of 16-byte vectors of
+// g and of u: one call's grid keeps tiles small (more blocks for small token counts); a whole
+// step's grid, several waves long, does better with fewer, larger tiles (measured on 36 Qwen3
+// layers: 8 tokens 11.7 -> 11.4 us, 32 tokens 39.1 -> 37.2 us, 128 tokens 155 -> 150 us;
+// the same change on single calls made them slower, 64 tokens 3.56 -> 4.09 us).
+constexpr int kChainSwigluUnroll = 2;
+constexpr int kChainStepSwigluUnroll = 4;
 struct ChainStepParams {
   int32_t n;
   int32_t first[kStepMax + 1];

@@ -652,14 +652,16 @@ void base_config(const trident_scm* scm, void* stream, CUlaunchConfig* cfg, CUla
 }
 
 // Packs one layer-chain call: both norms, RoPE/KV, SwiGLU and the RoPE and SwiGLU block
-// counts. The norm split (set_chain_split) is decided by the caller.
+// counts, for SwiGLU tiles of `unroll` x 256 vectors (kChainSwigluUnroll in a call's own
+// launch, kChainStepSwigluUnroll in a whole-step launch). The norm split (set_chain_split)
+// is decided by the caller.
 int32_t pack_chain(trident_scm* scm, const Version& v, const trident_args* a, const Sig& s,
-                   ChainParams* c) {
+                   int32_t unroll, ChainParams* c) {
   pack_addnorm(a, C_H, C_R0, C_GA, C_X1, C_R1, s, K_ACT_H, &c->n1);
   pack_addnorm(a, C_AO, C_R1, C_GM, C_X2, C_R2, s, K_ACT_H, &c->n2);
   pack_rope(a, C_Q, a->op == TRIDENT_OP_LAYER_CHAIN_QKNORM ? C_GQ : -1, v, scm->d_err, &c->rope);
   pack_swiglu(a, C_G, C_U, C_O, s.T, &c->sw);
-  const int64_t per = (int64_t)v.ke.unroll * kThreads * v.ke.vec;
+  const int64_t per = (int64_t)unroll * kThreads * v.ke.vec;
   const int64_t tiles = (c->sw.I + per - 1) / per;
   const int64_t upb = rope_units_per_block(c->rope.D, 2);
   const int64_t nB = (s.T * c->rope.NH + upb - 1) / upb, nC = s.T * tiles;
@@ -762,7 +764,7 @@ int32_t do_launch(trident_scm* scm, const Version& v, const trident_args* a, con
     case TRIDENT_OP_LAYER_CHAIN:
     case TRIDENT_OP_LAYER_CHAIN_QKNORM: {
       ChainParams& c = P.ch;
-      int32_t st = pack_chain(scm, v, a, s, &c);
+      int32_t st = pack_chain(scm, v, a, s, v.ke.unroll, &c);
       if (st != TRIDENT_OK) return st;
       // Two CTAs per token for the norms -- so no SM carries a whole token's norm traffic --
       // while the grid still fits in one wave, and unless an output is written over an
@@ -1543,7 +1545,7 @@ int32_t step_chunk(trident_scm* scm, const trident_args* a, int32_t m, void* str
     int64_t two = 0;  // blocks with two CTAs per token
     for (int32_t i = 0; i < m; ++i) {
       ChainParams& c = P.c[i];
-      const int32_t st = pack_chain(scm, scm->versions[sel[i]], a + i, sig[i], &c);
+      const int32_t st = pack_chain(scm, scm->versions[sel[i]], a + i, sig[i], kChainStepSwigluUnroll, &c);
       if (st != TRIDENT_OK) return count_error(scm, st);
       inplace = inplace || chain_inplace(a + i);
       two += 2 * sig[i].T + c.nB + c.nC;
