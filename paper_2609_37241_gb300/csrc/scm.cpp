@@ -1673,13 +1673,15 @@ TRIDENT_API int32_t trident_scm_device_status(trident_scm_t* scm, void* stream, 
 TRIDENT_API int32_t trident_launch_floor(trident_scm_t* scm, void* stream, int32_t n) {
   if (!scm || n < 0) return fail(TRIDENT_ERR_INVALID, "bad arguments");
   if (scm->dry) return fail(TRIDENT_ERR_STATE, "dry-run SCM launches nothing");
-  static std::once_flag once;
-  static CUfunction fn = nullptr;
-  std::call_once(once, [] {
+  CUfunction fn = nullptr;  // resolved in the SCM's own context (a handle is per context)
+  const int32_t rs = on_device(scm, [&]() -> int32_t {
     cudaFunction_t f = nullptr;
-    if (cudaGetFuncBySymbol(&f, empty_kernel_entry()) == cudaSuccess) fn = reinterpret_cast<CUfunction>(f);
+    if (cudaGetFuncBySymbol(&f, empty_kernel_entry()) != cudaSuccess || !f)
+      return fail(TRIDENT_ERR_CUDA, "cannot resolve the empty kernel");
+    fn = reinterpret_cast<CUfunction>(f);
+    return TRIDENT_OK;
   });
-  if (!fn) return fail(TRIDENT_ERR_CUDA, "cannot resolve the empty kernel");
+  if (rs != TRIDENT_OK) return rs;
   CUlaunchConfig cfg;
   CUlaunchAttribute attr;
   base_config(scm, stream, &cfg, &attr);
