@@ -203,14 +203,30 @@ __device__ __forceinline__ void norm_prefetch(const ChainParams& c, const int64_
   }
 }
 
-// prefetch == 1: every block; prefetch == 2: only the norm blocks (their rows are the first
-// loads of the longest blocks; the other roles' lines would compete with them for DRAM).
+// The token's RoPE head-rows (its q, k and v rows), prefetched by its norm blocks: part p of
+// SPLIT takes head-rows [p * ceil(NH / SPLIT), ...), one thread per 128-byte line.
+template <int DT, int SPLIT, int D>
+__device__ __forceinline__ void norm_rope_prefetch(const ChainParams& c, const int64_t row, const int part) {
+  constexpr int VE = Act<DT>::VE;
+  constexpr int EB = Act<DT>::BYTES;
+  constexpr int LINES = (D * EB + 127) / 128;      // 128-byte lines per head-row
+  constexpr int LANES_PER_LINE = 128 / (VE * EB);  // lanes of a head-row per line
+  const int per = (c.rope.NH + SPLIT - 1) / SPLIT;
+  const int k = threadIdx.x / LINES;
+  if (k >= per || part * per + k >= c.rope.NH) return;
+  rope_prefetch<DT, D>(c.rope, row * c.rope.NH + part * per + k, (threadIdx.x % LINES) * LANES_PER_LINE);
+}
+
+// prefetch == 1: every block its own first lines; prefetch == 2: only the norm blocks, which
+// take their token's rows and its RoPE head-rows (the other roles' own prefetches, issued by
+// hundreds of blocks while the previous kernel finishes, measured slower).
 template <int DT, int VPT, int SPLIT, int D, int SWU>
 __device__ __forceinline__ void chain_prefetch(const ChainParams& c, const int b) {
   constexpr int LPH = D / Act<DT>::VE;
   const int tid = threadIdx.x;
   if (b < c.nA) {
     norm_prefetch<DT, VPT, SPLIT>(c, b / SPLIT, b % SPLIT);
+    if (c.prefetch == 2) norm_rope_prefetch<DT, SPLIT, D>(c, b / SPLIT, b % SPLIT);
   } else if (c.prefetch == 2) {
     return;
   } else if (b < c.nA + c.nB) {

@@ -692,12 +692,14 @@ int32_t set_chain_split(ChainParams* c, int64_t T, int32_t split, int64_t* block
 }
 
 // Layer-chain prefetch before the PDL wait: every block's first lines for grids of at most
-// one block per SM (small_grid); otherwise, when norm_rows, only the norm blocks' rows --
-// the first loads of the longest blocks, which then come from L2 while every other block's
-// loads stream from DRAM. Measured: one call at 64 tokens (one wave) 3.80 -> 3.53 us per
-// layer step and at 128 tokens (two waves) 6.1 -> 5.8 us; prefetching every block's lines
-// there was slower (4.26 -> 4.68 us at 64 tokens). Whole-step launches take it only with two
-// norm CTAs per token (one wave): on multi-wave steps it measured 1-2 % slower.
+// one block per SM (small_grid); otherwise, when norm_rows, only the norm blocks prefetch:
+// their rows -- the first loads of the longest blocks, which then come from L2 while every
+// other block's loads stream from DRAM -- and their token's RoPE head-rows. Measured: one
+// call at 64 tokens (one wave) 3.80 -> 3.53 us per layer step with the rows (4.02 -> 3.78 us
+// in a timeline probe with the head-rows too), at 128 tokens (two waves) 6.1 -> 5.8 us;
+// prefetching every block's own lines there was slower (4.26 -> 4.68 us at 64 tokens).
+// Whole-step launches take it only with two norm CTAs per token (one wave): on multi-wave
+// steps it measured 1-2 % slower.
 inline int32_t chain_prefetch_mode(bool pdl, bool small_grid, bool norm_rows) {
   if (!pdl) return 0;
   return small_grid ? 1 : (norm_rows ? 2 : 0);
