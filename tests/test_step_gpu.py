@@ -140,16 +140,20 @@ def test_step_fp16_longer_than_one_chunk(S):
         check_chain(L.layer_chain(inp, cfg["theta"], cfg["eps"], FP16), out, inp, FP16)
 
 
-@pytest.mark.parametrize("entry,T", [("invoke", 64), ("step", 64), ("invoke", 4), ("step", 4)])
-def test_dependent_layers_back_to_back_with_pdl(S, entry, T):
-    """Six Llama layers where layer l+1's residual input is layer l's second residual
-    output, launched back to back with programmatic dependent launch (one invoke each
-    through the fast-call shim, or one invoke_step that must fall back to call-by-call
-    order). Each kernel's memory accesses wait for the previous kernel, so every layer equals
-    the oracle run in sequence. At 4 tokens the grid is small: it is token-major and
-    prefetches its rows into L2 before the wait, while the previous layer still writes them."""
+@pytest.mark.parametrize("entry,T,model", [("invoke", 64, "LLAMA"), ("step", 64, "LLAMA"), ("invoke", 4, "LLAMA"),
+                                           ("step", 4, "LLAMA"), ("invoke", 64, "QWEN3"), ("invoke", 128, "LLAMA"),
+                                           ("invoke", 128, "QWEN3")])
+def test_dependent_layers_back_to_back_with_pdl(S, entry, T, model):
+    """Six layers where layer l+1's residual input is layer l's second residual output,
+    launched back to back with programmatic dependent launch (one invoke each through the
+    fast-call shim, or one invoke_step that must fall back to call-by-call order). Each
+    kernel's memory accesses wait for the previous kernel, so every layer equals the oracle
+    run in sequence. At 4 tokens the grid is small: it is token-major and prefetches its rows
+    into L2 before the wait, while the previous layer still writes them; at 64 and 128 tokens
+    the norm blocks prefetch their rows and their token's RoPE head-rows before the wait (two
+    CTAs per token at 64, one at 128)."""
     import ctypes
-    cfg = synth.LLAMA
+    cfg = getattr(synth, model)
     n = 6
     s, op = step_scm(S, cfg, BF16, S.LAYOUT_ROWSTRIDED)
     inps, outs, args = build_layers(S, cfg, T, n, seed=606)
@@ -172,7 +176,7 @@ def test_dependent_layers_back_to_back_with_pdl(S, entry, T):
     r0 = inps[0]["r0"]
     for l in range(n):
         inp = dict(inps[l], r0=r0)
-        ref = L.layer_chain(inp, cfg["theta"], cfg["eps"], BF16)
+        ref = L.layer_chain(inp, cfg["theta"], cfg["eps"], BF16, qknorm=cfg["qknorm"])
         check_chain(ref, outs[l][1], inp)
         r0 = ref["r2"]
 
