@@ -1114,8 +1114,17 @@ def run_ours(a):
             (1, 8, 32, 128) if not a.quick else (1, 128))
         for T in toks:
             qw[str(T)], _ = bench_layer(c, synth.QWEN3, T, K=max(20, min(K, 2000) // 36), W=W,
-                                        layers=36)
+                                        layers=synth.QWEN3["layers"])
         add_floor_fractions(qw, floor_us)
+        peak, _ = measured_peaks()
+        for T, v in qw.items():  # the steps that are device-bound: HBM fraction of the whole step
+            o = v.get("one_launch_step")
+            if o:
+                b = synth.QWEN3["layers"] * chain_bytes_per_launch(synth.QWEN3, int(T))
+                o["bytes_per_step"] = int(b)
+                o["hbm_frac"] = round(b / o["us"] / 1e3 / peak, 3)
+                if "replayed" in o:
+                    o["replayed"]["hbm_frac"] = round(b / o["replayed"]["us"] / 1e3 / peak, 3)
         extra["qwen3_36layer_step"] = qw
     if rank == 0 and want("host"):
         progress("host dispatch")
