@@ -458,9 +458,13 @@ def check_chain(ref, out, inp, dtype=BF16):
     assert np.array_equal(hb("v_cache"), ref["v_cache"])
 
 
+@pytest.mark.parametrize("pdl", [False, True], ids=["plain", "pdl"])
 @pytest.mark.parametrize("cfg_name,T", [("LLAMA", 1), ("LLAMA", 4), ("LLAMA", 16), ("LLAMA", 64),
                                         ("QWEN3", 1), ("QWEN3", 8), ("QWEN3", 32), ("QWEN3", 128)])
-def test_layer_chain_fused_matches_oracle(S, cfg_name, T):
+def test_layer_chain_fused_matches_oracle(S, cfg_name, T, pdl):
+    """The benchmarked layer configurations, with and without programmatic dependent launch
+    (with it, as bench.py launches: token-major grids prefetch every block's lines, larger ones
+    the norm blocks' rows and their tokens' RoPE head-rows, before the wait)."""
     cfg = getattr(synth, cfg_name)
     g = np.random.default_rng(T)
     inp = synth.layer_inputs(g, T, cfg)
@@ -469,7 +473,8 @@ def test_layer_chain_fused_matches_oracle(S, cfg_name, T):
     op = S.OP_LAYER_CHAIN_QKNORM if qk else S.OP_LAYER_CHAIN
     fixed = [cfg["H"], cfg["Hq"], cfg["Hkv"], cfg["D"], cfg["S"], cfg["I"]]
     lay = S.LAYOUT_ROWSTRIDED if T > 1 else S.LAYOUT_CONTIG
-    s = one_version_scm(S, S.make_spec(op, BF16, fixed, 1, 4096, layout=lay, rope_theta=cfg["theta"]))
+    s = one_version_scm(S, S.make_spec(op, BF16, fixed, 1, 4096, layout=lay, rope_theta=cfg["theta"]),
+                        flags=S.OPT_PDL if pdl else 0)
     ts, out = chain_device(inp, BF16, qk)
     invoke_ok(s, S, S.make_args(op, ts, eps=cfg["eps"], rope_theta=cfg["theta"]))
     torch.cuda.synchronize()
