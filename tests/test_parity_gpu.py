@@ -482,6 +482,26 @@ def test_layer_chain_fused_matches_oracle(S, cfg_name, T, pdl):
     check_chain(ref, out, inp)
 
 
+def test_layer_chain_largest_bucket(S):
+    """The largest token count the benchmark's chain versions accept (4096 Llama tokens: a grid
+    of 32,768 blocks, one CTA per token for the norms, the norm-row and RoPE-row prefetch under
+    PDL), every output against the oracle."""
+    cfg = synth.LLAMA
+    T = 4096
+    g = np.random.default_rng(4096)
+    inp = synth.layer_inputs(g, T, cfg)
+    ref = L.layer_chain(inp, cfg["theta"], cfg["eps"], BF16)
+    fixed = [cfg["H"], cfg["Hq"], cfg["Hkv"], cfg["D"], cfg["S"], cfg["I"]]
+    s = one_version_scm(S, S.make_spec(S.OP_LAYER_CHAIN, BF16, fixed, 1, 4096, layout=S.LAYOUT_ROWSTRIDED,
+                                       rope_theta=cfg["theta"]), flags=S.OPT_PDL)
+    ts, out = chain_device(inp, BF16, False)
+    invoke_ok(s, S, S.make_args(S.OP_LAYER_CHAIN, ts, eps=cfg["eps"], rope_theta=cfg["theta"]))
+    torch.cuda.synchronize()
+    assert S.trident_scm_device_status(s.h, stream())[1] == 0
+    s.close()
+    check_chain(ref, out, inp)
+
+
 @pytest.mark.parametrize("dtype,H,Hq,I,T,qk", [
     (FP16, 4096, 32, 14336, 4, False),     # fp16 chain
     (BF16, 8192, 64, 28672, 3, False),     # H 8192 instantiation (4 vectors per thread)
