@@ -188,8 +188,9 @@ __device__ __forceinline__ void chain_block_tok(const ChainParams& c) {
 template <int DT, int VPT, int SPLIT>
 __device__ __forceinline__ void norm_prefetch(const ChainParams& c, const int64_t row, const int part) {
   constexpr int EB = Act<DT>::BYTES;
+  constexpr int VE = Act<DT>::VE;
   const int tid = threadIdx.x;
-  if ((tid & 7) != 0) return;  // 8 threads x 16 bytes = one line
+  if ((tid & 3) != 0) return;  // a line is 8 threads' 16-byte row vectors, 4 threads' gamma floats
   const uint4* hp = reinterpret_cast<const uint4*>(row_ptr(c.n1.x, row, c.n1.x_rs, EB));
   const uint4* rp = reinterpret_cast<const uint4*>(row_ptr(c.n1.r, row, c.n1.r_rs, EB));
   const uint4* ap = reinterpret_cast<const uint4*>(row_ptr(c.n2.x, row, c.n2.x_rs, EB));
@@ -197,9 +198,13 @@ __device__ __forceinline__ void norm_prefetch(const ChainParams& c, const int64_
   for (int v = 0; v < VPT; ++v) {
     if (v % SPLIT != part) continue;
     const int64_t vi = (int64_t)v * kThreads + tid;
-    prefetch_l2(hp + vi);
-    prefetch_l2(rp + vi);
-    prefetch_l2(ap + vi);
+    if ((tid & 7) == 0) {
+      prefetch_l2(hp + vi);
+      prefetch_l2(rp + vi);
+      prefetch_l2(ap + vi);
+    }
+    prefetch_l2(c.n1.gamma + vi * VE);  // this part's half of both norms' weights
+    prefetch_l2(c.n2.gamma + vi * VE);
   }
 }
 
