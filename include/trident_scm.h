@@ -439,7 +439,13 @@ int32_t trident_scm_set_tree_hook(trident_scm_t* scm, trident_tree_hook hook, vo
 int32_t trident_scm_select(const trident_scm_t* scm, const trident_args* args,
                            int32_t* out_selected);
 
-/* Copies the counters into *out. */
+/* Copies the counters into *out (calls, hits, misses, hook calls and failures, errors,
+ * guard evaluations, fused launches, replayed calls). §4.1 measures a warm path: calls
+ * that stay on the compiled hit path (§3.5: only a miss returns to the compile path),
+ * timed on the host until the call returns and end to end until the device finishes;
+ * these counters show which path each call took, and trident_scm_host_times gives the
+ * host time of the hits. Each counter is read on its own, so counters that concurrent
+ * invokers are updating may be a few calls apart. Errors: ERR_INVALID (scm or out NULL). */
 int32_t trident_scm_stats(const trident_scm_t* scm, trident_scm_stats_t* out);
 
 /* Copies per-version hit counts into out[0..cap-1]; *n (may be NULL) gets the count. */
@@ -483,11 +489,18 @@ int32_t trident_scm_device_status(trident_scm_t* scm, void* stream, uint32_t* ou
  * synchronising the stream. Errors: ERR_INVALID, ERR_CUDA. */
 int32_t trident_rope_kv_noalloc(const trident_args* args, void* stream, uint32_t* out_status);
 
-/* Frees the SCM, its tables and device memory. The caller must ensure no call on it
- * is running and its kernels have finished. NULL is ignored. */
+/* Frees the SCM, its tables and device memory. §3.4: the callable keeps the compiled
+ * engine alive, so everything a version needs stays valid for as long as the callable
+ * exists; here the handle is that callable, and it owns its versions, resolved kernels,
+ * frequency tables and status word until this call ends its lifetime. The caller must
+ * ensure no call on it is running and its kernels have finished. NULL is ignored. */
 void trident_scm_destroy(trident_scm_t* scm);
 
-/* Thread-local message of the last error returned on this thread ("" if none). */
+/* Thread-local message of the last error returned on this thread ("" if none). §3.2 and
+ * §3.4-3.5: an execution error ends dispatch and reaches the caller through the FFI's
+ * error channel, distinct from a miss; the negative status says which kind of error and
+ * this message says what failed. The buffer belongs to the calling thread and is
+ * overwritten by that thread's next failing call. */
 const char* trident_scm_last_error(void);
 
 /* Static name of a status code. */
