@@ -168,6 +168,12 @@ typedef enum trident_variant {
 #define TRIDENT_OPT_FAIL_LAUNCHES 0x10 /* fault injection on the host, for tests: every launch
                                           step of a hit reports ERR_CUDA without launching */
 #define TRIDENT_OPT_NO_STEP_REPLAY 0x20 /* invoke_step never replays a stored chunk */
+#define TRIDENT_OPT_TEST_WAIT_TIMEOUT 0x40 /* for tests of the device-side timeout path: the
+                                          bulk-copy add+RMSNorm kernel gives up its first
+                                          wait for its copies at once (0 polls), so every
+                                          block takes the timeout path -- sets
+                                          TRIDENT_DEVERR_TIMEOUT, drains its copies with the
+                                          full bounded wait and returns without writing */
 
 /* ---------------------------------------------------------------- structs */
 /* Caller-owned tensor descriptor (DLPack-like, §3.4: tensors cross the boundary as
@@ -482,11 +488,14 @@ int32_t trident_scm_device_status(trident_scm_t* scm, void* stream, uint32_t* ou
  * a head size above 256 (more than 128 frequency pairs) is rejected with ERR_INVALID.
  * The first call on a device looks up the array's device address (cudaGetSymbolAddress),
  * so make that first call before any stream capture. Every call shares the array, which
- * keeps the last call's table: the table is rebuilt on the device when (theta, D)
- * changes, and the status word is cleared at the start of each call. Calls that overlap on the GPU (other
- * streams, other host threads) race on the array. *out_status (may be NULL) receives the
- * status word (TRIDENT_DEVERR_* bits) by an asynchronous copy on `stream`: read it after
- * synchronising the stream. Errors: ERR_INVALID, ERR_CUDA. */
+ * keeps the last call's contents: each call first launches, on `stream`, a small kernel
+ * that clears the status word and rewrites the table for the call's own (theta, D), so
+ * nothing depends on what an earlier call left there. Calls that overlap on the GPU
+ * (other streams, other host threads) race on the array. *out_status (may be NULL)
+ * receives the status word (TRIDENT_DEVERR_* bits) by a cudaMemcpyAsync on `stream`
+ * after the RoPE kernel; read it after synchronising the stream. Into page-locked host
+ * memory that copy is asynchronous; into pageable memory it makes the host wait until the
+ * kernel has finished. Errors: ERR_INVALID, ERR_CUDA. */
 int32_t trident_rope_kv_noalloc(const trident_args* args, void* stream, uint32_t* out_status);
 
 /* Frees the SCM, its tables and device memory. §3.4: the callable keeps the compiled

@@ -124,17 +124,17 @@ __global__ void __launch_bounds__(kThreads, 4) addnorm_bulk_kernel(const AddNorm
       g[v][4 * q] = gg.x; g[v][4 * q + 1] = gg.y; g[v][4 * q + 2] = gg.z; g[v][4 * q + 3] = gg.w;
     }
   }
-  auto landed = [&]() -> bool {
+  auto landed = [&](uint32_t polls) -> bool {
     uint32_t done = 0;
-    for (int it = 0; it < (1 << 20) && !done; ++it)
+    for (uint32_t it = 0; it < polls && !done; ++it)
       asm volatile("{ .reg .pred q; mbarrier.try_wait.parity.shared::cta.b64 q, [%1], 0; selp.u32 %0, 1, 0, q; }"
                    : "=r"(done) : "r"(bar_a) : "memory");
     return done != 0;
   };
-  const bool ok = landed();
+  const bool ok = landed(p.first_wait_polls);
   if (__syncthreads_or(!ok)) {  // one decision for the whole block
     if (tid == 0 && p.err) atomicOr(p.err, kErrTimeout);
-    if (!ok) landed();  // a second bounded wait for the copies before the block exits
+    if (!ok) landed(kBulkWaitPolls);  // a second bounded wait for the copies before the block exits
     return;
   }
   uint4* rop = reinterpret_cast<uint4*>(row_ptr(p.r_out, row, p.ro_rs, EB));

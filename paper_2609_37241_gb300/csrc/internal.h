@@ -25,8 +25,14 @@ struct AddNormParams {
   int64_t x_rs, r_rs, y_rs, ro_rs;
   float eps, inv_H;
   int32_t prefetch;  // 1: prefetch this block's first lines into L2 before the PDL wait
+  uint32_t first_wait_polls;  // bulk-copy kernel: polls of its first wait for the copies
+                              // (kBulkWaitPolls; 0 under TRIDENT_OPT_TEST_WAIT_TIMEOUT)
   uint32_t* err;     // device status word (the bulk-copy kernel reports a timed-out wait)
 };
+
+// Bound of every mbarrier wait of the bulk-copy kernel (try_wait polls, each itself bounded
+// by the hardware's suspend time).
+constexpr uint32_t kBulkWaitPolls = 1u << 20;
 
 // RMSNorm over T rows of H elements (no residual). Row strides in elements.
 struct RmsNormParams {

@@ -12,9 +12,11 @@
 // Scratch layout (kScratchBytes = 256 + 1024 bytes, held by every GPU that loads the
 // library until the process exits): bytes [0, 4) the status word, bytes [256, end) the
 // frequency table, (hi, lo) fp32 pairs of theta^(-2i/D) for i < D/2, at most kMaxPairs =
-// 128 pairs (D <= 256). The table is recomputed on the device (fp64, split into two fp32)
-// only when (theta, D) differs from what the array held after the previous call on that
-// device; the status word is cleared at the start of every call.
+// 128 pairs (D <= 256). Every call first launches one small kernel on the caller's stream
+// that clears the status word and rewrites the table for its own (theta, D), then the
+// RoPE kernel. The host keeps no record of what the array holds, so nothing on the host
+// can disagree with the device: whatever ran on the stream before, and whether or not an
+// earlier launch failed, the RoPE kernel reads the table its own call wrote.
 #include <cuda_runtime.h>
 
 #include <cmath>
@@ -37,23 +39,20 @@ struct DeviceScratch {
   std::once_flag once;
   cudaError_t setup_error = cudaSuccess;
   unsigned char* addr = nullptr;  // device address of g_scratch on this device
-  std::mutex mu;                  // guards the table key below
-  double theta = 0.0;
-  int32_t D = 0;
 };
 DeviceScratch g_dev[kMaxDevices];
 
-// Fills the frequency table: f_i = theta^(-2i/D) in fp64, stored as (fp32(f), fp32(f - hi)).
-__global__ void fill_inv_freq(float2* tab, int32_t D, double theta) {
+// Prepares the scratch for one call: clears the status word and writes the frequency
+// table f_i = theta^(-2i/D) in fp64, stored as (fp32(f), fp32(f - hi)), for i < D/2.
+__global__ void prepare_scratch(uint32_t* status, float2* tab, int32_t D, double theta) {
   const int i = threadIdx.x;
+  if (i == 0) *status = 0u;
   if (i < D / 2) {
     const double f = pow(theta, -2.0 * (double)i / (double)D);
     const float hi = (float)f;
     tab[i] = make_float2(hi, (float)(f - (double)hi));
   }
 }
-
-__global__ void clear_word(uint32_t* w) { *w = 0u; }
 
 }  // namespace
 }  // namespace trident
@@ -93,15 +92,9 @@ extern "C" __attribute__((visibility("default"))) int32_t trident_rope_kv_noallo
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   uint32_t* status = reinterpret_cast<uint32_t*>(ds.addr);
   float2* table = reinterpret_cast<float2*>(ds.addr + kTableOffset);
-  {
-    std::lock_guard<std::mutex> lk(ds.mu);
-    clear_word<<<1, 1, 0, s>>>(status);
-    if (!(ds.theta == args->rope_theta && ds.D == p.D)) {
-      fill_inv_freq<<<1, (unsigned)kMaxPairs, 0, s>>>(table, p.D, args->rope_theta);
-      ds.theta = args->rope_theta;
-      ds.D = p.D;
-    }
-  }
+  prepare_scratch<<<1, (unsigned)kMaxPairs, 0, s>>>(status, table, p.D, args->rope_theta);
+  if (cudaGetLastError() != cudaSuccess)
+    return internal_fail(TRIDENT_ERR_CUDA, "scratch preparation launch failed");
   p.inv_freq = table;
   p.err = status;
   const int64_t upb = rope_units_per_block(p.D, 2);

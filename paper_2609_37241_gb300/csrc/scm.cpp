@@ -554,6 +554,7 @@ void pack_addnorm(const trident_args* a, int x, int r, int g, int y, int ro, con
   p->eps = (float)a->eps;
   p->inv_H = (float)(1.0 / (double)p->H);
   p->prefetch = 0;
+  p->first_wait_polls = kBulkWaitPolls;
   p->err = nullptr;
 }
 
@@ -726,6 +727,7 @@ int32_t do_launch(trident_scm* scm, const Version& v, const trident_args* a, con
     case TRIDENT_OP_ADD_RMSNORM:
       pack_addnorm(a, 0, 1, 2, 3, 4, s, K_ACT_H, &P.an);
       P.an.err = scm->d_err;
+      if (scm->opt.flags & TRIDENT_OPT_TEST_WAIT_TIMEOUT) P.an.first_wait_polls = 0;
       cfg.gridDimX = cap_grid(s.T);
       break;
     case TRIDENT_OP_RMSNORM:
@@ -1124,7 +1126,7 @@ TRIDENT_API int32_t trident_scm_create(const trident_scm_options* opt, trident_c
   if (o.timing_ring == 0) o.timing_ring = 65536;
   if (o.timing_ring < 1 || o.timing_ring > (1 << 24)) return fail(TRIDENT_ERR_INVALID, "timing_ring");
   if (o.flags & ~(TRIDENT_OPT_DRY_RUN | TRIDENT_OPT_NO_ALIAS_CHECK | TRIDENT_OPT_PDL | TRIDENT_OPT_TIMING |
-                  TRIDENT_OPT_FAIL_LAUNCHES | TRIDENT_OPT_NO_STEP_REPLAY))
+                  TRIDENT_OPT_FAIL_LAUNCHES | TRIDENT_OPT_NO_STEP_REPLAY | TRIDENT_OPT_TEST_WAIT_TIMEOUT))
     return fail(TRIDENT_ERR_INVALID, "unknown option flags");
   if (o.device < 0) return fail(TRIDENT_ERR_INVALID, "device");
   trident_scm* s = new (std::nothrow) trident_scm();

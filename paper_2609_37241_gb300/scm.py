@@ -23,6 +23,7 @@ LAYOUT_CONTIG, LAYOUT_ROWSTRIDED, LAYOUT_ANY = 0, 1, 2
 VARIANT_AUTO, VARIANT_GENERIC, VARIANT_VECTOR = 0, 1, 2
 OPT_DRY_RUN, OPT_NO_ALIAS_CHECK, OPT_PDL, OPT_TIMING, OPT_FAIL_LAUNCHES = 0x1, 0x2, 0x4, 0x8, 0x10
 OPT_NO_STEP_REPLAY = 0x20
+OPT_TEST_WAIT_TIMEOUT = 0x40
 DEVERR_POS, DEVERR_TIMEOUT = 0x1, 0x2
 MAX_TENSORS, MAX_FIXED = 20, 8
 STEP_MAX = 48  # calls per launch of trident_scm_invoke_step
@@ -237,12 +238,13 @@ def trident_launch_floor(scm, stream=None, n=1):
     return lib().trident_launch_floor(scm, stream, n)
 
 
-def trident_rope_kv_noalloc(args, stream=None):
-    """RoPE + KV append with no allocation (static scratch). Returns (status, status_word);
-    the status word is valid once the stream has been synchronised."""
-    word = c_u32(0)
-    st = lib().trident_rope_kv_noalloc(ctypes.byref(args), stream, ctypes.byref(word))
-    return st, word
+def trident_rope_kv_noalloc(args, stream=None, status_word=None):
+    """RoPE + KV append with no allocation (static scratch). Returns the status code.
+    status_word: None (the device status word is not copied out), or the address of a
+    4-byte host word -- page-locked for the copy to stay asynchronous -- that receives the
+    TRIDENT_DEVERR_* bits once the stream has been synchronised."""
+    out = None if status_word is None else ctypes.cast(ctypes.c_void_p(status_word), ctypes.POINTER(c_u32))
+    return lib().trident_rope_kv_noalloc(ctypes.byref(args), stream, out)
 
 
 def trident_scm_destroy(scm):

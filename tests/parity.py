@@ -83,3 +83,24 @@ def padded(bits, dtype, pad, device="cuda"):
     view = buf[:, :W]
     view.copy_(dev(bits, dtype, device))
     return view
+
+
+def check_rope(ref, got, inputs, dtype=BF16):
+    """RoPE + KV append against the oracle (`oracle.layer.rope_kv` output `ref`): q and the
+    written k-cache rows within tolerance, tokens with a position outside the cache left
+    untouched, every other cache slot still the sentinel, the v cache a bit copy, and the
+    k / v inputs unchanged. got: host bit arrays q, k_cache, v_cache, k, v."""
+    q, k, v, pos = inputs
+    valid = (pos >= 0) & (pos < ref["k_cache"].shape[1])
+    check_act(got["q"][valid], ref["q_ref"][valid], ref["q"][valid], dtype, "q", exact_frac=0.99)
+    assert np.array_equal(got["q"][~valid], q[~valid])  # skipped tokens untouched
+    # k cache: rotated rows at the valid positions, sentinel (bit-exact) everywhere else
+    kc_ref_rows = ref["k_cache"][:, pos[valid], :]
+    kc_got_rows = got["k_cache"][:, pos[valid], :]
+    check_act(kc_got_rows.transpose(1, 0, 2), ref["k_ref"][valid], kc_ref_rows.transpose(1, 0, 2),
+              dtype, "k_cache", exact_frac=0.99)
+    written = np.zeros(ref["k_cache"].shape[1], bool)
+    written[pos[valid]] = True
+    assert np.all(got["k_cache"][:, ~written, :] == synth.CACHE_SENTINEL)
+    assert np.array_equal(got["v_cache"], ref["v_cache"])  # bit copy + sentinel
+    assert np.array_equal(got["k"], k) and np.array_equal(got["v"], v)  # inputs unchanged
