@@ -131,12 +131,19 @@ __device__ __forceinline__ void chain_norm(const ChainParams& c, const int64_t r
   }
 }
 
-// RoPE role: RoPE block rb (< nB), i.e. head-rows [rb * UPB, (rb + 1) * UPB).
+// RoPE role: RoPE block rb (< nB), i.e. head-rows [rb * UPB, (rb + 1) * UPB); fq holds the
+// lane's frequencies, loaded before the PDL wait (rope_lane_freqs).
 template <int DT, int D, bool QKNORM>
-__device__ __forceinline__ void chain_rope(const ChainParams& c, const int64_t rb) {
+__device__ __forceinline__ void chain_rope(const ChainParams& c, const int64_t rb, const float* fq) {
   constexpr int LPH = D / Act<DT>::VE;
   const int64_t unit = rb * (kThreads / LPH) + threadIdx.x / LPH;
-  if (unit < c.rope.T * c.rope.NH) rope_head_row<DT, D, QKNORM>(c.rope, unit, threadIdx.x % LPH);
+  if (unit < c.rope.T * c.rope.NH) rope_head_row<DT, D, QKNORM>(c.rope, unit, threadIdx.x % LPH, fq);
+}
+
+// Before the PDL wait: the RoPE lane frequencies of a RoPE block (other roles load none).
+template <int DT, int D>
+__device__ __forceinline__ void chain_rope_freqs(const ChainParams& c, const bool is_rope, float* fq) {
+  if (is_rope) rope_lane_freqs<DT, D>(c.rope.inv_freq, threadIdx.x % (D / Act<DT>::VE), fq);
 }
 
 // SwiGLU role: column tile `col_tile` of row `row`, SWU x 256 16-byte vectors of g and of u
@@ -148,12 +155,12 @@ __device__ __forceinline__ void chain_swiglu(const ChainParams& c, const int64_t
 
 // Block b of one call's role-major grid (b < nA + nB + nC): [norms | RoPE | SwiGLU].
 template <int DT, int VPT, int SPLIT, int D, bool QKNORM, int SWU>
-__device__ __forceinline__ void chain_block(const ChainParams& c, const int b) {
+__device__ __forceinline__ void chain_block(const ChainParams& c, const int b, const float* fq) {
   if (b < c.nA) {
     const int64_t row = b / SPLIT;
     chain_norm<DT, VPT, SPLIT>(c, row, b - (int)row * SPLIT);
   } else if (b < c.nA + c.nB) {
-    chain_rope<DT, D, QKNORM>(c, b - c.nA);
+    chain_rope<DT, D, QKNORM>(c, b - c.nA, fq);
   } else {
     const int64_t tile = b - c.nA - c.nB;
     if (tile >= c.sw_tiles) return;
@@ -170,12 +177,12 @@ __device__ __forceinline__ void chain_block(const ChainParams& c, const int b) {
 // give one SM four norm blocks (160 KB) while another gets 24 KB. Both indices come from
 // special registers, so no remapped index stays live in a register through the body.
 template <int DT, int VPT, int SPLIT, int D, bool QKNORM>
-__device__ __forceinline__ void chain_block_tok(const ChainParams& c) {
+__device__ __forceinline__ void chain_block_tok(const ChainParams& c, const float* fq) {
   const int q = blockIdx.x;
   if (q < SPLIT) {
     chain_norm<DT, VPT, SPLIT>(c, blockIdx.y, q);
   } else if (q < SPLIT + c.rope_per_tok) {
-    chain_rope<DT, D, QKNORM>(c, (int64_t)blockIdx.y * c.rope_per_tok + (q - SPLIT));
+    chain_rope<DT, D, QKNORM>(c, (int64_t)blockIdx.y * c.rope_per_tok + (q - SPLIT), fq);
   } else {
     chain_swiglu<DT, kChainSwigluUnroll>(c, blockIdx.y, q - SPLIT - c.rope_per_tok);
   }
@@ -265,14 +272,20 @@ template <int DT, int VPT, int SPLIT, int D, bool QKNORM>
 __global__ void __launch_bounds__(kThreads, VPT == 2 ? 4 : 2)
     chain_kernel(const __grid_constant__ ChainParams c) {
   pdl_trigger();
+  float fq[2 * Act<DT>::VE];
   if (c.tok_grid) {
     if (c.prefetch) chain_prefetch_tok<DT, VPT, SPLIT, D>(c);
+    chain_rope_freqs<DT, D>(c, (int)blockIdx.x >= SPLIT && (int)blockIdx.x < SPLIT + c.rope_per_tok, fq);
     pdl_wait();
-    chain_block_tok<DT, VPT, SPLIT, D, QKNORM>(c);
+    chain_block_tok<DT, VPT, SPLIT, D, QKNORM>(c, fq);
   } else {
-    if (c.prefetch) chain_prefetch<DT, VPT, SPLIT, D, kChainSwigluUnroll>(c, blockIdx.x);
+    // A role-major grid fills the GPU: its RoPE blocks become resident only as the previous
+    // kernel's blocks retire, and their frequency loads measured faster after the wait.
+    const int b = blockIdx.x;
+    if (c.prefetch) chain_prefetch<DT, VPT, SPLIT, D, kChainSwigluUnroll>(c, b);
     pdl_wait();
-    chain_block<DT, VPT, SPLIT, D, QKNORM, kChainSwigluUnroll>(c, blockIdx.x);
+    chain_rope_freqs<DT, D>(c, b >= c.nA && b < c.nA + c.nB, fq);
+    chain_block<DT, VPT, SPLIT, D, QKNORM, kChainSwigluUnroll>(c, b, fq);
   }
 }
 
@@ -289,9 +302,13 @@ __global__ void __launch_bounds__(kThreads, VPT == 2 ? 4 : 2)
     if (b >= p.first[mid]) lo = mid;
     else hi = mid - 1;
   }
-  if (p.c[lo].prefetch) chain_prefetch<DT, VPT, SPLIT, D, kChainStepSwigluUnroll>(p.c[lo], b - p.first[lo]);
+  const ChainParams& c = p.c[lo];
+  const int bl = b - p.first[lo];
+  if (c.prefetch) chain_prefetch<DT, VPT, SPLIT, D, kChainStepSwigluUnroll>(c, bl);
+  float fq[2 * Act<DT>::VE];
+  chain_rope_freqs<DT, D>(c, bl >= c.nA && bl < c.nA + c.nB, fq);
   pdl_wait();
-  chain_block<DT, VPT, SPLIT, D, QKNORM, kChainStepSwigluUnroll>(p.c[lo], b - p.first[lo]);
+  chain_block<DT, VPT, SPLIT, D, QKNORM, kChainStepSwigluUnroll>(c, bl, fq);
 }
 
 template <int DT, int SPLIT, bool QK>

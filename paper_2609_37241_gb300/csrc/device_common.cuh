@@ -195,14 +195,71 @@ __device__ __forceinline__ void rope_prefetch(const RopeParams& p, int64_t unit,
   if (lane == 0) prefetch_l2(p.pos + t);
 }
 
+// The (hi, lo) frequencies of lane `lane` of a head-row, for its VE elements
+// i = (lane % (LPH/2)) * VE + e. The frequency table belongs to the version: it is written
+// once, when the version is registered (and the registration waits for that copy), and is
+// never written again, so kernels read it before griddepcontrol.wait, while the previous
+// kernel of the stream still runs. Every RoPE lane of a grid reads the same few lines of
+// the table; read after the wait, those reads queue behind each other at the L2 slices
+// that hold the lines, on the critical path of every RoPE block. The same lane position
+// has the same frequencies in every head-row, so a lane loads them once.
+template <int DT, int D>
+__device__ __forceinline__ void rope_lane_freqs(const float2* inv_freq, int lane, float* fq) {
+  constexpr int VE = Act<DT>::VE;
+  constexpr int HALF = D / VE / 2;
+  const float* fr = reinterpret_cast<const float*>(inv_freq) + 2 * (lane % HALF) * VE;
+#pragma unroll
+  for (int q = 0; q < VE / 2; ++q) {
+    const float4 f4 = ldg_f4(fr + 4 * q);
+    fq[4 * q] = f4.x; fq[4 * q + 1] = f4.y; fq[4 * q + 2] = f4.z; fq[4 * q + 3] = f4.w;
+  }
+}
+
 // One head-row (token t, head hh) handled by LPH = D / VE consecutive lanes, each lane
 // owning VE consecutive elements. Rotate-half pairs element i with i + D/2, i.e. lane
 // l with lane l ^ (LPH/2). hh < Hq: q head (rotated in place); hh < Hq + Hkv: k head
-// (rotated into k_cache); else v head (copied into v_cache). Every load -- the row, the
-// position, the lane's frequencies and norm weights -- is issued before any of them is
-// used, so a head-row costs one memory round trip.
+// (rotated into k_cache); else v head (copied into v_cache). fq holds the lane's
+// frequencies (rope_lane_freqs). A head-row is processed in two steps: rope_row_load issues
+// every load it needs -- the row slice, the position and the norm weights -- and
+// rope_row_finish uses them, so a lane group that owns several head-rows issues all of
+// their loads before it waits for any (one memory round trip in all).
+template <int DT, int D>
+__device__ __forceinline__ void rope_row_where(const RopeParams& p, int64_t unit, int64_t* t, int* h,
+                                               bool* is_q, bool* is_v) {
+  *t = unit / p.NH;
+  const int hh = (int)(unit - *t * p.NH);
+  *is_v = hh >= p.Hq + p.Hkv;
+  *is_q = hh < p.Hq;
+  *h = *is_q ? hh : (*is_v ? hh - p.Hq - p.Hkv : hh - p.Hq);
+}
+
 template <int DT, int D, bool QKNORM>
-__device__ __forceinline__ void rope_head_row(const RopeParams& p, int64_t unit, int lane) {
+__device__ __forceinline__ void rope_row_load(const RopeParams& p, int64_t unit, int lane, uint4* raw,
+                                              int32_t* pos, float* gg) {
+  constexpr int VE = Act<DT>::VE;
+  constexpr int EB = Act<DT>::BYTES;
+  int64_t t;
+  int h;
+  bool is_q, is_v;
+  rope_row_where<DT, D>(p, unit, &t, &h, &is_q, &is_v);
+  const char* src = is_q ? row_ptr(p.q, t, p.q_rs, EB) : is_v ? row_ptr(p.v, t, p.v_rs, EB)
+                                                             : row_ptr(p.k, t, p.k_rs, EB);
+  src += ((int64_t)h * D + lane * VE) * EB;
+  *raw = is_q ? ld16(src) : ldg16(src);
+  *pos = __ldg(p.pos + t);
+  if (QKNORM && !is_v) {
+    const float* gam = (is_q ? p.gamma_q : p.gamma_k) + lane * VE;
+#pragma unroll
+    for (int q = 0; q < VE / 4; ++q) {
+      const float4 g4 = ldg_f4(gam + 4 * q);
+      gg[4 * q] = g4.x; gg[4 * q + 1] = g4.y; gg[4 * q + 2] = g4.z; gg[4 * q + 3] = g4.w;
+    }
+  }
+}
+
+template <int DT, int D, bool QKNORM>
+__device__ __forceinline__ void rope_row_finish(const RopeParams& p, int64_t unit, int lane, const uint4 raw,
+                                                const int32_t pos, const float* gg, const float* fq) {
   constexpr int VE = Act<DT>::VE;
   constexpr int LPH = D / VE;
   constexpr int HALF = LPH / 2;
@@ -210,35 +267,10 @@ __device__ __forceinline__ void rope_head_row(const RopeParams& p, int64_t unit,
   static_assert(LPH >= 2 && LPH <= 32 && (LPH & (LPH - 1)) == 0, "head size");
   const unsigned group_mask =
       (LPH == 32) ? 0xffffffffu : (((1u << LPH) - 1u) << ((threadIdx.x & 31) & ~(LPH - 1)));
-
-  const int64_t t = unit / p.NH;
-  const int hh = (int)(unit - t * p.NH);
-  const bool is_v = hh >= p.Hq + p.Hkv;
-  const bool is_q = hh < p.Hq;
-  const int h = is_q ? hh : (is_v ? hh - p.Hq - p.Hkv : hh - p.Hq);
-  const char* src = is_q ? row_ptr(p.q, t, p.q_rs, EB) : is_v ? row_ptr(p.v, t, p.v_rs, EB)
-                                                             : row_ptr(p.k, t, p.k_rs, EB);
-  src += ((int64_t)h * D + lane * VE) * EB;
-  const uint4 raw = is_q ? ld16(src) : ldg16(src);
-  const int32_t pos = __ldg(p.pos + t);
-  float fq[2 * VE];  // (hi, lo) of the lane's VE frequencies i = (lane % HALF) * VE + e
-  float gg[VE];
-  if (!is_v) {
-    const float* fr = reinterpret_cast<const float*>(p.inv_freq) + 2 * (lane % HALF) * VE;
-#pragma unroll
-    for (int q = 0; q < VE / 2; ++q) {
-      const float4 f4 = ldg_f4(fr + 4 * q);
-      fq[4 * q] = f4.x; fq[4 * q + 1] = f4.y; fq[4 * q + 2] = f4.z; fq[4 * q + 3] = f4.w;
-    }
-    if (QKNORM) {
-      const float* gam = (is_q ? p.gamma_q : p.gamma_k) + lane * VE;
-#pragma unroll
-      for (int q = 0; q < VE / 4; ++q) {
-        const float4 g4 = ldg_f4(gam + 4 * q);
-        gg[4 * q] = g4.x; gg[4 * q + 1] = g4.y; gg[4 * q + 2] = g4.z; gg[4 * q + 3] = g4.w;
-      }
-    }
-  }
+  int64_t t;
+  int h;
+  bool is_q, is_v;
+  rope_row_where<DT, D>(p, unit, &t, &h, &is_q, &is_v);
   if (pos < 0 || (int64_t)pos >= p.S) {
     if (lane == 0) atomicOr(p.err, kErrPos);
     return;
@@ -278,6 +310,15 @@ __device__ __forceinline__ void rope_head_row(const RopeParams& p, int64_t unit,
     char* dst = reinterpret_cast<char*>(p.k_cache) + (((int64_t)h * p.S + pos) * D + lane * VE) * EB;
     st16(dst, pack<DT>(y));
   }
+}
+
+template <int DT, int D, bool QKNORM>
+__device__ __forceinline__ void rope_head_row(const RopeParams& p, int64_t unit, int lane, const float* fq) {
+  uint4 raw;
+  int32_t pos;
+  float gg[Act<DT>::VE];
+  rope_row_load<DT, D, QKNORM>(p, unit, lane, &raw, &pos, gg);
+  rope_row_finish<DT, D, QKNORM>(p, unit, lane, raw, pos, gg, fq);
 }
 
 // ---------------------------------------------------------------- SwiGLU tile

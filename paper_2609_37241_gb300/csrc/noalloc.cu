@@ -16,7 +16,9 @@
 // that clears the status word and rewrites the table for its own (theta, D), then the
 // RoPE kernel. The host keeps no record of what the array holds, so nothing on the host
 // can disagree with the device: whatever ran on the stream before, and whether or not an
-// earlier launch failed, the RoPE kernel reads the table its own call wrote.
+// earlier launch failed, the RoPE kernel reads the table its own call wrote. The RoPE
+// kernel reads its frequencies before griddepcontrol.wait; it is launched here without
+// programmatic serialisation, so it starts only after the preparing kernel has finished.
 #include <cuda_runtime.h>
 
 #include <cmath>

@@ -19,10 +19,12 @@ __global__ void __launch_bounds__(kThreads) rope_vec_kernel(const RopeParams p) 
   const int64_t total = p.T * p.NH;
   const int lane = threadIdx.x % LPH;
   if (p.prefetch) rope_prefetch<DT, D>(p, (int64_t)blockIdx.x * UPB + threadIdx.x / LPH, lane);
+  float fq[2 * Act<DT>::VE];
+  rope_lane_freqs<DT, D>(p.inv_freq, lane, fq);  // the version's table: readable before the wait
   pdl_wait();
   for (int64_t unit = (int64_t)blockIdx.x * UPB + threadIdx.x / LPH; unit < total;
        unit += (int64_t)gridDim.x * UPB) {
-    rope_head_row<DT, D, QKNORM>(p, unit, lane);
+    rope_head_row<DT, D, QKNORM>(p, unit, lane, fq);
   }
 }
 

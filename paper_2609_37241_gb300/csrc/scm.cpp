@@ -778,13 +778,16 @@ int32_t do_launch(trident_scm* scm, const Version& v, const trident_args* a, con
       st = set_chain_split(&c, s.T, split, &blocks);
       if (st != TRIDENT_OK) return st;
       cfg.gridDimX = (unsigned)blocks;
-      // Token-major grid (chain_block_tok) for grids of at most one block per SM, when every
-      // token has the same number of RoPE blocks: consecutive blocks then mix roles (measured:
-      // 16 tokens 3.55 -> 2.85 us per layer step, 1 token 2.20 -> 2.04 us). A grid that fills
-      // the GPU keeps the role-major order, which starts the longest (norm) blocks first
-      // (64 tokens: 3.98 us role-major, 4.05 us token-major).
+      // Token-major grid (chain_block_tok) for grids of at most two blocks per SM, when every
+      // token has the same number of RoPE blocks: consecutive blocks then mix roles, so the
+      // blocks that land together on one SM are not all norm blocks (measured: 16 tokens
+      // 3.55 -> 2.85 us per layer step, 1 token 2.20 -> 2.04 us; 32 tokens, 288 blocks, 36
+      // Qwen3-style layers 131.5 -> 109.6 us). A grid that nearly fills the GPU keeps the
+      // role-major order, which starts the longest (norm) blocks first (64 tokens: 3.98 us
+      // role-major, 4.05 us token-major; 48 and 64 tokens in other interleaved orders were
+      // slower as well).
       const int64_t upb = rope_units_per_block(c.rope.D, 2);
-      if (c.rope.NH % upb == 0 && s.T >= 1 && s.T <= 65535 && blocks <= scm->sm_count) {
+      if (c.rope.NH % upb == 0 && s.T >= 1 && s.T <= 65535 && blocks <= 2 * scm->sm_count) {
         c.tok_grid = 1;
         c.rope_per_tok = (int32_t)(c.rope.NH / upb);
         cfg.gridDimX = (unsigned)(split + c.rope_per_tok + c.sw_tiles_per_row);
@@ -983,7 +986,11 @@ int32_t get_rope_table(trident_scm* scm, double theta, int32_t D, const float2**
   float2* dev = nullptr;
   if (cudaMalloc(&dev, host.size() * sizeof(float2)) != cudaSuccess)
     return fail(TRIDENT_ERR_CUDA, "cudaMalloc of the RoPE frequency table failed");
-  if (cudaMemcpy(dev, host.data(), host.size() * sizeof(float2), cudaMemcpyHostToDevice) != cudaSuccess) {
+  // The copy must have landed before this registration returns: kernels read the table
+  // before their programmatic-launch wait, on any stream (a pageable-memory copy may return
+  // while its DMA is still in flight, hence the synchronisation).
+  if (cudaMemcpy(dev, host.data(), host.size() * sizeof(float2), cudaMemcpyHostToDevice) != cudaSuccess ||
+      cudaDeviceSynchronize() != cudaSuccess) {
     cudaFree(dev);
     return fail(TRIDENT_ERR_CUDA, "upload of the RoPE frequency table failed");
   }
