@@ -15,13 +15,30 @@ from . import build_oracle
 BF16, FP16, FP32 = 1, 2, 3
 
 _lib = None
+_parallel = False
+
+
+def set_parallel(parallel):
+    """Use the OpenMP build of the C oracle (all host cores; same values) from now on, or
+    the serial default again. For timing the oracle only."""
+    global _lib, _parallel
+    if bool(parallel) != _parallel:
+        _parallel = bool(parallel)
+        _lib = None
+
+
+def threads():
+    """Threads the C oracle's loops run on (1 for the serial build)."""
+    return int(lib().orc_threads())
 
 
 def lib():
     global _lib
     if _lib is None:
-        path = build_oracle.build()
+        path = build_oracle.build(parallel=_parallel)
         L = ctypes.CDLL(path)
+        L.orc_threads.restype = ctypes.c_int
+        L.orc_threads.argtypes = []
         P = ctypes.c_void_p
         i64, c_int, dbl = ctypes.c_int64, ctypes.c_int, ctypes.c_double
         L.orc_widen.restype = dbl

@@ -24,10 +24,27 @@
  * once, round-to-nearest-even, to the activation dtype (bit patterns).
  * Activations are raw bit patterns: uint16 for bf16/fp16, uint32 for fp32.
  * Build with -ffp-contract=off so that no multiply-add is fused behind our back.
+ *
+ * The token (or element) loops carry an OpenMP work-sharing pragma. The default build has
+ * no -fopenmp, so the pragmas are ignored and every loop runs serially in order; a second
+ * build with -fopenmp (liboracle_omp.so) exists only to time the oracle on all host cores.
+ * Every iteration writes its own outputs, so both builds compute the same values.
  */
 #include <math.h>
 #include <stdint.h>
 #include <string.h>
+#ifdef _OPENMP
+#include <omp.h>
+#endif
+
+/* Threads the work-sharing loops use (1 in the default build). */
+int orc_threads(void) {
+#ifdef _OPENMP
+  return omp_get_max_threads();
+#else
+  return 1;
+#endif
+}
 
 enum { OR_BF16 = 1, OR_FP16 = 2, OR_FP32 = 3 };
 
@@ -137,6 +154,7 @@ static void store_act(void* p, int64_t i, int dtype, uint32_t bits) {
 void orc_add_rmsnorm(int64_t T, int64_t H, int dtype, const void* x, const void* r,
                      const float* gamma, double eps, double* y_ref, void* y_bits,
                      void* r_out_bits) {
+#pragma omp parallel for schedule(static)
   for (int64_t t = 0; t < T; ++t) {
     double sumsq = 0.0;
     for (int64_t j = 0; j < H; ++j) {
@@ -160,6 +178,7 @@ void orc_add_rmsnorm(int64_t T, int64_t H, int dtype, const void* x, const void*
  * y = x / sqrt(mean(x^2) + eps) * gamma, in fp64. */
 void orc_rmsnorm(int64_t T, int64_t H, int dtype, const void* x, const float* gamma, double eps,
                  double* y_ref, void* y_bits) {
+#pragma omp parallel for schedule(static)
   for (int64_t t = 0; t < T; ++t) {
     double sumsq = 0.0;
     for (int64_t j = 0; j < H; ++j) {
@@ -208,9 +227,11 @@ int orc_rope_kv(int64_t T, int64_t Hq, int64_t Hkv, int64_t D, int64_t S, int dt
                 double eps, void* q, double* q_ref, const void* k, const void* v,
                 const int32_t* pos, void* k_cache, void* v_cache, double* k_ref) {
   int bad = 0;
-  double buf[1024];
   if (D > 1024) return -1;
+  /* positions are distinct within a call, so tokens write disjoint cache rows */
+#pragma omp parallel for schedule(static) reduction(| : bad)
   for (int64_t t = 0; t < T; ++t) {
+    double buf[1024];
     int64_t p = pos[t];
     if (p < 0 || p >= S) {
       bad = 1;
@@ -298,6 +319,7 @@ void orc_masked_fill(int64_t n, int dtype, const void* x, const uint8_t* mask, d
  * g, u, out_bits: n contiguous elements; ref: n unrounded results. */
 void orc_swiglu(int64_t n, int dtype, const void* g, const void* u, double* ref,
                 void* out_bits) {
+#pragma omp parallel for schedule(static)
   for (int64_t i = 0; i < n; ++i) {
     double gv = load_act(g, i, dtype);
     double uv = load_act(u, i, dtype);

@@ -482,3 +482,24 @@ def test_bucket_definition():
     for b in range(10):
         lo, hi = G.bucket_range(b)
         assert all(G.bucket_of(t) == b for t in range(lo, hi + 1))
+
+
+def test_parallel_oracle_build_matches_serial():
+    """The OpenMP build of the C oracle (used only to time it on all host cores) computes
+    exactly the serial build's values: every loop iteration writes its own outputs."""
+    cfg = dict(synth.LLAMA)
+    cfg.update(H=256, Hq=4, Hkv=2, D=64, S=64, I=320)
+    inp = synth.layer_inputs(np.random.default_rng(5), 7, cfg)
+    inp["pos"][3] = cfg["S"]  # one bad position: the reduction of the flag
+    serial = L.layer_chain(inp, cfg["theta"], cfg["eps"], synth.BF16)
+    try:
+        L.set_parallel(True)
+        par = L.layer_chain(inp, cfg["theta"], cfg["eps"], synth.BF16)
+        assert L.threads() >= 1
+    finally:
+        L.set_parallel(False)
+    assert serial.keys() == par.keys()
+    for k in serial:
+        a, b = np.atleast_1d(np.asarray(serial[k])), np.atleast_1d(np.asarray(par[k]))
+        assert a.dtype == b.dtype and a.shape == b.shape, k
+        assert np.array_equal(a.view(np.uint8), b.view(np.uint8)), k  # bitwise (NaN included)
