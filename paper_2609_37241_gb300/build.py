@@ -87,5 +87,7 @@ def build_fastcall(force=False, verbose=False):
 
 
 if __name__ == "__main__":
-    print(build(force="--force" in sys.argv, verbose=True,
-                extra_flags=["-Xptxas", "-v"] if "--ptxas" in sys.argv else []))
+    flags = (["-Xptxas", "-v"] if "--ptxas" in sys.argv else []) + (["-DTRIDENT_NVTX"] if "--nvtx" in sys.argv else [])
+    # --nvtx: NVTX ranges around the boundary calls (off by default); rebuild without it to
+    # remove them again (--force)
+    print(build(force="--force" in sys.argv or "--nvtx" in sys.argv, verbose=True, extra_flags=flags))

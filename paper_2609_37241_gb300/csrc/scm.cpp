@@ -41,6 +41,21 @@
 
 #define TRIDENT_API extern "C" __attribute__((visibility("default")))
 
+// NVTX ranges around the boundary calls, for profilers' timelines. Compiled in only with
+// -DTRIDENT_NVTX (build.py --nvtx); off by default, the calls then contain no trace of them.
+#ifdef TRIDENT_NVTX
+#include <nvtx3/nvToolsExt.h>
+namespace {
+struct NvtxRange {
+  explicit NvtxRange(const char* name) { nvtxRangePushA(name); }
+  ~NvtxRange() { nvtxRangePop(); }
+};
+}  // namespace
+#define TRIDENT_RANGE(name) NvtxRange trident_nvtx_range_(name)
+#else
+#define TRIDENT_RANGE(name) ((void)0)
+#endif
+
 using namespace trident;
 
 namespace {
@@ -1345,6 +1360,7 @@ int32_t run_miss(trident_scm* scm, bool have_hook, Hook call_hook, int32_t* out_
 
 TRIDENT_API int32_t trident_scm_invoke(trident_scm_t* scm, const trident_args* args, void* stream,
                                        int32_t* out_selected) {
+  TRIDENT_RANGE("trident_scm_invoke");
   if (out_selected) *out_selected = -1;
   if (!scm) return fail(TRIDENT_ERR_INVALID, "scm is NULL");
   const uint64_t t0 = scm->ring ? now_ns() : 0;
@@ -1362,6 +1378,7 @@ TRIDENT_API int32_t trident_scm_invoke(trident_scm_t* scm, const trident_args* a
 
 TRIDENT_API int32_t trident_scm_invoke_tree(trident_scm_t* scm, const trident_node* nodes, int32_t nargs,
                                             int32_t nnodes, void* stream, int32_t* out_selected) {
+  TRIDENT_RANGE("trident_scm_invoke_tree");
   if (out_selected) *out_selected = -1;
   if (!scm) return fail(TRIDENT_ERR_INVALID, "scm is NULL");
   const uint64_t t0 = scm->ring ? now_ns() : 0;
@@ -1400,6 +1417,7 @@ TRIDENT_API int32_t trident_scm_set_tree_hook(trident_scm_t* scm, trident_tree_h
 
 TRIDENT_API int32_t trident_scm_invoke_seq(trident_scm_t* scm, const trident_args* args, int32_t n,
                                            void* stream, int32_t* out_selected) {
+  TRIDENT_RANGE("trident_scm_invoke_seq");
   if (!scm || (!args && n > 0) || n < 0) return fail(TRIDENT_ERR_INVALID, "bad sequence");
   int32_t result = TRIDENT_OK;
   for (int32_t i = 0; i < n; ++i) {
@@ -1607,6 +1625,7 @@ int32_t step_chunk(trident_scm* scm, const trident_args* a, int32_t m, void* str
 
 TRIDENT_API int32_t trident_scm_invoke_step(trident_scm_t* scm, const trident_args* args, int32_t n,
                                             void* stream, int32_t* out_selected) {
+  TRIDENT_RANGE("trident_scm_invoke_step");
   if (!scm || (!args && n > 0) || n < 0) return fail(TRIDENT_ERR_INVALID, "bad sequence");
   int32_t result = TRIDENT_OK;
   for (int32_t c0 = 0; c0 < n; c0 += kStepMax) {

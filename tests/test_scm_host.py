@@ -470,3 +470,16 @@ def test_launch_floor_probe_rejects_dry_runs_and_bad_counts(S):
     assert S.trident_launch_floor(s.h, None, -1) == S.ERR_INVALID
     assert S.trident_launch_floor(None, None, 1) == S.ERR_INVALID
     s.close()
+
+
+def test_nvtx_ranges_build_only_with_the_flag(S, tmp_path):
+    """NVTX ranges around the boundary calls are compiled in only with -DTRIDENT_NVTX: the
+    default library references no NVTX symbol, and the flagged host core still compiles."""
+    from paper_2609_37241_gb300 import build as B
+    nm = subprocess.run(["nm", "-D", S.LIB_PATH], capture_output=True, text=True).stdout
+    assert "nvtx" not in nm.lower()
+    src = os.path.join(B.CSRC, "scm.cpp")
+    obj = tmp_path / "scm_nvtx.o"
+    subprocess.run([B.nvcc(), *B.ARCH, *B.FLAGS, "-DTRIDENT_NVTX", "-c", src, "-o", str(obj)], check=True)
+    syms = subprocess.run(["nm", str(obj)], capture_output=True, text=True).stdout
+    assert "nvtx" in syms.lower()
