@@ -204,3 +204,29 @@ def test_step_replays_follow_new_data(S):
     st = s.stats()
     assert (st.step_replays, st.fused_launches, st.hits) == (2 * n, 4, 4 * n)
     s.close()
+
+
+def test_multi_wave_steps_back_to_back(S):
+    """Steps whose blocks outnumber the resident slots (several waves), 70 launches back to
+    back under PDL, most of them from the replay cache, with new data in the same buffers at
+    two points; every layer of every checked step equals the oracle."""
+    cfg = synth.QWEN3
+    T, n = 32, 6  # 6 x 288 blocks with one CTA per token: several waves
+    s, _ = step_scm(S, cfg, BF16, S.LAYOUT_ROWSTRIDED)
+    inps, outs, args = build_layers(S, cfg, T, n, seed=90)
+    for step in range(70):
+        if step in (40, 69):  # new data in the same buffers (inputs, caches and outputs)
+            g = np.random.default_rng(900 + step)
+            for l in range(n):
+                inps[l] = synth.layer_inputs(g, T, cfg)
+                fresh, _ = chain_device(inps[l], BF16, True)
+                for dst, src in zip(outs[l][0], fresh):
+                    dst.copy_(src)
+        assert run_step(S, s, args) == [0] * n
+        if step in (0, 40, 69):
+            torch.cuda.synchronize()
+            for inp, (_, out) in zip(inps, outs):
+                check_chain(L.layer_chain(inp, cfg["theta"], cfg["eps"], BF16, qknorm=True), out, inp)
+    st = s.stats()
+    assert st.fused_launches == 70 and st.step_replays > 0
+    s.close()
