@@ -479,7 +479,11 @@ def check_chain(ref, out, inp, dtype=BF16):
 
 @pytest.mark.parametrize("pdl", [False, True], ids=["plain", "pdl"])
 @pytest.mark.parametrize("cfg_name,T", [("LLAMA", 1), ("LLAMA", 4), ("LLAMA", 16), ("LLAMA", 64),
-                                        ("QWEN3", 1), ("QWEN3", 8), ("QWEN3", 32), ("QWEN3", 128)])
+                                        ("QWEN3", 1), ("QWEN3", 8), ("QWEN3", 32), ("QWEN3", 128),
+                                        # either side of the token-major / role-major boundary
+                                        # (two blocks per SM: 33 Llama tokens are 297 blocks,
+                                        # 34 are 306) and of the one-wave limit of two norm CTAs
+                                        ("LLAMA", 33), ("LLAMA", 34), ("LLAMA", 67)])
 def test_layer_chain_fused_matches_oracle(S, cfg_name, T, pdl):
     """The benchmarked layer configurations, with and without programmatic dependent launch
     (with it, as bench.py launches: token-major grids prefetch every block's lines, larger ones
