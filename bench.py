@@ -1137,7 +1137,7 @@ def run_ours(a):
     if rank == 0 and want("layers"):
         progress("per-token layer steps")
         per_t = {}
-        for T in (1, 4, 16, 64):
+        for T in toks_arg or (1, 4, 16, 64):
             per_t[str(T)], _ = bench_layer(c, cfg, T, K=max(500, min(K, 2000)), W=W)
         add_floor_fractions(per_t, floor_us)
         extra["llama_per_tokens"] = per_t
@@ -1296,7 +1296,7 @@ def main():
     p.add_argument("--warmup", type=int, default=20)
     p.add_argument("--impl", default="ours", choices=["ours", "reference"])
     p.add_argument("--quick", action="store_true", help="smaller sections (for smoke runs)")
-    p.add_argument("--tokens", default="", help="comma list of token counts for the qwen3 and sweep sections")
+    p.add_argument("--tokens", default="", help="comma list of token counts for the layers, qwen3 and sweep sections")
     p.add_argument("--sections", default="all",
                    help="comma list of: floor,layers,qwen3,host,stress,motivation,kernels,sweep,roofline,e2e,cpu"
                         " (default all;"

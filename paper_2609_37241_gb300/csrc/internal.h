@@ -128,6 +128,7 @@ struct ChainStepParams {
 struct KernelEntry {
   const void* fn = nullptr;
   const void* fn_inplace = nullptr;  // chain only: the entry for calls that write in place
+  const void* fn_late = nullptr;     // chain only: fn with the late launch trigger (LATE)
   const void* fn_step = nullptr;          // chain only: several calls per launch (ChainStepParams)
   const void* fn_step_inplace = nullptr;  // ... one block per token for the norms
   const void* fn_large = nullptr;  // add+RMSNorm: the entry for calls of >= large_rows rows

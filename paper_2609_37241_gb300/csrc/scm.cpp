@@ -390,6 +390,7 @@ struct Version {
   KernelEntry ke;
   CUfunction fn;
   CUfunction fn_inplace;  // layer chain: one block per token when outputs alias inputs
+  CUfunction fn_late;     // layer chain: `fn` with the late launch trigger
   int32_t wave_blocks;    // layer chain: blocks of `fn` resident at once on the whole GPU
   CUfunction fn_large;          // add+RMSNorm: entry for calls of >= ke.large_rows rows
   CUfunction step_fn;           // layer chain: several calls per launch (two blocks per token)
@@ -738,6 +739,7 @@ int32_t do_launch(trident_scm* scm, const Version& v, const trident_args* a, con
     ChainParams ch;
   } P;
   void* kp[1] = {&P};
+  bool late = false;  // layer chain: launch fn_late (the late launch trigger)
   switch (op) {
     case TRIDENT_OP_ADD_RMSNORM:
       pack_addnorm(a, 0, 1, 2, 3, 4, s, K_ACT_H, &P.an);
@@ -807,6 +809,13 @@ int32_t do_launch(trident_scm* scm, const Version& v, const trident_args* a, con
         c.rope_per_tok = (int32_t)(c.rope.NH / upb);
         cfg.gridDimX = (unsigned)(split + c.rope_per_tok + c.sw_tiles_per_row);
         cfg.gridDimY = (unsigned)s.T;
+      } else if ((scm->opt.flags & TRIDENT_OPT_PDL) && blocks + c.nA <= v.wave_blocks) {
+        // A role-major grid whose norm blocks and the next such grid fit the resident slots
+        // together: RoPE and SwiGLU blocks trigger the next launch at exit (late_trigger), so
+        // the next grid is placed whole while this one's norm blocks finish (measured, 48
+        // tokens: norm blocks one per SM instead of up to four, 3.42 -> 3.28 us per launch;
+        // at 64 tokens, where 96 blocks would then start late, 3.51 -> 3.69 us, so not there).
+        late = true;
       }
       break;
     }
@@ -832,6 +841,8 @@ int32_t do_launch(trident_scm* scm, const Version& v, const trident_args* a, con
   CUfunction fn = v.fn;
   if ((op == TRIDENT_OP_LAYER_CHAIN || op == TRIDENT_OP_LAYER_CHAIN_QKNORM) && P.ch.a_split == 1)
     fn = v.fn_inplace;
+  else if (late && v.fn_late)
+    fn = v.fn_late;
   if (v.fn_large && s.T >= v.ke.large_rows) fn = v.fn_large;  // many rows: the bulk-copy kernel
   return launch_on(scm, &cfg, fn, kp);
 }
@@ -1002,10 +1013,11 @@ int32_t get_rope_table(trident_scm* scm, double theta, int32_t D, const float2**
   if (cudaMalloc(&dev, host.size() * sizeof(float2)) != cudaSuccess)
     return fail(TRIDENT_ERR_CUDA, "cudaMalloc of the RoPE frequency table failed");
   // The copy must have landed before this registration returns: kernels read the table
-  // before their programmatic-launch wait, on any stream (a pageable-memory copy may return
-  // while its DMA is still in flight, hence the synchronisation).
+  // before their programmatic-launch wait, on any stream. A copy from pageable memory may
+  // return while its DMA is still in flight on the legacy default stream, so that stream
+  // (and only it: other streams' work does not hold the registration up) is synchronised.
   if (cudaMemcpy(dev, host.data(), host.size() * sizeof(float2), cudaMemcpyHostToDevice) != cudaSuccess ||
-      cudaDeviceSynchronize() != cudaSuccess) {
+      cudaStreamSynchronize(cudaStreamLegacy) != cudaSuccess) {
     cudaFree(dev);
     return fail(TRIDENT_ERR_CUDA, "upload of the RoPE frequency table failed");
   }
@@ -1227,6 +1239,12 @@ int32_t append_version(trident_scm_t* scm, const trident_spec_desc* desc, int32_
         if (cudaGetFuncBySymbol(&g, v.ke.fn_inplace) != cudaSuccess || !g)
           return fail(TRIDENT_ERR_CUDA, "cannot resolve the in-place kernel entry");
         v.fn_inplace = reinterpret_cast<CUfunction>(g);
+        if (v.ke.fn_late) {
+          cudaFunction_t l = nullptr;
+          if (cudaGetFuncBySymbol(&l, v.ke.fn_late) != cudaSuccess || !l)
+            return fail(TRIDENT_ERR_CUDA, "cannot resolve the late-trigger kernel entry");
+          v.fn_late = reinterpret_cast<CUfunction>(l);
+        }
         cudaFunction_t h = nullptr, k = nullptr;
         if (cudaGetFuncBySymbol(&h, v.ke.fn_step) != cudaSuccess || !h ||
             cudaGetFuncBySymbol(&k, v.ke.fn_step_inplace) != cudaSuccess || !k)
