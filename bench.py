@@ -430,7 +430,7 @@ def bench_launch_floor(c, n=2000):
     S, t = c.S, c.torch
     res = {}
     for name, flags in (("pdl", S.OPT_PDL), ("no_pdl", 0)):
-        s = S.Scm(device=c.dev.index or 0, flags=flags)
+        s = S.Scm(device=c.dev.index or 0, flags=flags | S.OPT_TIMING)
         assert S.trident_launch_floor(s.h, c.sp.value, 20) == S.OK, S.trident_scm_last_error()
         t.cuda.synchronize()
         e0, e1 = c.events()
@@ -441,10 +441,18 @@ def bench_launch_floor(c, n=2000):
         h1 = time.perf_counter()
         t.cuda.synchronize()
         assert st == S.OK, S.trident_scm_last_error()
+        # the launch call alone, per launch (library clock), in bursts of 32 with the queue
+        # drained in between -- the same pattern as the host cost per hit
+        for _ in range(1000 // 32 + 1):
+            assert S.trident_launch_floor(s.h, c.sp.value, 32) == S.OK, S.trident_scm_last_error()
+            t.cuda.synchronize()
+        ns = np.array(S.trident_scm_host_times(s.h, 1000)[1], np.float64)
         res[name] = dict(device_us=round(e0.elapsed_time(e1) * 1e3 / n, 3),
-                         host_us=round((h1 - h0) * 1e6 / n, 3))
+                         host_us=round((h1 - h0) * 1e6 / n, 3),
+                         launch_call_ns=dict(median=float(np.median(ns)), p99=float(np.percentile(ns, 99)),
+                                             samples=int(ns.size)))
         s.close()
-    c.launches += 2 * (n + 20)
+    c.launches += 2 * (n + 20 + 32 * (1000 // 32 + 1))
     return res
 
 
@@ -628,11 +636,21 @@ def bench_host_hit(c, n=1000):
     st, bb_ns = S.trident_scm_host_times(s.h, n)
     bb_ns = np.array(bb_ns[-n:], np.float64)
     # dispatch cost: the same calls in bursts of 32 with the queue drained in between (a
-    # decode step issues a few dozen calls, then waits for its results), warm caches
-    for _ in range(n // 32 + 1):
-        for _ in range(32):
-            inv(s.h, ar, c.sp, ctypes.byref(sel))
-        t.cuda.synchronize()
+    # decode step issues a few dozen calls, then waits for its results), warm caches; from
+    # the fast-call shim (the binding the headline uses) and, for comparison, from ctypes,
+    # whose own work between calls (about 1 us) leaves colder caches for the next call
+    def bursts(call):
+        for _ in range(n // 32 + 1):
+            for _ in range(32):
+                call()
+            t.cuda.synchronize()
+        return np.array(S.trident_scm_host_times(s.h, n)[1][-n:], np.float64)
+
+    ns_ctypes = bursts(lambda: inv(s.h, ar, c.sp, ctypes.byref(sel)))
+    ns, binding = ns_ctypes, "ctypes"
+    if c.fc is not None:
+        fhit, fh, fa, fs = c.fc.invoke, s.h.value, ctypes.addressof(a), c.sp.value or 0
+        ns, binding = bursts(lambda: fhit(fh, fa, fs)), "fastcall"
     fast_us = None
     if c.fc is not None:
         finv, hh, addr, sp = c.fc.invoke, s.h.value, ctypes.addressof(a), c.sp.value or 0
@@ -653,7 +671,6 @@ def bench_host_hit(c, n=1000):
         c.L.trident_scm_invoke(d.h, ar, c.sp, None)
     dns = np.array(S.trident_scm_host_times(d.h, n)[1], np.float64)
     d.close()
-    st, ns = S.trident_scm_host_times(s.h, n)  # the last n hits: the bursts
     hits = S.trident_scm_spec_hits(s.h)[1]
     # one call at a time (after the samples above were read): device us from an event
     # recorded before the call to one after it, and host us from the call to the return of
@@ -671,8 +688,7 @@ def bench_host_hit(c, n=1000):
         ev_us.append(e0.elapsed_time(e1) * 1e3)
         wall_us.append((w1 - w0) * 1e6)
     assert_all_hit(s, "host dispatch")
-    ns = np.array(ns[-n:], np.float64)
-    c.launches += 2 * n + 32 * (n // 32 + 1) + 200
+    c.launches += 2 * n + 32 * (n // 32 + 1) * (2 if c.fc is not None else 1) + 200
     s.close()
     # the fused layer chain (18 tensors, 64 tokens): host ns per hit with the launch, and alone
     cfg = synth.LLAMA
@@ -685,21 +701,27 @@ def bench_host_hit(c, n=1000):
                                 rope_theta=cfg["theta"]))
         ca = sets.fused_args(c, 0)
         cinv, caddr = c.invoker(cs), ctypes.addressof(ca)
-        for _ in range(n + 50):
+        for _ in range(50):
             cinv(caddr)
         t.cuda.synchronize()
+        for _ in range(n // 32 + 1):  # in bursts, as above (a device step is longer than a call)
+            for _ in range(32):
+                cinv(caddr)
+            t.cuda.synchronize()
         cns = np.array(S.trident_scm_host_times(cs.h, n)[1], np.float64)
         chain_ns[label] = dict(median_ns=float(np.median(cns)), p99_ns=float(np.percentile(cns, 99)))
         if label == "live":
             assert_all_hit(cs, "chain host")
-            c.launches += n + 50
+            c.launches += 50 + 32 * (n // 32 + 1)
         cs.close()
     del sets
     return dict(hits_on_bf16_contig=int(hits[3]), calls=n, selected=sel.value, layer_chain=chain_ns,
                 isolated_call=dict(event_us_median=round(float(np.median(ev_us)), 3),
                                    launch_to_completion_us_median=round(float(np.median(wall_us)), 3),
                                    calls=len(ev_us)),
-                median_ns=float(np.median(ns)), p99_ns=float(np.percentile(ns, 99)),
+                median_ns=float(np.median(ns)), p99_ns=float(np.percentile(ns, 99)), binding=binding,
+                ctypes_bursts=dict(median_ns=float(np.median(ns_ctypes)),
+                                   p99_ns=float(np.percentile(ns_ctypes, 99))),
                 min_ns=float(ns.min()), guards_only_median_ns=float(np.median(dns)),
                 guards_only_p99_ns=float(np.percentile(dns, 99)),
                 back_to_back=dict(median_ns=float(np.median(bb_ns)), p99_ns=float(np.percentile(bb_ns, 99)),

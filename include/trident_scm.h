@@ -459,7 +459,8 @@ int32_t trident_scm_spec_hits(const trident_scm_t* scm, uint64_t* out, int32_t c
 
 /* With TRIDENT_OPT_TIMING: copies the host nanoseconds of the most recent hits (entry
  * of invoke to return, launch included) into out[0..cap-1], oldest first; *n gets the
- * count. Samples are recorded per hit, so concurrent invokers may interleave. */
+ * count. Samples are recorded per hit (and per launch of trident_launch_floor), so
+ * concurrent invokers may interleave. */
 int32_t trident_scm_host_times(const trident_scm_t* scm, uint32_t* out, int32_t cap, int32_t* n);
 
 /* Latency-floor probe (measurement, not part of the dispatch path): launches n empty
@@ -467,8 +468,10 @@ int32_t trident_scm_host_times(const trident_scm_t* scm, uint32_t* out, int32_t 
  * launch) back to back on `stream`, with the SCM's launch configuration (its context, and
  * programmatic stream serialisation when TRIDENT_OPT_PDL is set) through the same driver
  * entry point as a hit. The time per launch is the single-launch floor against which
- * decode-size steps are reported. Reads and writes no memory. Errors: ERR_INVALID (scm
- * NULL or n < 0), ERR_STATE (dry-run SCM), ERR_CUDA. */
+ * decode-size steps are reported. With TRIDENT_OPT_TIMING each launch's host nanoseconds
+ * (the launch call alone: no guards, no packing) go to the host-time ring, the baseline
+ * against which a hit's host time is read. Reads and writes no memory. Errors:
+ * ERR_INVALID (scm NULL or n < 0), ERR_STATE (dry-run SCM), ERR_CUDA. */
 int32_t trident_launch_floor(trident_scm_t* scm, void* stream, int32_t n);
 
 /* Reads the device status word (TRIDENT_DEVERR_* bits) after synchronising `stream`;

@@ -978,6 +978,13 @@ inline uint64_t now_ns() {
              std::chrono::steady_clock::now().time_since_epoch()).count();
 }
 
+// One host-time sample (ns since t0) into the SCM's ring (TRIDENT_OPT_TIMING).
+void record_host_time(trident_scm* scm, uint64_t t0) {
+  const uint64_t k = scm->ring_n.fetch_add(1, std::memory_order_relaxed);
+  const uint64_t dt = now_ns() - t0;
+  scm->ring[k % (uint64_t)scm->ring_cap] = dt > 0xffffffffull ? 0xffffffffu : (uint32_t)dt;
+}
+
 int32_t count_error(trident_scm* scm, int32_t st) {
   if (st == TRIDENT_ERR_INVALID) scm->err_invalid.fetch_add(1, std::memory_order_relaxed);
   else if (st == TRIDENT_ERR_CUDA) scm->err_cuda.fetch_add(1, std::memory_order_relaxed);
@@ -1345,11 +1352,7 @@ int32_t run_hit(trident_scm* scm, int32_t sel, const trident_args* args, const S
   scm->hits.fetch_add(1, std::memory_order_relaxed);
   scm->hits_per[sel].fetch_add(1, std::memory_order_relaxed);
   scm->guard_evals.fetch_add((uint64_t)sel + 1, std::memory_order_relaxed);
-  if (scm->ring) {
-    const uint64_t k = scm->ring_n.fetch_add(1, std::memory_order_relaxed);
-    const uint64_t dt = now_ns() - t0;
-    scm->ring[k % (uint64_t)scm->ring_cap] = dt > 0xffffffffull ? 0xffffffffu : (uint32_t)dt;
-  }
+  if (scm->ring) record_host_time(scm, t0);
   return TRIDENT_OK;
 }
 
@@ -1736,8 +1739,10 @@ TRIDENT_API int32_t trident_launch_floor(trident_scm_t* scm, void* stream, int32
   cfg.blockDimX = 32;
   cfg.gridDimX = 1;
   for (int32_t i = 0; i < n; ++i) {
+    const uint64_t t0 = scm->ring ? now_ns() : 0;
     const int32_t st = launch_on(scm, &cfg, fn, nullptr);
     if (st != TRIDENT_OK) return st;
+    if (scm->ring) record_host_time(scm, t0);
   }
   return TRIDENT_OK;
 }

@@ -197,3 +197,17 @@ def test_launch_floor_probe_runs(S, pdl):
     torch.cuda.synchronize()
     assert S.trident_scm_device_status(s.h, st)[1] == 0
     s.close()
+
+
+def test_launch_floor_records_each_launch_with_timing(S):
+    """With TRIDENT_OPT_TIMING every launch of the probe leaves one host-time sample (the
+    launch call alone), and no hit or miss is counted for it."""
+    s = S.Scm(device=0, flags=S.OPT_PDL | S.OPT_TIMING)
+    st = torch.cuda.current_stream().cuda_stream
+    assert S.trident_launch_floor(s.h, st, 37) == S.OK, S.trident_scm_last_error()
+    torch.cuda.synchronize()
+    rc, ns = S.trident_scm_host_times(s.h, 100)
+    assert rc == S.OK and len(ns) == 37 and all(0 < x < 10 ** 9 for x in ns)
+    stats = s.stats()
+    assert stats.hits == 0 and stats.misses == 0
+    s.close()
