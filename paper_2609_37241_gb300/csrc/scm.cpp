@@ -795,27 +795,33 @@ int32_t do_launch(trident_scm* scm, const Version& v, const trident_args* a, con
       st = set_chain_split(&c, s.T, split, &blocks);
       if (st != TRIDENT_OK) return st;
       cfg.gridDimX = (unsigned)blocks;
-      // Token-major grid (chain_block_tok) for grids of at most two blocks per SM, when every
-      // token has the same number of RoPE blocks: consecutive blocks then mix roles, so the
-      // blocks that land together on one SM are not all norm blocks (measured: 16 tokens
-      // 3.55 -> 2.85 us per layer step, 1 token 2.20 -> 2.04 us; 32 tokens, 288 blocks, 36
-      // Qwen3-style layers 131.5 -> 109.6 us). A grid that nearly fills the GPU keeps the
+      // Under PDL, a role-major grid of more than a quarter block per SM whose blocks, with
+      // its own norm blocks, fit the resident slots launches fn_late: its RoPE and SwiGLU
+      // blocks trigger the next launch at their exit, so the next grid is placed whole while
+      // this one's norm blocks finish, one norm block per SM instead of up to four. Same-box
+      // A/B of Llama layer steps against the token-major grid below: 6 tokens 2.22 -> 2.12
+      // us, 8 tokens 2.33 -> 2.14, 16 tokens 2.58 -> 2.29, 24 tokens 3.19 -> 2.44, 32
+      // tokens 2.98 -> 2.57, 48 tokens (role-major before) 3.21 -> 2.99; equal at 2 and 4
+      // tokens, and at 1 token 1.5-2 % slower (nothing to place, and the next launch starts
+      // later), hence the lower bound; at 64 tokens, where 96 blocks would start late, the
+      // probe measured 3.51 -> 3.69 us, hence the upper one.
+      // Otherwise a token-major grid (chain_block_tok) for grids of at most two blocks per SM,
+      // when every token has the same number of RoPE blocks: consecutive blocks then mix
+      // roles, so the blocks that land together on one SM are not all norm blocks (measured
+      // against role-major grids without the late trigger: 16 tokens 3.55 -> 2.85 us per
+      // layer step, 1 token 2.20 -> 2.04 us). A grid that nearly fills the GPU keeps the
       // role-major order, which starts the longest (norm) blocks first (64 tokens: 3.98 us
       // role-major, 4.05 us token-major; 48 and 64 tokens in other interleaved orders were
       // slower as well).
       const int64_t upb = rope_units_per_block(c.rope.D, 2);
-      if (c.rope.NH % upb == 0 && s.T >= 1 && s.T <= 65535 && blocks <= 2 * scm->sm_count) {
+      if ((scm->opt.flags & TRIDENT_OPT_PDL) && split == 2 && v.fn_late && 4 * blocks > scm->sm_count &&
+          blocks + c.nA <= v.wave_blocks) {
+        late = true;
+      } else if (c.rope.NH % upb == 0 && s.T >= 1 && s.T <= 65535 && blocks <= 2 * scm->sm_count) {
         c.tok_grid = 1;
         c.rope_per_tok = (int32_t)(c.rope.NH / upb);
         cfg.gridDimX = (unsigned)(split + c.rope_per_tok + c.sw_tiles_per_row);
         cfg.gridDimY = (unsigned)s.T;
-      } else if ((scm->opt.flags & TRIDENT_OPT_PDL) && blocks + c.nA <= v.wave_blocks) {
-        // A role-major grid whose norm blocks and the next such grid fit the resident slots
-        // together: RoPE and SwiGLU blocks trigger the next launch at exit (late_trigger), so
-        // the next grid is placed whole while this one's norm blocks finish (measured, 48
-        // tokens: norm blocks one per SM instead of up to four, 3.42 -> 3.28 us per launch;
-        // at 64 tokens, where 96 blocks would then start late, 3.51 -> 3.69 us, so not there).
-        late = true;
       }
       break;
     }
@@ -835,7 +841,7 @@ int32_t do_launch(trident_scm* scm, const Version& v, const trident_args* a, con
     case TRIDENT_OP_QKNORM_ROPE_KV: P.rp.prefetch = pf; break;
     case TRIDENT_OP_SWIGLU: P.sw.prefetch = pf; break;
     case TRIDENT_OP_LAYER_CHAIN:
-    case TRIDENT_OP_LAYER_CHAIN_QKNORM: P.ch.prefetch = chain_prefetch_mode(pdl, pf != 0, true); break;
+    case TRIDENT_OP_LAYER_CHAIN_QKNORM: P.ch.prefetch = chain_prefetch_mode(pdl, pf != 0 && !late, true); break;
     default: P.pw.prefetch = pf; break;
   }
   CUfunction fn = v.fn;

@@ -480,11 +480,12 @@ def check_chain(ref, out, inp, dtype=BF16):
 @pytest.mark.parametrize("pdl", [False, True], ids=["plain", "pdl"])
 @pytest.mark.parametrize("cfg_name,T", [("LLAMA", 1), ("LLAMA", 4), ("LLAMA", 16), ("LLAMA", 64),
                                         ("QWEN3", 1), ("QWEN3", 8), ("QWEN3", 32), ("QWEN3", 128),
-                                        # either side of the token-major / role-major boundary
-                                        # (two blocks per SM: 33 Llama tokens are 297 blocks,
-                                        # 34 are 306) and of the one-wave limit of two norm CTAs;
-                                        # 34 Llama and 40 Qwen3 tokens take the late-trigger
-                                        # entry under PDL, 64 and 67 do not
+                                        # without PDL, either side of the token-major /
+                                        # role-major boundary (two blocks per SM: 33 Llama
+                                        # tokens are 297 blocks, 34 are 306) and of the one-wave
+                                        # limit of two norm CTAs; under PDL 16, 33, 34 Llama and
+                                        # 8, 32, 40 Qwen3 tokens take the late-trigger entry,
+                                        # 1 and 4 the token-major grid, 64 and 67 neither
                                         ("LLAMA", 33), ("LLAMA", 34), ("LLAMA", 67), ("QWEN3", 40)])
 def test_layer_chain_fused_matches_oracle(S, cfg_name, T, pdl):
     """The benchmarked layer configurations, with and without programmatic dependent launch
