@@ -131,11 +131,18 @@ __device__ __forceinline__ void chain_norm(const ChainParams& c, const int64_t r
   }
 }
 
-// RoPE role: RoPE block rb (< nB), i.e. head-rows [rb * UPB, (rb + 1) * UPB); fq holds the
-// lane's frequencies, loaded before the PDL wait (rope_lane_freqs).
-template <int DT, int D, bool QKNORM>
+// RoPE role: RoPE block rb (< nB), i.e. head-rows [rb * UPB, (rb + 1) * UPB) with UPB =
+// rope_k * 256 / LPH (rope_rows with rope_k = 3 on grids several waves long); fq holds the
+// lane's frequencies (rope_lane_freqs).
+// Only the one-CTA-per-token entries (SPLIT 1: in-place calls, and grids too large for one
+// wave) carry the rope_rows path, so the others keep their registers.
+template <int DT, int D, bool QKNORM, bool ROWS3>
 __device__ __forceinline__ void chain_rope(const ChainParams& c, const int64_t rb, const float* fq) {
   constexpr int LPH = D / Act<DT>::VE;
+  if (ROWS3 && c.rope_k == 3) {
+    rope_rows<DT, D, QKNORM, 3>(c.rope, rb, threadIdx.x % LPH, threadIdx.x / LPH, fq);
+    return;
+  }
   const int64_t unit = rb * (kThreads / LPH) + threadIdx.x / LPH;
   if (unit < c.rope.T * c.rope.NH) rope_head_row<DT, D, QKNORM>(c.rope, unit, threadIdx.x % LPH, fq);
 }
@@ -160,7 +167,7 @@ __device__ __forceinline__ void chain_block(const ChainParams& c, const int b, c
     const int64_t row = b / SPLIT;
     chain_norm<DT, VPT, SPLIT>(c, row, b - (int)row * SPLIT);
   } else if (b < c.nA + c.nB) {
-    chain_rope<DT, D, QKNORM>(c, b - c.nA, fq);
+    chain_rope<DT, D, QKNORM, SPLIT == 1>(c, b - c.nA, fq);
   } else {
     const int64_t tile = b - c.nA - c.nB;
     if (tile >= c.sw_tiles) return;
@@ -182,7 +189,7 @@ __device__ __forceinline__ void chain_block_tok(const ChainParams& c, const floa
   if (q < SPLIT) {
     chain_norm<DT, VPT, SPLIT>(c, blockIdx.y, q);
   } else if (q < SPLIT + c.rope_per_tok) {
-    chain_rope<DT, D, QKNORM>(c, (int64_t)blockIdx.y * c.rope_per_tok + (q - SPLIT), fq);
+    chain_rope<DT, D, QKNORM, false>(c, (int64_t)blockIdx.y * c.rope_per_tok + (q - SPLIT), fq);
   } else {
     chain_swiglu<DT, kChainSwigluUnroll>(c, blockIdx.y, q - SPLIT - c.rope_per_tok);
   }
@@ -242,6 +249,7 @@ __device__ __forceinline__ void chain_prefetch(const ChainParams& c, const int b
   } else if (c.prefetch == 2) {
     return;
   } else if (b < c.nA + c.nB) {
+    if (c.rope_k != 1) return;  // several head-rows per lane group: grids too long to prefetch
     rope_prefetch<DT, D>(c.rope, (int64_t)(b - c.nA) * (kThreads / LPH) + tid / LPH, tid % LPH);
   } else {
     const int64_t tile = b - c.nA - c.nB;

@@ -321,6 +321,107 @@ __device__ __forceinline__ void rope_head_row(const RopeParams& p, int64_t unit,
   rope_row_finish<DT, D, QKNORM>(p, unit, lane, raw, pos, gg, fq);
 }
 
+// K head-rows per lane group, for grids several waves long: lane group g (of G = 256 / LPH)
+// of RoPE block rb owns the units rb * G * K + g + G * j, j < K -- with NH = 48 and K = 3 one
+// token's q, k and v rows. A block then moves K times the bytes for the same fixed costs,
+// which pays where blocks queue for slots (a 1024-token layer 39.7 -> 34.8 us) and not where
+// a block's own latency is the step (one wave: slower per block). Rows of one token share
+// the position and so every angle: the lane computes its sines and cosines once, for the
+// token of the first row, and again only for a row of another token (NH not a multiple of
+// G), reloading its frequencies then. All K rows' loads are issued before any is used.
+template <int DT, int D, bool QKNORM, int K>
+__device__ __forceinline__ void rope_rows(const RopeParams& p, const int64_t rb, const int lane, const int g,
+                                          const float* fq) {
+  constexpr int VE = Act<DT>::VE;
+  constexpr int LPH = D / VE;
+  constexpr int HALF = LPH / 2;
+  constexpr int EB = Act<DT>::BYTES;
+  constexpr int G = kThreads / LPH;
+  const unsigned group_mask =
+      (LPH == 32) ? 0xffffffffu : (((1u << LPH) - 1u) << ((threadIdx.x & 31) & ~(LPH - 1)));
+  const int64_t nunits = p.T * p.NH;
+  const int64_t u0 = rb * (int64_t)(G * K) + g;
+  if (u0 >= nunits) return;
+  uint4 raw[K];
+#pragma unroll
+  for (int j = 0; j < K; ++j) {
+    const int64_t u = u0 + (int64_t)G * j;
+    if (u < nunits) {
+      int64_t t;
+      int h;
+      bool is_q, is_v;
+      rope_row_where<DT, D>(p, u, &t, &h, &is_q, &is_v);
+      const char* src = is_q ? row_ptr(p.q, t, p.q_rs, EB) : is_v ? row_ptr(p.v, t, p.v_rs, EB)
+                                                                 : row_ptr(p.k, t, p.k_rs, EB);
+      src += ((int64_t)h * D + lane * VE) * EB;
+      raw[j] = is_q ? ld16(src) : ldg16(src);
+    }
+  }
+  const int64_t t0 = u0 / p.NH;
+  const int32_t pos0 = __ldg(p.pos + t0);
+  float sn[VE], cs[VE];
+#pragma unroll
+  for (int e = 0; e < VE; ++e) rope_sincos((float)pos0, fq[2 * e], fq[2 * e + 1], &sn[e], &cs[e]);
+  const bool low = lane < HALF;
+#pragma unroll
+  for (int j = 0; j < K; ++j) {
+    const int64_t u = u0 + (int64_t)G * j;
+    if (u >= nunits) break;
+    int64_t t;
+    int h;
+    bool is_q, is_v;
+    rope_row_where<DT, D>(p, u, &t, &h, &is_q, &is_v);
+    // units ascend, so once a row belongs to a later token every following row does too
+    const bool same = t == t0;
+    const int32_t pos = same ? pos0 : __ldg(p.pos + t);
+    if (pos < 0 || (int64_t)pos >= p.S) {
+      if (lane == 0) atomicOr(p.err, kErrPos);
+      continue;
+    }
+    if (is_v) {  // bit copy into the cache
+      st16(reinterpret_cast<char*>(p.v_cache) + (((int64_t)h * p.S + pos) * D + lane * VE) * EB, raw[j]);
+      continue;
+    }
+    float x[VE];
+    unpack<DT>(raw[j], x);
+    if (QKNORM) {
+      const float* gam = (is_q ? p.gamma_q : p.gamma_k) + lane * VE;
+      float gg[VE];
+#pragma unroll
+      for (int q = 0; q < VE / 4; ++q) {
+        const float4 g4 = ldg_f4(gam + 4 * q);
+        gg[4 * q] = g4.x; gg[4 * q + 1] = g4.y; gg[4 * q + 2] = g4.z; gg[4 * q + 3] = g4.w;
+      }
+      float ss = 0.f;
+#pragma unroll
+      for (int e = 0; e < VE; ++e) ss = fmaf(x[e], x[e], ss);
+#pragma unroll
+      for (int o = LPH / 2; o > 0; o >>= 1) ss += __shfl_xor_sync(group_mask, ss, o, LPH);
+      const float inv = rsqrtf(ss * p.inv_D + p.eps);
+#pragma unroll
+      for (int e = 0; e < VE; ++e) x[e] = x[e] * inv * gg[e];
+    }
+    float other[VE];
+#pragma unroll
+    for (int e = 0; e < VE; ++e) other[e] = __shfl_xor_sync(group_mask, x[e], HALF, LPH);
+    if (!same) {
+      float f2[2 * VE];
+      rope_lane_freqs<DT, D>(p.inv_freq, lane, f2);
+#pragma unroll
+      for (int e = 0; e < VE; ++e) rope_sincos((float)pos, f2[2 * e], f2[2 * e + 1], &sn[e], &cs[e]);
+    }
+    float y[VE];
+#pragma unroll
+    for (int e = 0; e < VE; ++e)
+      y[e] = low ? fmaf(x[e], cs[e], -other[e] * sn[e]) : fmaf(x[e], cs[e], other[e] * sn[e]);
+    if (is_q) {
+      st16(row_ptr(p.q, t, p.q_rs, EB) + ((int64_t)h * D + lane * VE) * EB, pack<DT>(y));
+    } else {
+      st16(reinterpret_cast<char*>(p.k_cache) + (((int64_t)h * p.S + pos) * D + lane * VE) * EB, pack<DT>(y));
+    }
+  }
+}
+
 // ---------------------------------------------------------------- SwiGLU tile
 template <int DT> __device__ __forceinline__ float silu_mul(float g, float u);
 // bf16/fp16 outputs: fast exp and divide (relative error ~1e-6, far below the output ulp;

@@ -103,6 +103,7 @@ struct ChainParams {
                      // 2 only the norm blocks' rows, 0 none
   int32_t tok_grid;  // 1: grid (a_split + rope_per_tok + sw_tiles_per_row, T), token-major
   int32_t rope_per_tok;  // RoPE blocks per token (token-major grid: nB = T * rope_per_tok)
+  int32_t rope_k;    // head-rows per RoPE lane group: 1, or 3 on grids several waves long
   int64_t sw_tiles;  // T * sw_tiles_per_row (valid SwiGLU tiles)
 };
 

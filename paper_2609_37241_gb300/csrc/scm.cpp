@@ -690,6 +690,7 @@ int32_t pack_chain(trident_scm* scm, const Version& v, const trident_args* a, co
   c->prefetch = 0;
   c->tok_grid = 0;
   c->rope_per_tok = 0;
+  c->rope_k = 1;
   return TRIDENT_OK;
 }
 
@@ -701,12 +702,27 @@ bool chain_inplace(const trident_args* a) {
          t[C_R2].data == t[C_R0].data || t[C_X2].data == t[C_AO].data;
 }
 
-int32_t set_chain_split(ChainParams* c, int64_t T, int32_t split, int64_t* blocks) {
+// Sets the norm CTAs per token (split) and the RoPE head-rows per lane group (rope_k), and
+// with them nA, nB and the grid's block count.
+int32_t set_chain_split(ChainParams* c, int64_t T, int32_t split, int32_t rope_k, int64_t* blocks) {
   c->a_split = split;
   c->nA = (int32_t)(T * split);
+  c->rope_k = rope_k;
+  const int64_t upb = (int64_t)rope_units_per_block(c->rope.D, 2) * rope_k;
+  c->nB = (int32_t)((T * c->rope.NH + upb - 1) / upb);
   *blocks = (int64_t)c->nA + c->nB + c->nC;
   return TRIDENT_OK;
 }
+
+// Three head-rows per RoPE lane group (rope_rows) on grids several waves long: a grid whose
+// one-CTA-per-token form with one head-row per lane group (`one` blocks) exceeds the resident
+// slots. There blocks queue for slots and a RoPE block that moves three rows for the same
+// fixed costs pays; within one wave a block's own latency is the step (a single-wave grid of
+// such blocks measured slower: 64 tokens 3.52 -> 4.46 us). Same-box A/B: Llama layer steps
+// at 128 tokens 5.61 -> 5.12 us, 256 tokens 9.37 -> 8.39 us; 36 Qwen3-style layers in one
+// launch at 32 / 64 / 128 / 256 tokens 36.7 / 70.5 / 142.9 / 281.0 -> 35.2 / 65.6 / 128.6 /
+// 252.7 us.
+inline int32_t chain_rope_k(int64_t one, int64_t wave_blocks) { return one > wave_blocks ? 3 : 1; }
 
 // Layer-chain prefetch before the PDL wait: every block's first lines for grids of at most
 // one block per SM (small_grid); otherwise, when norm_rows, only the norm blocks prefetch:
@@ -791,8 +807,9 @@ int32_t do_launch(trident_scm* scm, const Version& v, const trident_args* a, con
       // while the grid still fits in one wave, and unless an output is written over an
       // input the partner CTA still reads (in-place calls keep one CTA per token).
       const int32_t split = (!chain_inplace(a) && 2 * s.T + c.nB + c.nC <= v.wave_blocks) ? 2 : 1;
+      const int32_t rope_k = split == 1 ? chain_rope_k(s.T + c.nB + c.nC, v.wave_blocks) : 1;
       int64_t blocks = 0;
-      st = set_chain_split(&c, s.T, split, &blocks);
+      st = set_chain_split(&c, s.T, split, rope_k, &blocks);
       if (st != TRIDENT_OK) return st;
       cfg.gridDimX = (unsigned)blocks;
       // Under PDL, a role-major grid of more than a quarter block per SM whose blocks, with
@@ -1598,19 +1615,21 @@ int32_t step_chunk(trident_scm* scm, const trident_args* a, int32_t m, void* str
   CUfunction fn = nullptr;
   if (!scm->dry) {
     bool inplace = false;
-    int64_t two = 0;  // blocks with two CTAs per token
+    int64_t two = 0, one = 0;  // blocks with two / one CTAs per token (one head-row per lane group)
     for (int32_t i = 0; i < m; ++i) {
       ChainParams& c = P.c[i];
       const int32_t st = pack_chain(scm, scm->versions[sel[i]], a + i, sig[i], kChainStepSwigluUnroll, &c);
       if (st != TRIDENT_OK) return count_error(scm, st);
       inplace = inplace || chain_inplace(a + i);
       two += 2 * sig[i].T + c.nB + c.nC;
+      one += sig[i].T + c.nB + c.nC;
     }
     const int32_t split = (!inplace && two <= v0->step_wave_blocks) ? 2 : 1;
+    const int32_t rope_k = split == 1 ? chain_rope_k(one, v0->step_wave_blocks) : 1;
     int64_t first = 0;
     for (int32_t i = 0; i < m; ++i) {
       int64_t blocks = 0;
-      set_chain_split(&P.c[i], sig[i].T, split, &blocks);
+      set_chain_split(&P.c[i], sig[i].T, split, rope_k, &blocks);
       P.first[i] = (int32_t)first;
       first += blocks;
       if (first > 0x7fffffff)

@@ -533,6 +533,9 @@ def test_layer_chain_largest_bucket(S):
     (BF16, 8192, 64, 28672, 3, False),     # H 8192 instantiation (4 vectors per thread)
     (BF16, 8192, 64, 28672, 200, True),    # H 8192, grid beyond one wave: one block per token
     (FP16, 8192, 64, 28672, 5, True),
+    # several waves with 36 head-rows per token: three-row RoPE lane groups whose rows belong
+    # to two tokens (the H 8192 case above covers it with q/k norm, 80 head-rows per token)
+    (BF16, 4096, 20, 14336, 300, False),
 ])
 def test_layer_chain_other_sizes_and_dtypes(S, dtype, H, Hq, I, T, qk):
     cfg = dict(H=H, Hq=Hq, Hkv=8, D=128, S=2048, I=I, theta=1e6, qknorm=qk, eps=1e-6)
