@@ -1071,6 +1071,38 @@ def bench_sweep(c, reps=20, quick=False, tokens=None):
     return out
 
 
+def bench_chain_large(c, reps=10):
+    """The fused layer chain where it is bandwidth-bound: Llama- and Qwen3-style layers at
+    4096 and 8192 tokens (the KV cache's 8192 slots bound T), one launch per call, `reps`
+    calls back to back, each moving far more than the L2 (0.7-1.4 GB), against the measured
+    copy bandwidth. Token counts of several waves: one norm CTA per token, three head-rows per
+    RoPE lane group."""
+    S = c.S
+    peak, _ = measured_peaks()
+    out = []
+    for name, cfg in (("llama", c.synth.LLAMA), ("qwen3", c.synth.QWEN3)):
+        qk = cfg.get("qknorm", False)
+        fixed = [cfg[k] for k in ("H", "Hq", "Hkv", "D", "S", "I")]
+        op = S.OP_LAYER_CHAIN_QKNORM if qk else S.OP_LAYER_CHAIN
+        scm = S.Scm(device=c.dev.index or 0, flags=S.OPT_PDL)
+        scm.register(S.make_spec(op, S.BF16, fixed, 1, 1 << 20, layout=S.LAYOUT_ROWSTRIDED,
+                                 rope_theta=cfg["theta"]))
+        inv = c.invoker(scm)
+        for T in ((4096, 8192) if name == "llama" else (4096,)):
+            sets = ChainSets(c, cfg, T, min_bytes=2 * L2_BYTES, max_sets=2)
+            args = [sets.fused_args(c, i) for i in range(sets.R)]
+            addrs = [ctypes.addressof(a) for a in args]
+            us, _ = time_steps(c, lambda i: inv(addrs[i % len(addrs)]), reps, 3)
+            c.launches += reps + 3
+            b = chain_bytes_per_launch(cfg, T)
+            out.append(dict(layer=name, T=T, us=round(us, 3), gbs=round(b / us / 1e3, 1),
+                            frac_measured=round(b / us / 1e3 / peak, 3), bytes_per_launch=int(b)))
+            del args, addrs, sets
+        assert_all_hit(scm, "chain large")
+        scm.close()
+    return out
+
+
 def kernel_duration_chain(c, cfg, T, reps=200):
     """Average duration of the fused chain kernel: `reps` launches issued back to back by
     one native call (device-bound), CUDA events on the launching stream."""
@@ -1197,6 +1229,8 @@ def run_ours(a):
     if rank == 0 and want("sweep"):
         progress("hbm sweep")
         extra["hbm_sweep"] = bench_sweep(c, quick=a.quick, tokens=toks_arg)
+        if not a.quick and not toks_arg:
+            extra["hbm_sweep"]["layer_chain"] = bench_chain_large(c)
     if rank == 0 and want("roofline"):
         progress("roofline kernel")
         kd = kernel_duration_chain(c, cfg, HEADLINE_T)

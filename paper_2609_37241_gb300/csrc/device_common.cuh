@@ -179,16 +179,42 @@ __device__ __forceinline__ void rope_sincos(float pos, float fhi, float flo, flo
 }
 
 // ---------------------------------------------------------------- RoPE head-row
+// Token and head-row of a unit: unit = t * NH + hh. A division by a runtime divisor is a
+// long instruction sequence; for units below 2^32 (every grid in practice) the quotient comes
+// from the host's round-up multiplier for NH (Granlund and Montgomery, "Division by invariant
+// integers using multiplication", 1994): t = (h + ((u - h) >> 1)) >> (shift - 1) with
+// h = umulhi(u, magic), exact for every 32-bit u.
+__device__ __forceinline__ void rope_unit_split(const RopeParams& p, int64_t unit, int64_t* t, int* hh) {
+  if (unit <= 0xffffffffll) {
+    const uint32_t u = (uint32_t)unit;
+    const uint32_t h = __umulhi(u, p.nh_magic);
+    const uint32_t q = (h + ((u - h) >> 1)) >> (p.nh_shift - 1);
+    *t = q;
+    *hh = (int)(u - q * (uint32_t)p.NH);
+  } else {
+    *t = unit / p.NH;
+    *hh = (int)(unit - *t * p.NH);
+  }
+}
+
+// q, k or v head of head-row hh of a token.
+__device__ __forceinline__ void rope_head_of(const RopeParams& p, int hh, int* h, bool* is_q, bool* is_v) {
+  *is_v = hh >= p.Hq + p.Hkv;
+  *is_q = hh < p.Hq;
+  *h = *is_q ? hh : (*is_v ? hh - p.Hq - p.Hkv : hh - p.Hq);
+}
+
 // L2 prefetch of head-row `unit`'s source line(s) and position (lanes on a line boundary).
 template <int DT, int D>
 __device__ __forceinline__ void rope_prefetch(const RopeParams& p, int64_t unit, int lane) {
   constexpr int VE = Act<DT>::VE;
   constexpr int EB = Act<DT>::BYTES;
   if (unit >= p.T * p.NH || (lane * VE * EB) % 128 != 0) return;
-  const int64_t t = unit / p.NH;
-  const int hh = (int)(unit - t * p.NH);
-  const bool is_q = hh < p.Hq, is_v = hh >= p.Hq + p.Hkv;
-  const int h = is_q ? hh : (is_v ? hh - p.Hq - p.Hkv : hh - p.Hq);
+  int64_t t;
+  int hh, h;
+  bool is_q, is_v;
+  rope_unit_split(p, unit, &t, &hh);
+  rope_head_of(p, hh, &h, &is_q, &is_v);
   const char* src = is_q ? row_ptr(p.q, t, p.q_rs, EB) : is_v ? row_ptr(p.v, t, p.v_rs, EB)
                                                              : row_ptr(p.k, t, p.k_rs, EB);
   prefetch_l2(src + ((int64_t)h * D + lane * VE) * EB);
@@ -226,11 +252,9 @@ __device__ __forceinline__ void rope_lane_freqs(const float2* inv_freq, int lane
 template <int DT, int D>
 __device__ __forceinline__ void rope_row_where(const RopeParams& p, int64_t unit, int64_t* t, int* h,
                                                bool* is_q, bool* is_v) {
-  *t = unit / p.NH;
-  const int hh = (int)(unit - *t * p.NH);
-  *is_v = hh >= p.Hq + p.Hkv;
-  *is_q = hh < p.Hq;
-  *h = *is_q ? hh : (*is_v ? hh - p.Hq - p.Hkv : hh - p.Hq);
+  int hh;
+  rope_unit_split(p, unit, t, &hh);
+  rope_head_of(p, hh, h, is_q, is_v);
 }
 
 template <int DT, int D, bool QKNORM>
@@ -342,35 +366,48 @@ __device__ __forceinline__ void rope_rows(const RopeParams& p, const int64_t rb,
   const int64_t nunits = p.T * p.NH;
   const int64_t u0 = rb * (int64_t)(G * K) + g;
   if (u0 >= nunits) return;
+  // rows u0 + G * j: token and head-row of the first by one division, the rest by stepping
+  int64_t t0;
+  int hh0;
+  rope_unit_split(p, u0, &t0, &hh0);
   uint4 raw[K];
+  {
+    int64_t t = t0;
+    int hh = hh0;
 #pragma unroll
-  for (int j = 0; j < K; ++j) {
-    const int64_t u = u0 + (int64_t)G * j;
-    if (u < nunits) {
-      int64_t t;
-      int h;
-      bool is_q, is_v;
-      rope_row_where<DT, D>(p, u, &t, &h, &is_q, &is_v);
-      const char* src = is_q ? row_ptr(p.q, t, p.q_rs, EB) : is_v ? row_ptr(p.v, t, p.v_rs, EB)
-                                                                 : row_ptr(p.k, t, p.k_rs, EB);
-      src += ((int64_t)h * D + lane * VE) * EB;
-      raw[j] = is_q ? ld16(src) : ldg16(src);
+    for (int j = 0; j < K; ++j) {
+      if (j > 0) {
+        hh += G;
+        while (hh >= p.NH) { hh -= p.NH; ++t; }
+      }
+      if (u0 + (int64_t)G * j < nunits) {
+        int h;
+        bool is_q, is_v;
+        rope_head_of(p, hh, &h, &is_q, &is_v);
+        const char* src = is_q ? row_ptr(p.q, t, p.q_rs, EB) : is_v ? row_ptr(p.v, t, p.v_rs, EB)
+                                                                   : row_ptr(p.k, t, p.k_rs, EB);
+        src += ((int64_t)h * D + lane * VE) * EB;
+        raw[j] = is_q ? ld16(src) : ldg16(src);
+      }
     }
   }
-  const int64_t t0 = u0 / p.NH;
   const int32_t pos0 = __ldg(p.pos + t0);
   float sn[VE], cs[VE];
 #pragma unroll
   for (int e = 0; e < VE; ++e) rope_sincos((float)pos0, fq[2 * e], fq[2 * e + 1], &sn[e], &cs[e]);
   const bool low = lane < HALF;
+  int64_t t = t0;
+  int hh = hh0;
 #pragma unroll
   for (int j = 0; j < K; ++j) {
-    const int64_t u = u0 + (int64_t)G * j;
-    if (u >= nunits) break;
-    int64_t t;
+    if (j > 0) {
+      hh += G;
+      while (hh >= p.NH) { hh -= p.NH; ++t; }
+    }
+    if (u0 + (int64_t)G * j >= nunits) break;
     int h;
     bool is_q, is_v;
-    rope_row_where<DT, D>(p, u, &t, &h, &is_q, &is_v);
+    rope_head_of(p, hh, &h, &is_q, &is_v);
     // units ascend, so once a row belongs to a later token every following row does too
     const bool same = t == t0;
     const int32_t pos = same ? pos0 : __ldg(p.pos + t);

@@ -78,6 +78,8 @@ struct RopeParams {
   int32_t Hq, Hkv, D, NH;  // NH = Hq + 2 Hkv head-rows per token
   float eps, inv_D;
   int32_t prefetch;
+  uint32_t nh_magic;  // unit / NH for units below 2^32 without a divide: see rope_unit_split
+  int32_t nh_shift;
 };
 
 // out = silu(g) * u over T rows of I elements.

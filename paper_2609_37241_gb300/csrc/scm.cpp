@@ -603,6 +603,16 @@ void pack_pointwise(const trident_args* a, const Sig& s, PointwiseParams* p) {
   p->prefetch = 0;
 }
 
+// Round-up multiplier and shift for dividing 32-bit unsigned integers by d (2 <= d < 2^31):
+// l = ceil(log2 d), m = floor(2^32 (2^l - d) / d) + 1; the kernels take the quotient as
+// (h + ((n - h) >> 1)) >> (l - 1) with h = umulhi(n, m) (Granlund and Montgomery, 1994).
+void div_magic(uint32_t d, uint32_t* m, int32_t* l) {
+  int32_t s = 0;
+  while ((1ull << s) < d) ++s;
+  *m = (uint32_t)(((1ull << 32) * ((1ull << s) - d)) / d + 1);
+  *l = s;
+}
+
 void pack_rope(const trident_args* a, int base, int gq, const Version& v, uint32_t* err,
                RopeParams* p) {
   const trident_tensor* t = a->t;
@@ -620,6 +630,7 @@ void pack_rope(const trident_args* a, int base, int gq, const Version& v, uint32
   p->Hkv = (int32_t)t[base + 1].shape[1];
   p->D = (int32_t)t[base].shape[2];
   p->NH = p->Hq + 2 * p->Hkv;
+  div_magic((uint32_t)p->NH, &p->nh_magic, &p->nh_shift);
   p->eps = (float)a->eps;
   p->inv_D = (float)(1.0 / (double)p->D);
   p->prefetch = 0;
