@@ -160,6 +160,17 @@ __device__ __forceinline__ void chain_swiglu(const ChainParams& c, const int64_t
   swiglu_tile<DT, SWU>(c.sw, row, col_tile * SWU * kThreads, threadIdx.x);
 }
 
+// Row of SwiGLU tile `tile`. A single call's kernel (SWU = kChainSwigluUnroll) divides by
+// the host's multiplier (fast_div: the 64-token layer step 3.32 -> 3.29 us); the whole-step
+// kernel (SWU = kChainStepSwigluUnroll), which reads its call's parameters at a block-varying
+// index, keeps the division (the multiplier measured 3-5 % slower there).
+static_assert(kChainSwigluUnroll != kChainStepSwigluUnroll, "the tile width tells the kernels apart");
+template <int SWU>
+__device__ __forceinline__ int64_t swiglu_tile_row(const ChainParams& c, const int64_t tile) {
+  if (SWU == kChainStepSwigluUnroll) return tile / c.sw_tiles_per_row;
+  return fast_div((uint32_t)tile, c.sw_magic, c.sw_shift);
+}
+
 // Block b of one call's role-major grid (b < nA + nB + nC): [norms | RoPE | SwiGLU].
 template <int DT, int VPT, int SPLIT, int D, bool QKNORM, int SWU>
 __device__ __forceinline__ void chain_block(const ChainParams& c, const int b, const float* fq) {
@@ -171,7 +182,7 @@ __device__ __forceinline__ void chain_block(const ChainParams& c, const int b, c
   } else {
     const int64_t tile = b - c.nA - c.nB;
     if (tile >= c.sw_tiles) return;
-    const int64_t row = tile / c.sw_tiles_per_row;
+    const int64_t row = swiglu_tile_row<SWU>(c, tile);
     chain_swiglu<DT, SWU>(c, row, tile - row * c.sw_tiles_per_row);
   }
 }
@@ -254,7 +265,7 @@ __device__ __forceinline__ void chain_prefetch(const ChainParams& c, const int b
   } else {
     const int64_t tile = b - c.nA - c.nB;
     if (tile >= c.sw_tiles) return;
-    const int64_t row = tile / c.sw_tiles_per_row;
+    const int64_t row = swiglu_tile_row<SWU>(c, tile);
     swiglu_prefetch<DT, SWU>(c.sw, row, (tile - row * c.sw_tiles_per_row) * SWU * kThreads, tid);
   }
 }

@@ -179,16 +179,23 @@ __device__ __forceinline__ void rope_sincos(float pos, float fhi, float flo, flo
 }
 
 // ---------------------------------------------------------------- RoPE head-row
-// Token and head-row of a unit: unit = t * NH + hh. A division by a runtime divisor is a
-// long instruction sequence; for units below 2^32 (every grid in practice) the quotient comes
-// from the host's round-up multiplier for NH (Granlund and Montgomery, "Division by invariant
-// integers using multiplication", 1994): t = (h + ((u - h) >> 1)) >> (shift - 1) with
-// h = umulhi(u, magic), exact for every 32-bit u.
+// n / d for a 32-bit n and a divisor d known per launch, from the host's round-up multiplier
+// m and shift l for d (div_magic; Granlund and Montgomery, "Division by invariant integers
+// using multiplication", 1994): (h + ((n - h) >> 1)) >> (l - 1) with h = umulhi(n, m), exact
+// for every 32-bit n; l = 0 stands for d = 1. A division by a runtime divisor is otherwise a
+// long instruction sequence (64-bit: several times longer).
+__device__ __forceinline__ uint32_t fast_div(uint32_t n, uint32_t m, int32_t l) {
+  if (l == 0) return n;
+  const uint32_t h = __umulhi(n, m);
+  return (h + ((n - h) >> 1)) >> (l - 1);
+}
+
+// Token and head-row of a unit: unit = t * NH + hh (units below 2^32, every grid in practice,
+// by fast_div).
 __device__ __forceinline__ void rope_unit_split(const RopeParams& p, int64_t unit, int64_t* t, int* hh) {
   if (unit <= 0xffffffffll) {
     const uint32_t u = (uint32_t)unit;
-    const uint32_t h = __umulhi(u, p.nh_magic);
-    const uint32_t q = (h + ((u - h) >> 1)) >> (p.nh_shift - 1);
+    const uint32_t q = fast_div(u, p.nh_magic, p.nh_shift);
     *t = q;
     *hh = (int)(u - q * (uint32_t)p.NH);
   } else {

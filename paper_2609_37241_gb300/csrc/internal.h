@@ -78,7 +78,7 @@ struct RopeParams {
   int32_t Hq, Hkv, D, NH;  // NH = Hq + 2 Hkv head-rows per token
   float eps, inv_D;
   int32_t prefetch;
-  uint32_t nh_magic;  // unit / NH for units below 2^32 without a divide: see rope_unit_split
+  uint32_t nh_magic;  // unit / NH for units below 2^32 by fast_div
   int32_t nh_shift;
 };
 
@@ -106,6 +106,8 @@ struct ChainParams {
   int32_t tok_grid;  // 1: grid (a_split + rope_per_tok + sw_tiles_per_row, T), token-major
   int32_t rope_per_tok;  // RoPE blocks per token (token-major grid: nB = T * rope_per_tok)
   int32_t rope_k;    // head-rows per RoPE lane group: 1, or 3 on grids several waves long
+  uint32_t sw_magic;  // tile / sw_tiles_per_row by fast_div
+  int32_t sw_shift;
   int64_t sw_tiles;  // T * sw_tiles_per_row (valid SwiGLU tiles)
 };
 

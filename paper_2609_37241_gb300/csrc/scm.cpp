@@ -603,9 +603,10 @@ void pack_pointwise(const trident_args* a, const Sig& s, PointwiseParams* p) {
   p->prefetch = 0;
 }
 
-// Round-up multiplier and shift for dividing 32-bit unsigned integers by d (2 <= d < 2^31):
+// Round-up multiplier and shift for dividing 32-bit unsigned integers by d (1 <= d < 2^31):
 // l = ceil(log2 d), m = floor(2^32 (2^l - d) / d) + 1; the kernels take the quotient as
-// (h + ((n - h) >> 1)) >> (l - 1) with h = umulhi(n, m) (Granlund and Montgomery, 1994).
+// (h + ((n - h) >> 1)) >> (l - 1) with h = umulhi(n, m) (fast_div; Granlund and Montgomery,
+// 1994), and l = 0 (d = 1) as n itself.
 void div_magic(uint32_t d, uint32_t* m, int32_t* l) {
   int32_t s = 0;
   while ((1ull << s) < d) ++s;
@@ -697,6 +698,7 @@ int32_t pack_chain(trident_scm* scm, const Version& v, const trident_args* a, co
   c->nB = (int32_t)nB;
   c->nC = (int32_t)nC;
   c->sw_tiles_per_row = (int32_t)tiles;
+  div_magic((uint32_t)tiles, &c->sw_magic, &c->sw_shift);
   c->sw_tiles = nC;
   c->prefetch = 0;
   c->tok_grid = 0;
