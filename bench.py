@@ -316,14 +316,18 @@ def max_over_ranks(x, world, device="cpu"):
     return float(t.item())
 
 
-def time_steps(c, fn, K, W):
+def time_steps(c, fn, K, W, lead_cycles=0):
     """Runs fn(i) for W warm-up then K timed steps; returns (us per step on the device
-    clock, host us per step)."""
+    clock, host us per step). With lead_cycles, a sleep kernel of that many cycles runs
+    ahead of the first timed step (outside the window), so the window opens on a busy
+    device with the first steps already queued."""
     t = c.torch
     for i in range(W):
         fn(i)
     t.cuda.synchronize()
     e0, e1 = c.events()
+    if lead_cycles:
+        t.cuda._sleep(lead_cycles)
     h0 = time.perf_counter()
     e0.record(c.stream)
     for i in range(K):
@@ -1103,17 +1107,20 @@ def bench_chain_large(c, reps=10):
     return out
 
 
-def kernel_duration_chain(c, cfg, T, reps=200):
-    """Average duration of the fused chain kernel: `reps` launches issued back to back by
-    one native call (device-bound), CUDA events on the launching stream."""
+def kernel_duration_chain(c, cfg, T, calls=40):
+    """Average duration of the fused chain kernel: one launch per rotating input set, issued
+    back to back by one native call (device-bound), `calls` such calls timed with CUDA events
+    on the launching stream after a lead kernel (so the window holds about a thousand launches
+    of a busy device, not the first launch of an idle one)."""
     S = c.S
     sets = ChainSets(c, cfg, T)
     scm = layer_scm(c, cfg)
-    n = min(reps, sets.R)
+    n = sets.R
     arr = (S.trident_args * n)(*[sets.fused_args(c, i) for i in range(n)])
-    us, _ = time_steps(c, lambda i: c.L.trident_scm_invoke_seq(scm.h, arr, n, c.sp, None), 5, 3)
+    us, _ = time_steps(c, lambda i: c.L.trident_scm_invoke_seq(scm.h, arr, n, c.sp, None), calls, 3,
+                       lead_cycles=HEADLINE_LEAD_CYCLES)
     assert_all_hit(scm, "roofline kernel")
-    c.launches += 8 * n
+    c.launches += (calls + 3) * n
     scm.close()
     return us / n
 
