@@ -160,19 +160,18 @@ __device__ __forceinline__ void chain_swiglu(const ChainParams& c, const int64_t
   swiglu_tile<DT, SWU>(c.sw, row, col_tile * SWU * kThreads, threadIdx.x);
 }
 
-// Row of SwiGLU tile `tile`. A single call's kernel (SWU = kChainSwigluUnroll) divides by
-// the host's multiplier (fast_div: the 64-token layer step 3.32 -> 3.29 us); the whole-step
-// kernel (SWU = kChainStepSwigluUnroll), which reads its call's parameters at a block-varying
-// index, keeps the division (the multiplier measured 3-5 % slower there).
-static_assert(kChainSwigluUnroll != kChainStepSwigluUnroll, "the tile width tells the kernels apart");
-template <int SWU>
+// Row of SwiGLU tile `tile`. A single call's kernel divides by the host's multiplier
+// (fast_div: the 64-token layer step 3.32 -> 3.29 us); the whole-step kernel (STEP), which
+// reads its call's parameters at a block-varying index, keeps the division (the multiplier
+// measured 3-5 % slower there).
+template <bool STEP>
 __device__ __forceinline__ int64_t swiglu_tile_row(const ChainParams& c, const int64_t tile) {
-  if (SWU == kChainStepSwigluUnroll) return tile / c.sw_tiles_per_row;
+  if (STEP) return tile / c.sw_tiles_per_row;
   return fast_div((uint32_t)tile, c.sw_magic, c.sw_shift);
 }
 
 // Block b of one call's role-major grid (b < nA + nB + nC): [norms | RoPE | SwiGLU].
-template <int DT, int VPT, int SPLIT, int D, bool QKNORM, int SWU>
+template <int DT, int VPT, int SPLIT, int D, bool QKNORM, int SWU, bool STEP>
 __device__ __forceinline__ void chain_block(const ChainParams& c, const int b, const float* fq) {
   if (b < c.nA) {
     const int64_t row = b / SPLIT;
@@ -182,7 +181,7 @@ __device__ __forceinline__ void chain_block(const ChainParams& c, const int b, c
   } else {
     const int64_t tile = b - c.nA - c.nB;
     if (tile >= c.sw_tiles) return;
-    const int64_t row = swiglu_tile_row<SWU>(c, tile);
+    const int64_t row = swiglu_tile_row<STEP>(c, tile);
     chain_swiglu<DT, SWU>(c, row, tile - row * c.sw_tiles_per_row);
   }
 }
@@ -250,7 +249,7 @@ __device__ __forceinline__ void norm_rope_prefetch(const ChainParams& c, const i
 // prefetch == 1: every block its own first lines; prefetch == 2: only the norm blocks, which
 // take their token's rows and its RoPE head-rows (the other roles' own prefetches, issued by
 // hundreds of blocks while the previous kernel finishes, measured slower).
-template <int DT, int VPT, int SPLIT, int D, int SWU>
+template <int DT, int VPT, int SPLIT, int D, int SWU, bool STEP>
 __device__ __forceinline__ void chain_prefetch(const ChainParams& c, const int b) {
   constexpr int LPH = D / Act<DT>::VE;
   const int tid = threadIdx.x;
@@ -265,7 +264,7 @@ __device__ __forceinline__ void chain_prefetch(const ChainParams& c, const int b
   } else {
     const int64_t tile = b - c.nA - c.nB;
     if (tile >= c.sw_tiles) return;
-    const int64_t row = swiglu_tile_row<SWU>(c, tile);
+    const int64_t row = swiglu_tile_row<STEP>(c, tile);
     swiglu_prefetch<DT, SWU>(c.sw, row, (tile - row * c.sw_tiles_per_row) * SWU * kThreads, tid);
   }
 }
@@ -293,12 +292,12 @@ __device__ __forceinline__ void chain_prefetch_tok(const ChainParams& c) {
 // norm block per SM, instead of filling each slot the moment it frees (up to four norm
 // blocks on one SM). The trigger is otherwise the kernel's first instruction: even one
 // parameter read ahead of it measured 0.05 us slower per launch.
-template <int DT, int VPT, int SPLIT, int D, bool QKNORM, bool LATE>
+template <int DT, int VPT, int SPLIT, int D, bool QKNORM, bool LATE, int SWU>
 __global__ void __launch_bounds__(kThreads, VPT == 2 ? 4 : 2)
     chain_kernel(const __grid_constant__ ChainParams c) {
   if (!LATE || (int)blockIdx.x < c.nA) pdl_trigger();
   float fq[2 * Act<DT>::VE];
-  if (!LATE && c.tok_grid) {
+  if (!LATE && SWU == kChainSwigluUnroll && c.tok_grid) {
     if (c.prefetch) chain_prefetch_tok<DT, VPT, SPLIT, D>(c);
     chain_rope_freqs<DT, D>(c, (int)blockIdx.x >= SPLIT && (int)blockIdx.x < SPLIT + c.rope_per_tok, fq);
     pdl_wait();
@@ -307,10 +306,10 @@ __global__ void __launch_bounds__(kThreads, VPT == 2 ? 4 : 2)
     // A role-major grid fills the GPU: its RoPE blocks become resident only as the previous
     // kernel's blocks retire, and their frequency loads measured faster after the wait.
     const int b = blockIdx.x;
-    if (c.prefetch) chain_prefetch<DT, VPT, SPLIT, D, kChainSwigluUnroll>(c, b);
+    if (c.prefetch) chain_prefetch<DT, VPT, SPLIT, D, SWU, false>(c, b);
     pdl_wait();
     chain_rope_freqs<DT, D>(c, b >= c.nA && b < c.nA + c.nB, fq);
-    chain_block<DT, VPT, SPLIT, D, QKNORM, kChainSwigluUnroll>(c, b, fq);
+    chain_block<DT, VPT, SPLIT, D, QKNORM, SWU, false>(c, b, fq);
   }
 }
 
@@ -329,25 +328,27 @@ __global__ void __launch_bounds__(kThreads, VPT == 2 ? 4 : 2)
   }
   const ChainParams& c = p.c[lo];
   const int bl = b - p.first[lo];
-  if (c.prefetch) chain_prefetch<DT, VPT, SPLIT, D, kChainStepSwigluUnroll>(c, bl);
+  if (c.prefetch) chain_prefetch<DT, VPT, SPLIT, D, kChainStepSwigluUnroll, true>(c, bl);
   float fq[2 * Act<DT>::VE];
   chain_rope_freqs<DT, D>(c, bl >= c.nA && bl < c.nA + c.nB, fq);
   pdl_wait();
-  chain_block<DT, VPT, SPLIT, D, QKNORM, kChainStepSwigluUnroll>(c, bl, fq);
+  chain_block<DT, VPT, SPLIT, D, QKNORM, kChainStepSwigluUnroll, true>(c, bl, fq);
 }
 
 template <int DT, int SPLIT, bool QK>
-static void pick(int64_t H, const void** one, const void** step, const void** late) {
-  // late: the LATE entry, for the two-blocks-per-token split only (nullptr for SPLIT 1)
+static void pick(int64_t H, const void** one, const void** step, const void** extra) {
+  // extra: for SPLIT 2 the LATE entry, for SPLIT 1 the wide-tile entry
   constexpr int per = kThreads * Act<DT>::VE;
   if (H == per * 2) {
-    *one = (const void*)chain_kernel<DT, 2, SPLIT, 128, QK, false>;
+    *one = (const void*)chain_kernel<DT, 2, SPLIT, 128, QK, false, kChainSwigluUnroll>;
     *step = (const void*)chain_step_kernel<DT, 2, SPLIT, 128, QK>;
-    if constexpr (SPLIT == 2) *late = (const void*)chain_kernel<DT, 2, SPLIT, 128, QK, true>;
+    if constexpr (SPLIT == 2) *extra = (const void*)chain_kernel<DT, 2, SPLIT, 128, QK, true, kChainSwigluUnroll>;
+    else *extra = (const void*)chain_kernel<DT, 2, SPLIT, 128, QK, false, kChainWideSwigluUnroll>;
   } else if (H == per * 4) {
-    *one = (const void*)chain_kernel<DT, 4, SPLIT, 128, QK, false>;
+    *one = (const void*)chain_kernel<DT, 4, SPLIT, 128, QK, false, kChainSwigluUnroll>;
     *step = (const void*)chain_step_kernel<DT, 4, SPLIT, 128, QK>;
-    if constexpr (SPLIT == 2) *late = (const void*)chain_kernel<DT, 4, SPLIT, 128, QK, true>;
+    if constexpr (SPLIT == 2) *extra = (const void*)chain_kernel<DT, 4, SPLIT, 128, QK, true, kChainSwigluUnroll>;
+    else *extra = (const void*)chain_kernel<DT, 4, SPLIT, 128, QK, false, kChainWideSwigluUnroll>;
   }
 }
 
@@ -360,23 +361,24 @@ bool chain_kernel(int32_t dtype, int64_t H, int32_t D, bool qknorm, KernelEntry*
   out->unroll = kChainSwigluUnroll;
   // fn: two blocks per token for the norms; fn_late: the same with the late launch trigger;
   // fn_inplace: one block per token (calls whose outputs overwrite inputs, and grids too
-  // large for one wave); fn_step*: the same for several calls per launch
-  out->fn = out->fn_inplace = out->fn_step = out->fn_step_inplace = out->fn_late = nullptr;
+  // large for one wave); fn_wide: fn_inplace with wider SwiGLU tiles (grids of many waves);
+  // fn_step*: the same for several calls per launch
+  out->fn = out->fn_inplace = out->fn_step = out->fn_step_inplace = out->fn_late = out->fn_wide = nullptr;
   if (dtype == DT_BF16) {
     if (qknorm) {
       pick<DT_BF16, 2, true>(H, &out->fn, &out->fn_step, &out->fn_late);
-      pick<DT_BF16, 1, true>(H, &out->fn_inplace, &out->fn_step_inplace, nullptr);
+      pick<DT_BF16, 1, true>(H, &out->fn_inplace, &out->fn_step_inplace, &out->fn_wide);
     } else {
       pick<DT_BF16, 2, false>(H, &out->fn, &out->fn_step, &out->fn_late);
-      pick<DT_BF16, 1, false>(H, &out->fn_inplace, &out->fn_step_inplace, nullptr);
+      pick<DT_BF16, 1, false>(H, &out->fn_inplace, &out->fn_step_inplace, &out->fn_wide);
     }
   } else {
     if (qknorm) {
       pick<DT_FP16, 2, true>(H, &out->fn, &out->fn_step, &out->fn_late);
-      pick<DT_FP16, 1, true>(H, &out->fn_inplace, &out->fn_step_inplace, nullptr);
+      pick<DT_FP16, 1, true>(H, &out->fn_inplace, &out->fn_step_inplace, &out->fn_wide);
     } else {
       pick<DT_FP16, 2, false>(H, &out->fn, &out->fn_step, &out->fn_late);
-      pick<DT_FP16, 1, false>(H, &out->fn_inplace, &out->fn_step_inplace, nullptr);
+      pick<DT_FP16, 1, false>(H, &out->fn_inplace, &out->fn_step_inplace, &out->fn_wide);
     }
   }
   if (!out->fn) { *why = "layer chain supports H in {4096, 8192}"; return false; }

@@ -123,6 +123,9 @@ constexpr int kStepMax = 48;
 // the same change on single calls made them slower, 64 tokens 3.56 -> 4.09 us).
 constexpr int kChainSwigluUnroll = 2;
 constexpr int kChainStepSwigluUnroll = 4;
+// A single call's grid of many waves (one CTA per token) takes the wider tiles too: blocks
+// queue for slots there, and a tile that moves twice the bytes for the same fixed costs pays.
+constexpr int kChainWideSwigluUnroll = 4;
 struct ChainStepParams {
   int32_t n;
   int32_t first[kStepMax + 1];
@@ -134,6 +137,7 @@ struct KernelEntry {
   const void* fn = nullptr;
   const void* fn_inplace = nullptr;  // chain only: the entry for calls that write in place
   const void* fn_late = nullptr;     // chain only: fn with the late launch trigger (LATE)
+  const void* fn_wide = nullptr;     // chain only: fn_inplace with kChainWideSwigluUnroll tiles
   const void* fn_step = nullptr;          // chain only: several calls per launch (ChainStepParams)
   const void* fn_step_inplace = nullptr;  // ... one block per token for the norms
   const void* fn_large = nullptr;  // add+RMSNorm: the entry for calls of >= large_rows rows

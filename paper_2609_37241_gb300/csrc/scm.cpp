@@ -391,6 +391,7 @@ struct Version {
   CUfunction fn;
   CUfunction fn_inplace;  // layer chain: one block per token when outputs alias inputs
   CUfunction fn_late;     // layer chain: `fn` with the late launch trigger
+  CUfunction fn_wide;     // layer chain: `fn_inplace` with kChainWideSwigluUnroll tiles
   int32_t wave_blocks;    // layer chain: blocks of `fn` resident at once on the whole GPU
   CUfunction fn_large;          // add+RMSNorm: entry for calls of >= ke.large_rows rows
   CUfunction step_fn;           // layer chain: several calls per launch (two blocks per token)
@@ -684,6 +685,16 @@ void base_config(const trident_scm* scm, void* stream, CUlaunchConfig* cfg, CUla
 // counts, for SwiGLU tiles of `unroll` x 256 vectors (kChainSwigluUnroll in a call's own
 // launch, kChainStepSwigluUnroll in a whole-step launch). The norm split (set_chain_split)
 // is decided by the caller.
+// SwiGLU tiles of `unroll` x 256 vectors per row: their count, nC, and the row multiplier.
+void set_chain_tiles(ChainParams* c, int64_t T, int32_t unroll, int32_t vec) {
+  const int64_t per = (int64_t)unroll * kThreads * vec;
+  const int64_t tiles = (c->sw.I + per - 1) / per;
+  c->nC = (int32_t)(T * tiles);
+  c->sw_tiles_per_row = (int32_t)tiles;
+  div_magic((uint32_t)tiles, &c->sw_magic, &c->sw_shift);
+  c->sw_tiles = T * tiles;
+}
+
 int32_t pack_chain(trident_scm* scm, const Version& v, const trident_args* a, const Sig& s,
                    int32_t unroll, ChainParams* c) {
   pack_addnorm(a, C_H, C_R0, C_GA, C_X1, C_R1, s, K_ACT_H, &c->n1);
@@ -696,10 +707,7 @@ int32_t pack_chain(trident_scm* scm, const Version& v, const trident_args* a, co
   const int64_t nB = (s.T * c->rope.NH + upb - 1) / upb, nC = s.T * tiles;
   if (2 * s.T + nB + nC > 0x7fffffff) return fail(TRIDENT_ERR_INVALID, "layer chain too large for one launch");
   c->nB = (int32_t)nB;
-  c->nC = (int32_t)nC;
-  c->sw_tiles_per_row = (int32_t)tiles;
-  div_magic((uint32_t)tiles, &c->sw_magic, &c->sw_shift);
-  c->sw_tiles = nC;
+  set_chain_tiles(c, s.T, unroll, v.ke.vec);
   c->prefetch = 0;
   c->tok_grid = 0;
   c->rope_per_tok = 0;
@@ -769,6 +777,7 @@ int32_t do_launch(trident_scm* scm, const Version& v, const trident_args* a, con
   } P;
   void* kp[1] = {&P};
   bool late = false;  // layer chain: launch fn_late (the late launch trigger)
+  bool wide = false;  // layer chain: launch fn_wide (wider SwiGLU tiles)
   switch (op) {
     case TRIDENT_OP_ADD_RMSNORM:
       pack_addnorm(a, 0, 1, 2, 3, 4, s, K_ACT_H, &P.an);
@@ -820,7 +829,13 @@ int32_t do_launch(trident_scm* scm, const Version& v, const trident_args* a, con
       // while the grid still fits in one wave, and unless an output is written over an
       // input the partner CTA still reads (in-place calls keep one CTA per token).
       const int32_t split = (!chain_inplace(a) && 2 * s.T + c.nB + c.nC <= v.wave_blocks) ? 2 : 1;
-      const int32_t rope_k = split == 1 ? chain_rope_k(s.T + c.nB + c.nC, v.wave_blocks) : 1;
+      const int64_t one = s.T + c.nB + c.nC;  // one CTA per token, one head-row per lane group
+      const int32_t rope_k = split == 1 ? chain_rope_k(one, v.wave_blocks) : 1;
+      // Wider SwiGLU tiles (fn_wide) on grids of more than four waves: same-box probe, one
+      // Llama layer at 1024 / 4096 tokens 34.2 / 122.8 -> 31.3 / 112.6 us; at 256 tokens
+      // (3.4 waves) 9.81 -> 9.75 us, at 128 tokens (1.7 waves) 4.72 -> 5.11 us.
+      wide = split == 1 && v.fn_wide && one > 4 * (int64_t)v.wave_blocks;
+      if (wide) set_chain_tiles(&c, s.T, kChainWideSwigluUnroll, v.ke.vec);
       int64_t blocks = 0;
       st = set_chain_split(&c, s.T, split, rope_k, &blocks);
       if (st != TRIDENT_OK) return st;
@@ -876,7 +891,7 @@ int32_t do_launch(trident_scm* scm, const Version& v, const trident_args* a, con
   }
   CUfunction fn = v.fn;
   if ((op == TRIDENT_OP_LAYER_CHAIN || op == TRIDENT_OP_LAYER_CHAIN_QKNORM) && P.ch.a_split == 1)
-    fn = v.fn_inplace;
+    fn = wide ? v.fn_wide : v.fn_inplace;
   else if (late && v.fn_late)
     fn = v.fn_late;
   if (v.fn_large && s.T >= v.ke.large_rows) fn = v.fn_large;  // many rows: the bulk-copy kernel
@@ -1287,6 +1302,12 @@ int32_t append_version(trident_scm_t* scm, const trident_spec_desc* desc, int32_
           if (cudaGetFuncBySymbol(&l, v.ke.fn_late) != cudaSuccess || !l)
             return fail(TRIDENT_ERR_CUDA, "cannot resolve the late-trigger kernel entry");
           v.fn_late = reinterpret_cast<CUfunction>(l);
+        }
+        if (v.ke.fn_wide) {
+          cudaFunction_t w = nullptr;
+          if (cudaGetFuncBySymbol(&w, v.ke.fn_wide) != cudaSuccess || !w)
+            return fail(TRIDENT_ERR_CUDA, "cannot resolve the wide-tile kernel entry");
+          v.fn_wide = reinterpret_cast<CUfunction>(w);
         }
         cudaFunction_t h = nullptr, k = nullptr;
         if (cudaGetFuncBySymbol(&h, v.ke.fn_step) != cudaSuccess || !h ||
