@@ -9,13 +9,17 @@
 // horizontal fusion where blocks take different roles:
 //   norm     two add+RMSNorm steps, one or two blocks per token (the longest per-block
 //            work)
-//   RoPE     RoPE/KV head-rows, (256 / (D/8)) per block
-//   SwiGLU   tiles of one row each
-// A grid that fills the GPU is role-major ([norms | RoPE | SwiGLU], so the longest blocks
-// start first); a grid of at most one block per SM is token-major (chain_block_tok), so
-// consecutive blocks mix roles. One launch replaces four, which is what matters at decode
-// sizes, where each step moves well under a microsecond of HBM traffic. chain_step_kernel
-// runs several independent calls' grids in one launch.
+//   RoPE     RoPE/KV head-rows, (256 / (D/8)) per block, or three times that (three rows
+//            of one token per lane group) on grids several waves long
+//   SwiGLU   tiles of one row each, twice as wide on grids of many waves
+// Grids are role-major ([norms | RoPE | SwiGLU], so the longest blocks start first), the
+// smallest ones token-major (chain_block_tok), so that consecutive blocks mix roles. Under
+// programmatic dependent launch, role-major grids that fit the resident slots with their
+// own norm blocks run the LATE entry, whose short blocks trigger the next launch only at
+// their exit (the next grid is then placed one norm block per SM). One launch replaces
+// four, which is what matters at decode sizes, where each step moves well under a
+// microsecond of HBM traffic. chain_step_kernel runs several independent calls' grids in
+// one launch.
 #include "device_common.cuh"
 
 namespace trident {
