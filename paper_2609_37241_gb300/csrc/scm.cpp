@@ -841,7 +841,10 @@ int32_t do_launch(trident_scm* scm, const Version& v, const trident_args* a, con
       if (st != TRIDENT_OK) return st;
       cfg.gridDimX = (unsigned)blocks;
       // Under PDL, a role-major grid of more than a quarter block per SM whose blocks, with
-      // its own norm blocks, fit the resident slots launches fn_late: its RoPE and SwiGLU
+      // its own norm blocks, fit the resident slots (give or take an eighth of them: a few
+      // dozen blocks placed late cost less than the stacked norm blocks, Llama 56 tokens
+      // 3.31 -> 3.19 us, 36 Qwen3-style launches at 64 tokens 125.9 -> 122.3 us; 62 Llama
+      // tokens equal) launches fn_late: its RoPE and SwiGLU
       // blocks trigger the next launch at their exit, so the next grid is placed whole while
       // this one's norm blocks finish, one norm block per SM instead of up to four. Same-box
       // A/B of Llama layer steps against the token-major grid below: 6 tokens 2.22 -> 2.12
@@ -860,7 +863,7 @@ int32_t do_launch(trident_scm* scm, const Version& v, const trident_args* a, con
       // slower as well).
       const int64_t upb = rope_units_per_block(c.rope.D, 2);
       if ((scm->opt.flags & TRIDENT_OPT_PDL) && split == 2 && v.fn_late && 4 * blocks > scm->sm_count &&
-          blocks + c.nA <= v.wave_blocks) {
+          blocks + c.nA <= v.wave_blocks + v.wave_blocks / 8) {
         late = true;
       } else if (c.rope.NH % upb == 0 && s.T >= 1 && s.T <= 65535 && blocks <= 2 * scm->sm_count) {
         c.tok_grid = 1;
