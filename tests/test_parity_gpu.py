@@ -580,16 +580,16 @@ def test_layer_chain_unfused_four_invokes_match(S, pdl):
     check_chain(ref, out, inp)
 
 
-def test_layer_chain_in_place_and_bad_position(S):
+@pytest.mark.parametrize("T", [6, 700])  # 700: several waves (three-row RoPE lane groups, wide tiles)
+def test_layer_chain_in_place_and_bad_position(S, T):
     cfg = synth.LLAMA
-    T = 6
     g = np.random.default_rng(5)
     inp = synth.layer_inputs(g, T, cfg)
     inp["pos"][3] = cfg["S"] + 7  # out of range: token 3's rope/append skipped and flagged
     ref = L.layer_chain(inp, cfg["theta"], cfg["eps"], BF16)
     assert ref["bad"] == 1
     fixed = [cfg["H"], cfg["Hq"], cfg["Hkv"], cfg["D"], cfg["S"], cfg["I"]]
-    s = one_version_scm(S, S.make_spec(S.OP_LAYER_CHAIN, BF16, fixed, 1, 64, layout=S.LAYOUT_CONTIG,
+    s = one_version_scm(S, S.make_spec(S.OP_LAYER_CHAIN, BF16, fixed, 1, 1024, layout=S.LAYOUT_CONTIG,
                                        rope_theta=cfg["theta"]))
     ts, out = chain_device(inp, BF16, False, layout="separate")
     # in place: x1 = h, r1 = r0, x2 = attn_out, r2 = r1, o = g
