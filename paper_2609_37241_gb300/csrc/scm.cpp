@@ -841,26 +841,24 @@ int32_t do_launch(trident_scm* scm, const Version& v, const trident_args* a, con
       if (st != TRIDENT_OK) return st;
       cfg.gridDimX = (unsigned)blocks;
       // Under PDL, a role-major grid of more than a quarter block per SM whose blocks, with
-      // its own norm blocks, fit the resident slots (give or take an eighth of them: a few
-      // dozen blocks placed late cost less than the stacked norm blocks, Llama 56 tokens
-      // 3.31 -> 3.19 us, 36 Qwen3-style launches at 64 tokens 125.9 -> 122.3 us; 62 Llama
-      // tokens equal) launches fn_late: its RoPE and SwiGLU
-      // blocks trigger the next launch at their exit, so the next grid is placed whole while
-      // this one's norm blocks finish, one norm block per SM instead of up to four. Same-box
-      // A/B of Llama layer steps against the token-major grid below: 6 tokens 2.22 -> 2.12
-      // us, 8 tokens 2.33 -> 2.14, 16 tokens 2.58 -> 2.29, 24 tokens 3.19 -> 2.44, 32
-      // tokens 2.98 -> 2.57, 48 tokens (role-major before) 3.21 -> 2.99; equal at 2 and 4
-      // tokens, and at 1 token 1.5-2 % slower (nothing to place, and the next launch starts
-      // later), hence the lower bound; at 64 tokens, where 96 blocks would start late, the
-      // probe measured 3.51 -> 3.69 us, hence the upper one.
+      // its own norm blocks, fit the resident slots give or take an eighth of them launches
+      // fn_late: its RoPE and SwiGLU blocks trigger the next launch at their exit, so the
+      // next grid is placed whole while this one's norm blocks finish, one norm block per SM
+      // instead of up to four. Same-box A/B of Llama layer steps against the grids below: 6
+      // tokens 2.22 -> 2.12 us, 8 tokens 2.33 -> 2.14, 16 tokens 2.58 -> 2.29, 24 tokens
+      // 3.19 -> 2.44, 32 tokens 2.98 -> 2.57, 48 tokens 3.21 -> 2.99, 56 tokens 3.31 ->
+      // 3.19; equal at 2 and 4 tokens and at 1 token 1.5-2 % slower (nothing to place, and
+      // the next launch starts later), hence the lower bound; a few dozen blocks placed late
+      // cost less than stacked norm blocks (36 Qwen3-style launches at 64 tokens 125.9 ->
+      // 122.3 us, 62 Llama tokens equal), but at 64 Llama tokens, with 96 blocks placed late,
+      // the probe measured 3.51 -> 3.69 us, hence the upper bound.
       // Otherwise a token-major grid (chain_block_tok) for grids of at most two blocks per SM,
       // when every token has the same number of RoPE blocks: consecutive blocks then mix
       // roles, so the blocks that land together on one SM are not all norm blocks (measured
       // against role-major grids without the late trigger: 16 tokens 3.55 -> 2.85 us per
-      // layer step, 1 token 2.20 -> 2.04 us). A grid that nearly fills the GPU keeps the
-      // role-major order, which starts the longest (norm) blocks first (64 tokens: 3.98 us
-      // role-major, 4.05 us token-major; 48 and 64 tokens in other interleaved orders were
-      // slower as well).
+      // layer step, 1 token 2.20 -> 2.04 us). Larger grids are role-major, which starts the
+      // longest (norm) blocks first (64 tokens: 3.98 us role-major, 4.05 us token-major; 48
+      // and 64 tokens in other interleaved orders were slower as well).
       const int64_t upb = rope_units_per_block(c.rope.D, 2);
       if ((scm->opt.flags & TRIDENT_OPT_PDL) && split == 2 && v.fn_late && 4 * blocks > scm->sm_count &&
           blocks + c.nA <= v.wave_blocks + v.wave_blocks / 8) {
