@@ -609,6 +609,11 @@ void pack_pointwise(const trident_args* a, const Sig& s, PointwiseParams* p) {
 // (h + ((n - h) >> 1)) >> (l - 1) with h = umulhi(n, m) (fast_div; Granlund and Montgomery,
 // 1994), and l = 0 (d = 1) as n itself.
 void div_magic(uint32_t d, uint32_t* m, int32_t* l) {
+  if (d == 0) {  // no divisor: callers reject such calls first; stay defined regardless
+    *m = 0;
+    *l = 0;
+    return;
+  }
   int32_t s = 0;
   while ((1ull << s) < d) ++s;
   *m = (uint32_t)(((1ull << 32) * ((1ull << s) - d)) / d + 1);
@@ -1173,6 +1178,8 @@ int32_t trident::prepare_rope_args(const void* args_ptr, RopeParams* p, int32_t*
   if (!s.aux_dtype_ok) return fail(TRIDENT_ERR_INVALID, "gamma must be fp32 and pos int32");
   if (!s.ranks_ok || !s.shapes_ok) return fail(TRIDENT_ERR_INVALID, "inconsistent ranks or shapes");
   if (s.T < 1) return fail(TRIDENT_ERR_INVALID, "no tokens");
+  if (a->t[0].shape[1] < 1 || a->t[1].shape[1] < 1 || a->t[0].shape[2] < 1)
+    return fail(TRIDENT_ERR_INVALID, "no heads: q and k need at least one head of at least one element");
   if (s.layout < 0 || !s.aux_layout_ok) return fail(TRIDENT_ERR_INVALID, "unsupported layout");
   if (!s.aligned16) return fail(TRIDENT_ERR_INVALID, "tensors must be 16-byte aligned");
   if (!(a->rope_theta > 0.0 && std::isfinite(a->rope_theta)))

@@ -483,3 +483,16 @@ def test_nvtx_ranges_build_only_with_the_flag(S, tmp_path):
     subprocess.run([B.nvcc(), *B.ARCH, *B.FLAGS, "-DTRIDENT_NVTX", "-c", src, "-o", str(obj)], check=True)
     syms = subprocess.run(["nm", str(obj)], capture_output=True, text=True).stdout
     assert "nvtx" in syms.lower()
+
+
+def test_noalloc_rejects_calls_without_heads(S):
+    """The allocation-free RoPE entry validates its tuple on the host before any CUDA call: a
+    call whose q and k have no heads (nothing to map a unit to) is ERR_INVALID, as is a
+    malformed one, and neither needs a GPU."""
+    args = cases.make_args({"op": 2, "T": 4, "Hq": 0, "Hkv": 0, "D": 128, "S": 64})
+    st = S.trident_rope_kv_noalloc(cases.lib_args(dict(args, theta=1e4)), None)
+    assert st == S.ERR_INVALID and "no heads" in S.trident_scm_last_error()
+    args = cases.make_args({"op": 2, "T": 4, "Hq": 4, "Hkv": 2, "D": 128, "S": 64})
+    args["tensors"][3] = dict(args["tensors"][3], dtype=cases.DT["fp32"])  # positions must be int32
+    st = S.trident_rope_kv_noalloc(cases.lib_args(dict(args, theta=1e4)), None)
+    assert st == S.ERR_INVALID
