@@ -319,40 +319,63 @@ __global__ void __launch_bounds__(kThreads, VPT == 2 ? 4 : 2)
 
 // Several independent calls in one launch: a block finds its call by binary search over
 // the first-block table (uniform across the block, so the parameter reads broadcast).
-template <int DT, int VPT, int SPLIT, int D, bool QKNORM>
+// ROLE (one-CTA-per-token steps of one to two waves): role-major block order over the whole
+// step -- every call's norm blocks, then every call's RoPE blocks, then every call's SwiGLU
+// tiles -- so that the longer blocks fill the first wave (a separate entry: the call-major
+// kernel measured about 1 % slower with this branch in it).
+template <int DT, int VPT, int SPLIT, int D, bool QKNORM, bool ROLE>
 __global__ void __launch_bounds__(kThreads, VPT == 2 ? 4 : 2)
     chain_step_kernel(const __grid_constant__ ChainStepParams p) {
   pdl_trigger();
   const int b = blockIdx.x;
   int lo = 0, hi = p.n - 1;
-  while (lo < hi) {
-    const int mid = (lo + hi + 1) >> 1;
-    if (b >= p.first[mid]) lo = mid;
-    else hi = mid - 1;
+  if constexpr (ROLE) {
+    const int r = b < p.role_first[1][0] ? 0 : (b < p.role_first[2][0] ? 1 : 2);
+    const int32_t* f = p.role_first[r];
+    while (lo < hi) {
+      const int mid = (lo + hi + 1) >> 1;
+      if (b >= f[mid]) lo = mid;
+      else hi = mid - 1;
+    }
+    const ChainParams& c = p.c[lo];
+    const int bl = b - f[lo] + (r == 0 ? 0 : (r == 1 ? c.nA : c.nA + c.nB));
+    float fq[2 * Act<DT>::VE];
+    chain_rope_freqs<DT, D>(c, r == 1, fq);
+    pdl_wait();
+    chain_block<DT, VPT, SPLIT, D, QKNORM, kChainStepSwigluUnroll, true>(c, bl, fq);
+  } else {
+    while (lo < hi) {
+      const int mid = (lo + hi + 1) >> 1;
+      if (b >= p.first[mid]) lo = mid;
+      else hi = mid - 1;
+    }
+    const ChainParams& c = p.c[lo];
+    const int bl = b - p.first[lo];
+    if (c.prefetch) chain_prefetch<DT, VPT, SPLIT, D, kChainStepSwigluUnroll, true>(c, bl);
+    float fq[2 * Act<DT>::VE];
+    chain_rope_freqs<DT, D>(c, bl >= c.nA && bl < c.nA + c.nB, fq);
+    pdl_wait();
+    chain_block<DT, VPT, SPLIT, D, QKNORM, kChainStepSwigluUnroll, true>(c, bl, fq);
   }
-  const ChainParams& c = p.c[lo];
-  const int bl = b - p.first[lo];
-  if (c.prefetch) chain_prefetch<DT, VPT, SPLIT, D, kChainStepSwigluUnroll, true>(c, bl);
-  float fq[2 * Act<DT>::VE];
-  chain_rope_freqs<DT, D>(c, bl >= c.nA && bl < c.nA + c.nB, fq);
-  pdl_wait();
-  chain_block<DT, VPT, SPLIT, D, QKNORM, kChainStepSwigluUnroll, true>(c, bl, fq);
 }
 
 template <int DT, int SPLIT, bool QK>
-static void pick(int64_t H, const void** one, const void** step, const void** extra) {
-  // extra: for SPLIT 2 the LATE entry, for SPLIT 1 the wide-tile entry
+static void pick(int64_t H, const void** one, const void** step, const void** extra, const void** role) {
+  // extra: for SPLIT 2 the LATE entry, for SPLIT 1 the wide-tile entry; role: for SPLIT 1
+  // the role-major whole-step entry
   constexpr int per = kThreads * Act<DT>::VE;
   if (H == per * 2) {
     *one = (const void*)chain_kernel<DT, 2, SPLIT, 128, QK, false, kChainSwigluUnroll>;
-    *step = (const void*)chain_step_kernel<DT, 2, SPLIT, 128, QK>;
+    *step = (const void*)chain_step_kernel<DT, 2, SPLIT, 128, QK, false>;
     if constexpr (SPLIT == 2) *extra = (const void*)chain_kernel<DT, 2, SPLIT, 128, QK, true, kChainSwigluUnroll>;
     else *extra = (const void*)chain_kernel<DT, 2, SPLIT, 128, QK, false, kChainWideSwigluUnroll>;
+    if constexpr (SPLIT == 1) *role = (const void*)chain_step_kernel<DT, 2, SPLIT, 128, QK, true>;
   } else if (H == per * 4) {
     *one = (const void*)chain_kernel<DT, 4, SPLIT, 128, QK, false, kChainSwigluUnroll>;
-    *step = (const void*)chain_step_kernel<DT, 4, SPLIT, 128, QK>;
+    *step = (const void*)chain_step_kernel<DT, 4, SPLIT, 128, QK, false>;
     if constexpr (SPLIT == 2) *extra = (const void*)chain_kernel<DT, 4, SPLIT, 128, QK, true, kChainSwigluUnroll>;
     else *extra = (const void*)chain_kernel<DT, 4, SPLIT, 128, QK, false, kChainWideSwigluUnroll>;
+    if constexpr (SPLIT == 1) *role = (const void*)chain_step_kernel<DT, 4, SPLIT, 128, QK, true>;
   }
 }
 
@@ -366,23 +389,24 @@ bool chain_kernel(int32_t dtype, int64_t H, int32_t D, bool qknorm, KernelEntry*
   // fn: two blocks per token for the norms; fn_late: the same with the late launch trigger;
   // fn_inplace: one block per token (calls whose outputs overwrite inputs, and grids too
   // large for one wave); fn_wide: fn_inplace with wider SwiGLU tiles (grids of many waves);
-  // fn_step*: the same for several calls per launch
-  out->fn = out->fn_inplace = out->fn_step = out->fn_step_inplace = out->fn_late = out->fn_wide = nullptr;
+  // fn_step*: the same for several calls per launch (fn_step_role: role-major order)
+  out->fn = out->fn_inplace = out->fn_step = out->fn_step_inplace = out->fn_late = out->fn_wide =
+      out->fn_step_role = nullptr;
   if (dtype == DT_BF16) {
     if (qknorm) {
-      pick<DT_BF16, 2, true>(H, &out->fn, &out->fn_step, &out->fn_late);
-      pick<DT_BF16, 1, true>(H, &out->fn_inplace, &out->fn_step_inplace, &out->fn_wide);
+      pick<DT_BF16, 2, true>(H, &out->fn, &out->fn_step, &out->fn_late, nullptr);
+      pick<DT_BF16, 1, true>(H, &out->fn_inplace, &out->fn_step_inplace, &out->fn_wide, &out->fn_step_role);
     } else {
-      pick<DT_BF16, 2, false>(H, &out->fn, &out->fn_step, &out->fn_late);
-      pick<DT_BF16, 1, false>(H, &out->fn_inplace, &out->fn_step_inplace, &out->fn_wide);
+      pick<DT_BF16, 2, false>(H, &out->fn, &out->fn_step, &out->fn_late, nullptr);
+      pick<DT_BF16, 1, false>(H, &out->fn_inplace, &out->fn_step_inplace, &out->fn_wide, &out->fn_step_role);
     }
   } else {
     if (qknorm) {
-      pick<DT_FP16, 2, true>(H, &out->fn, &out->fn_step, &out->fn_late);
-      pick<DT_FP16, 1, true>(H, &out->fn_inplace, &out->fn_step_inplace, &out->fn_wide);
+      pick<DT_FP16, 2, true>(H, &out->fn, &out->fn_step, &out->fn_late, nullptr);
+      pick<DT_FP16, 1, true>(H, &out->fn_inplace, &out->fn_step_inplace, &out->fn_wide, &out->fn_step_role);
     } else {
-      pick<DT_FP16, 2, false>(H, &out->fn, &out->fn_step, &out->fn_late);
-      pick<DT_FP16, 1, false>(H, &out->fn_inplace, &out->fn_step_inplace, &out->fn_wide);
+      pick<DT_FP16, 2, false>(H, &out->fn, &out->fn_step, &out->fn_late, nullptr);
+      pick<DT_FP16, 1, false>(H, &out->fn_inplace, &out->fn_step_inplace, &out->fn_wide, &out->fn_step_role);
     }
   }
   if (!out->fn) { *why = "layer chain supports H in {4096, 8192}"; return false; }

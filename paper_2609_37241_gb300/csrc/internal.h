@@ -128,7 +128,9 @@ constexpr int kChainStepSwigluUnroll = 4;
 constexpr int kChainWideSwigluUnroll = 4;
 struct ChainStepParams {
   int32_t n;
-  int32_t first[kStepMax + 1];
+  int32_t first[kStepMax + 1];  // call-major: call i owns blocks [first[i], first[i+1])
+  int32_t role_first[3][kStepMax + 1];  // role-major: call i's norm / RoPE / SwiGLU blocks
+                                        // start at role_first[r][i]; [r][n] ends role r
   ChainParams c[kStepMax];
 };
 
@@ -138,6 +140,7 @@ struct KernelEntry {
   const void* fn_inplace = nullptr;  // chain only: the entry for calls that write in place
   const void* fn_late = nullptr;     // chain only: fn with the late launch trigger (LATE)
   const void* fn_wide = nullptr;     // chain only: fn_inplace with kChainWideSwigluUnroll tiles
+  const void* fn_step_role = nullptr;  // chain only: fn_step_inplace, role-major block order
   const void* fn_step = nullptr;          // chain only: several calls per launch (ChainStepParams)
   const void* fn_step_inplace = nullptr;  // ... one block per token for the norms
   const void* fn_large = nullptr;  // add+RMSNorm: the entry for calls of >= large_rows rows
