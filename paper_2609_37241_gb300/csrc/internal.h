@@ -113,7 +113,7 @@ struct ChainParams {
 
 // Several independent layer-chain calls in one launch (a decoder step's chains). Call i
 // owns blocks [first[i], first[i+1]); inside its range a block plays the same role as in
-// the single-call kernel. The struct is passed as the kernel parameter (about 21 KB, under
+// the single-call kernel. The struct is passed as the kernel parameter (about 25 KB, under
 // the 32 KB parameter limit), so no device buffer is written before the launch.
 constexpr int kStepMax = 48;
 // SwiGLU tile width of the layer chain's blocks, in 256-thread rounds of 16-byte vectors of
