@@ -510,8 +510,9 @@ def test_layer_chain_fused_matches_oracle(S, cfg_name, T, pdl):
 
 def test_layer_chain_largest_bucket(S):
     """The largest token count the benchmark's chain versions accept (4096 Llama tokens: a grid
-    of 32,768 blocks, one CTA per token for the norms, the norm-row and RoPE-row prefetch under
-    PDL), every output against the oracle."""
+    of 16,384 blocks several waves long -- one CTA per token for the norms, three head-rows per
+    RoPE lane group, SwiGLU tiles of 4 x 256 vectors -- with the norm-row prefetch under PDL),
+    every output against the oracle."""
     cfg = synth.LLAMA
     T = 4096
     g = np.random.default_rng(4096)
@@ -537,7 +538,8 @@ def test_layer_chain_largest_bucket(S):
     # to two tokens (the H 8192 case above covers it with q/k norm, 80 head-rows per token)
     (BF16, 4096, 20, 14336, 300, False),
 ])
-def test_layer_chain_other_sizes_and_dtypes(S, dtype, H, Hq, I, T, qk):
+@pytest.mark.parametrize("pdl", [False, True], ids=["plain", "pdl"])  # PDL: token-major / late trigger
+def test_layer_chain_other_sizes_and_dtypes(S, dtype, H, Hq, I, T, qk, pdl):
     cfg = dict(H=H, Hq=Hq, Hkv=8, D=128, S=2048, I=I, theta=1e6, qknorm=qk, eps=1e-6)
     g = np.random.default_rng(H + T)
     inp = synth.layer_inputs(g, T, cfg, dtype=dtype)
@@ -545,7 +547,8 @@ def test_layer_chain_other_sizes_and_dtypes(S, dtype, H, Hq, I, T, qk):
     op = S.OP_LAYER_CHAIN_QKNORM if qk else S.OP_LAYER_CHAIN
     fixed = [H, Hq, 8, 128, 2048, I]
     lay = S.LAYOUT_ROWSTRIDED if T > 1 else S.LAYOUT_CONTIG
-    s = one_version_scm(S, S.make_spec(op, dtype, fixed, 1, 4096, layout=lay, rope_theta=cfg["theta"]))
+    s = one_version_scm(S, S.make_spec(op, dtype, fixed, 1, 4096, layout=lay, rope_theta=cfg["theta"]),
+                        flags=S.OPT_PDL if pdl else 0)
     ts, out = chain_device(inp, dtype, qk)
     invoke_ok(s, S, S.make_args(op, ts, eps=cfg["eps"], rope_theta=cfg["theta"]))
     torch.cuda.synchronize()
