@@ -87,6 +87,16 @@ def chain_bytes_per_token(cfg, fused=True):
     return norm1 + norm2 + rope + swiglu
 
 
+def chain_read_write_bytes(cfg, T):
+    """(read, write) split of the fused chain's algorithmic bytes per launch."""
+    H, Hq, Hkv, D, I = cfg["H"], cfg["Hq"], cfg["Hkv"], cfg["D"], cfg["I"]
+    rope_rows = (Hq + 2 * Hkv) * D * 2
+    read = 2 * H * 2 + H * 2 + rope_rows + 4 + 2 * I * 2
+    write = 2 * H * 2 + 2 * H * 2 + rope_rows + I * 2
+    g = 2 * H * 4 + (2 * D * 4 if cfg.get("qknorm") else 0) + D * 4
+    return T * read + g, T * write
+
+
 def chain_bytes_per_launch(cfg, T, fused=True):
     # norm weights (+ q/k norm weights) and the RoPE frequency table, once per launch
     g = 2 * cfg["H"] * 4 + (2 * cfg["D"] * 4 if cfg.get("qknorm") else 0) + cfg["D"] * 4
@@ -1125,6 +1135,33 @@ def kernel_duration_chain(c, cfg, T, calls=40):
     return us / n
 
 
+def copy_floor(c, cfg, T, blocks_list=(152, 304, 456, 512, 576, 608, 640, 760, 912, 1216), calls=40):
+    """The copy floor for the chain's traffic: a plain streaming kernel that reads and writes
+    the same byte counts as one fused-chain launch at T tokens (the read sum XORed per thread,
+    the write a store of it), launched the same way -- PDL with an L2 prefetch before the
+    wait, one launch per rotating input set, `calls` native calls of `sets` launches after a
+    lead kernel. Gives, per grid size, the per-launch time the GPU needs for this traffic
+    with no arithmetic, no gathers and no role mix."""
+    torch, S = c.torch, c.S
+    rb, wb = chain_read_write_bytes(cfg, T)
+    rb, wb = (rb + 15) // 16 * 16, (wb + 15) // 16 * 16
+    sets = max(2, -(-2 * L2_BYTES // (rb + wb)))
+    src = torch.randint(-2 ** 31, 2 ** 31 - 1, (sets * rb // 4,), dtype=torch.int32, device=c.dev)
+    dst = torch.empty((sets * wb // 4,), dtype=torch.int32, device=c.dev)
+    scm = S.Scm(device=c.dev.index or 0, flags=S.OPT_PDL)
+    out = dict(read_bytes=int(rb), write_bytes=int(wb), sets=int(sets), launches_per_call=int(sets), grids={})
+    for blocks in blocks_list:
+        def call(i, blocks=blocks):
+            st = S.trident_copy_floor(scm.h, c.sp, src.data_ptr(), dst.data_ptr(), rb, wb, blocks, sets, sets)
+            assert st == S.OK, S.trident_scm_last_error()
+        us, _ = time_steps(c, call, calls, 3, lead_cycles=HEADLINE_LEAD_CYCLES)
+        c.launches += (calls + 3) * sets
+        out["grids"][str(blocks)] = round(us / sets, 3)
+    scm.close()
+    del src, dst
+    return out
+
+
 _T0 = time.perf_counter()
 
 
@@ -1251,6 +1288,13 @@ def run_ours(a):
                                  traffic_write=None if tr is None else tr[1],
                                  kernel="chain_kernel<bf16,H4096,D128>",
                                  bytes_per_launch=int(b), us_per_launch=round(kd, 3), peak_source=src)
+        progress("copy floor")
+        cf = copy_floor(c, cfg, HEADLINE_T)
+        best = min(cf["grids"].values())
+        cf.update(frac_of_peak={k: round((cf["read_bytes"] + cf["write_bytes"]) / v / 1e3 / peak, 3)
+                                for k, v in cf["grids"].items()},
+                  chain_over_best_copy=round(best / kd, 3))
+        extra["roofline"]["copy_floor"] = cf
     if rank == 0 and want("e2e"):
         progress("e2e")
         extra["e2e"] = bench_e2e(c, cfg, HEADLINE_T, K=min(K, 500), W=W)

@@ -474,6 +474,21 @@ int32_t trident_scm_host_times(const trident_scm_t* scm, uint32_t* out, int32_t 
  * ERR_INVALID (scm NULL or n < 0), ERR_STATE (dry-run SCM), ERR_CUDA. */
 int32_t trident_launch_floor(trident_scm_t* scm, void* stream, int32_t n);
 
+/* Copy-floor probe (measurement, not part of the dispatch path): n launches, back to back on
+ * `stream` through the same launch code as a hit, of a kernel with a layer chain's traffic
+ * and none of its arithmetic. Launch i reads read_bytes at src + (i % sets) * read_bytes and
+ * writes write_bytes at dst + (i % sets) * write_bytes with a grid of `blocks` blocks of 256
+ * threads: block b reads its even share of the 16-byte vectors and writes its even share,
+ * every written vector the XOR of the vectors its thread read; with TRIDENT_OPT_PDL each
+ * block first prefetches its read lines into L2 before its programmatic-launch wait, as the
+ * layer chain's blocks do. Give it the bytes, block count and rotation of a chain launch and
+ * the time per launch is what this GPU needs to move that traffic in that launch pattern: the
+ * floor the chain kernel is read against. src and dst are device pointers (caller-owned,
+ * 16-byte aligned, sets * read_bytes and sets * write_bytes long); the byte counts are
+ * multiples of 16. Errors: ERR_INVALID (bad arguments), ERR_STATE (dry-run SCM), ERR_CUDA. */
+int32_t trident_copy_floor(trident_scm_t* scm, void* stream, const void* src, void* dst, int64_t read_bytes,
+                           int64_t write_bytes, int32_t blocks, int32_t sets, int32_t n);
+
 /* Reads the device status word (TRIDENT_DEVERR_* bits) after synchronising `stream`;
  * clears it when clear != 0. Errors: ERR_STATE in dry-run mode, ERR_CUDA. */
 int32_t trident_scm_device_status(trident_scm_t* scm, void* stream, uint32_t* out_bits,

@@ -17,7 +17,7 @@ LIBDIR = os.path.join(PKG, "_lib")
 LIB = os.path.join(LIBDIR, "libtrident_scm.so")
 SOURCES = ["scm.cpp", "tree.cpp", "addnorm.cu", "rmsnorm.cu", "rope.cu", "swiglu.cu", "pointwise.cu", "chain.cu",
            "noalloc.cu"]
-HEADERS = ["internal.h", "device_common.cuh", "tree.h"]
+HEADERS = ["internal.h", "device_common.cuh", "tree.h", "measure.h"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC,-fvisibility=hidden",
          "-I", INC, "-I", CSRC]

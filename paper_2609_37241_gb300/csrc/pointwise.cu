@@ -6,6 +6,7 @@
 // UNROLL * 256 16-byte vectors, all loads of a tile issued before the first use (grid.y
 // walks the rows); the generic kernel is a flat grid-stride loop with scalar accesses.
 #include "device_common.cuh"
+#include "measure.h"
 
 namespace trident {
 
@@ -138,6 +139,34 @@ __global__ void empty_kernel() {
 }
 
 const void* empty_kernel_entry() { return (const void*)empty_kernel; }
+
+// Copy-floor probe (trident_copy_floor), see CopyFloorParams. With prefetch, a block's read
+// lines go to L2 between the launch trigger and the wait, as the layer chain's blocks do.
+__global__ void __launch_bounds__(kThreads) copy_floor_kernel(const CopyFloorParams p) {
+  pdl_trigger();
+  const int64_t g = gridDim.x;
+  const int64_t rpb = (p.nr + g - 1) / g, wpb = (p.nw + g - 1) / g;
+  const int64_t r0 = (int64_t)blockIdx.x * rpb, w0 = (int64_t)blockIdx.x * wpb;
+  const uint4* src = static_cast<const uint4*>(p.src);
+  uint4* dst = static_cast<uint4*>(p.dst);
+  if (p.prefetch) {
+    for (int64_t i = (int64_t)threadIdx.x * 8; i < rpb; i += (int64_t)kThreads * 8)
+      if (r0 + i < p.nr) prefetch_l2(src + r0 + i);
+  }
+  pdl_wait();
+  uint4 acc = make_uint4(0u, 0u, 0u, 0u);
+#pragma unroll 4
+  for (int64_t i = threadIdx.x; i < rpb; i += kThreads) {
+    if (r0 + i < p.nr) {
+      const uint4 v = ldg16(src + r0 + i);
+      acc.x ^= v.x; acc.y ^= v.y; acc.z ^= v.z; acc.w ^= v.w;
+    }
+  }
+  for (int64_t j = threadIdx.x; j < wpb; j += kThreads)
+    if (w0 + j < p.nw) st16(dst + w0 + j, acc);
+}
+
+const void* copy_floor_entry() { return (const void*)copy_floor_kernel; }
 
 bool pointwise_kernel(int32_t op, int32_t dtype, int32_t variant, int64_t W, KernelEntry* out,
                       const char** why) {

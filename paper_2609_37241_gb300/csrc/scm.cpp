@@ -36,6 +36,7 @@
 #include <vector>
 
 #include "internal.h"
+#include "measure.h"
 #include "tree.h"
 #include "trident_scm.h"
 
@@ -1834,6 +1835,42 @@ TRIDENT_API int32_t trident_launch_floor(trident_scm_t* scm, void* stream, int32
     const int32_t st = launch_on(scm, &cfg, fn, nullptr);
     if (st != TRIDENT_OK) return st;
     if (scm->ring) record_host_time(scm, t0);
+  }
+  return TRIDENT_OK;
+}
+
+TRIDENT_API int32_t trident_copy_floor(trident_scm_t* scm, void* stream, const void* src, void* dst,
+                                       int64_t read_bytes, int64_t write_bytes, int32_t blocks,
+                                       int32_t sets, int32_t n) {
+  if (!scm || !src || !dst || n < 0 || blocks < 1 || sets < 1 || read_bytes < 16 || write_bytes < 16 ||
+      read_bytes % 16 != 0 || write_bytes % 16 != 0 || reinterpret_cast<uintptr_t>(src) % 16 != 0 ||
+      reinterpret_cast<uintptr_t>(dst) % 16 != 0)
+    return fail(TRIDENT_ERR_INVALID, "bad arguments");
+  if (scm->dry) return fail(TRIDENT_ERR_STATE, "dry-run SCM launches nothing");
+  CUfunction fn = nullptr;
+  const int32_t rs = on_device(scm, [&]() -> int32_t {
+    cudaFunction_t f = nullptr;
+    if (cudaGetFuncBySymbol(&f, copy_floor_entry()) != cudaSuccess || !f)
+      return fail(TRIDENT_ERR_CUDA, "cannot resolve the copy kernel");
+    fn = reinterpret_cast<CUfunction>(f);
+    return TRIDENT_OK;
+  });
+  if (rs != TRIDENT_OK) return rs;
+  CUlaunchConfig cfg;
+  CUlaunchAttribute attr;
+  base_config(scm, stream, &cfg, &attr);
+  cfg.gridDimX = (unsigned)blocks;
+  CopyFloorParams P;
+  P.nr = read_bytes / 16;
+  P.nw = write_bytes / 16;
+  P.prefetch = (scm->opt.flags & TRIDENT_OPT_PDL) ? 1 : 0;
+  void* kp[1] = {&P};
+  for (int32_t i = 0; i < n; ++i) {
+    const int64_t k = i % sets;
+    P.src = static_cast<const char*>(src) + k * read_bytes;
+    P.dst = static_cast<char*>(dst) + k * write_bytes;
+    const int32_t st = launch_on(scm, &cfg, fn, kp);
+    if (st != TRIDENT_OK) return st;
   }
   return TRIDENT_OK;
 }

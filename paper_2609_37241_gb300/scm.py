@@ -113,6 +113,7 @@ def lib():
             "trident_scm_host_times": (c_i32, [c_vp, P(c_u32), c_i32, P(c_i32)]),
             "trident_scm_device_status": (c_i32, [c_vp, c_vp, P(c_u32), c_i32]),
             "trident_launch_floor": (c_i32, [c_vp, c_vp, c_i32]),
+            "trident_copy_floor": (c_i32, [c_vp, c_vp, c_vp, c_vp, c_i64, c_i64, c_i32, c_i32, c_i32]),
             "trident_scm_destroy": (None, [c_vp]),
             "trident_rope_kv_noalloc": (c_i32, [P(trident_args), c_vp, P(c_u32)]),
             "trident_scm_last_error": (ctypes.c_char_p, []),
@@ -236,6 +237,11 @@ def trident_scm_device_status(scm, stream=None, clear=True):
 def trident_launch_floor(scm, stream=None, n=1):
     """Latency-floor probe: n empty kernels launched back to back as a hit launches."""
     return lib().trident_launch_floor(scm, stream, n)
+
+
+def trident_copy_floor(scm, stream, src, dst, read_bytes, write_bytes, blocks, sets, n):
+    """Copy-floor probe: n launches of a chain-shaped copy (src/dst: device addresses)."""
+    return lib().trident_copy_floor(scm, stream, src, dst, read_bytes, write_bytes, blocks, sets, n)
 
 
 def trident_rope_kv_noalloc(args, stream=None, status_word=None):

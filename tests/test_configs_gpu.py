@@ -211,3 +211,36 @@ def test_launch_floor_records_each_launch_with_timing(S):
     stats = s.stats()
     assert stats.hits == 0 and stats.misses == 0
     s.close()
+
+
+@pytest.mark.parametrize("pdl", [False, True])
+def test_copy_floor_probe_writes_the_xor_of_each_threads_reads(S, pdl):
+    """The copy-floor probe: launch i reads set i % sets and writes set i % sets; each written
+    vector is the XOR of the 16-byte vectors its thread read (a model in numpy, ragged grid
+    shares included)."""
+    blocks, sets, rb, wb = 7, 2, 16 * 1000, 16 * 333
+    g = np.random.default_rng(3)
+    src_h = g.integers(0, 2 ** 32, size=(sets, rb // 4), dtype=np.uint32)
+    src = torch.from_numpy(src_h.view(np.int32)).cuda()
+    dst = torch.zeros((sets, wb // 4), dtype=torch.int32, device="cuda")
+    s = S.Scm(device=0, flags=S.OPT_PDL if pdl else 0)
+    st = torch.cuda.current_stream().cuda_stream
+    assert S.trident_copy_floor(s.h, st, src.data_ptr(), dst.data_ptr(), rb, wb, blocks, sets, sets) == S.OK, \
+        S.trident_scm_last_error()
+    torch.cuda.synchronize()
+    s.close()
+    got = dst.cpu().numpy().view(np.uint32).reshape(sets, -1, 4)
+    nr, nw = rb // 16, wb // 16
+    rpb, wpb = -(-nr // blocks), -(-nw // blocks)
+    for k in range(sets):
+        vec = src_h[k].reshape(-1, 4)
+        want = np.zeros((nw, 4), np.uint32)
+        for b in range(blocks):
+            acc = np.zeros((256, 4), np.uint32)
+            for i in range(rpb):
+                if b * rpb + i < nr:
+                    acc[i % 256] ^= vec[b * rpb + i]
+            for j in range(wpb):
+                if b * wpb + j < nw:
+                    want[b * wpb + j] = acc[j % 256]
+        assert np.array_equal(got[k], want), k

@@ -496,3 +496,15 @@ def test_noalloc_rejects_calls_without_heads(S):
     args["tensors"][3] = dict(args["tensors"][3], dtype=cases.DT["fp32"])  # positions must be int32
     st = S.trident_rope_kv_noalloc(cases.lib_args(dict(args, theta=1e4)), None)
     assert st == S.ERR_INVALID
+
+
+def test_copy_floor_probe_rejects_dry_runs_and_bad_arguments(S):
+    s = S.Scm(device=0, flags=S.OPT_DRY_RUN)
+    a, b = 1 << 20, 2 << 20  # never dereferenced: every call below is refused first
+    assert S.trident_copy_floor(s.h, None, a, b, 4096, 1024, 8, 2, 1) == S.ERR_STATE
+    for args in ((a, b, 4095, 1024, 8, 2, 1), (a, b, 4096, 0, 8, 2, 1), (a + 8, b, 4096, 1024, 8, 2, 1),
+                 (a, b, 4096, 1024, 0, 2, 1), (a, b, 4096, 1024, 8, 0, 1), (a, b, 4096, 1024, 8, 2, -1),
+                 (None, b, 4096, 1024, 8, 2, 1)):
+        assert S.trident_copy_floor(s.h, None, *args) == S.ERR_INVALID, args
+    assert S.trident_copy_floor(None, None, a, b, 4096, 1024, 8, 2, 1) == S.ERR_INVALID
+    s.close()
