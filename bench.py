@@ -1080,8 +1080,57 @@ def bench_sweep(c, reps=20, quick=False, tokens=None):
     del g, u, o
     assert_all_hit(s, "sweep")
     s.close()
+    out["rope_kv"] = sweep_rope_kv(c, Ts, reps, peak)
     big = [e for e in out["add_rmsnorm"] + out["swiglu"] if e["T"] >= 4096]
     out["min_frac_measured_T_ge_4096"] = min(e["frac_measured"] for e in big) if big else None
+    return out
+
+
+def sweep_rope_kv(c, Ts, reps, peak):
+    """RoPE + KV append (the single-op kernel) at the Llama layer's shapes (32 / 8 heads, D 128,
+    a cache of 8192 slots, q/k/v rows of one packed qkv row), T <= 8192 tokens of distinct
+    uniform positions. The `reps` launches take consecutive T-token windows of a qkv arena of
+    max(32768, 2 T) tokens; the two caches (16 MB each) are shared by all launches."""
+    t, S, synth = c.torch, c.S, c.synth
+    cfg = synth.LLAMA
+    Hq, Hkv, D, Sc = cfg["Hq"], cfg["Hkv"], cfg["D"], cfg["S"]
+    Ts = [T for T in Ts if T <= Sc]
+    if not Ts:
+        return []
+    W = (Hq + 2 * Hkv) * D
+    Tmax = max(32768, 2 * max(Ts))
+    s = S.Scm(device=c.dev.index or 0)
+    for lay in (S.LAYOUT_ROWSTRIDED, S.LAYOUT_CONTIG):  # a one-token window is also contiguous
+        s.register(S.make_spec(S.OP_ROPE_KV, S.BF16, [Hq, Hkv, D, Sc], 1, 1 << 20, layout=lay,
+                               rope_theta=cfg["theta"]))
+    qkv = synth.act_device((Tmax, W), S.BF16, 16, c.dev)
+    g = np.random.default_rng(17)
+    kc = t.zeros((Hkv, Sc, D), dtype=t.bfloat16, device=c.dev)
+    vc = t.zeros((Hkv, Sc, D), dtype=t.bfloat16, device=c.dev)
+    seq = c.L.trident_scm_invoke_seq
+    out = []
+    for T in Ts:
+        nwin = Tmax // T
+        pos = t.from_numpy(np.stack([synth.positions(g, T, Sc) for _ in range(reps)])).to(c.dev)
+
+        def args(i):
+            w = qkv[(i % nwin) * T:(i % nwin + 1) * T]
+            q = w[:, :Hq * D].view(T, Hq, D)
+            k = w[:, Hq * D:(Hq + Hkv) * D].view(T, Hkv, D)
+            v = w[:, (Hq + Hkv) * D:].view(T, Hkv, D)
+            return S.make_args(S.OP_ROPE_KV, [q, k, v, pos[i], kc, vc],
+                               rope_theta=cfg["theta"])
+        arr = (S.trident_args * reps)(*[args(i) for i in range(reps)])
+        us, _ = time_steps(c, lambda i: seq(s.h, arr, reps, c.sp, None), 3, 2)
+        us /= reps
+        c.launches += 5 * reps
+        b = ((2 * Hq + 4 * Hkv) * D * 2 + 4) * T + D * 4
+        out.append(dict(T=T, us=round(us, 3), gbs=round(b / us / 1e3, 1),
+                        frac_measured=round(b / us / 1e3 / peak, 3),
+                        frac_8tbs=round(b / us / 1e3 / NOMINAL_HBM_GBS, 3)))
+    assert_all_hit(s, "rope sweep")
+    s.close()
+    del qkv, kc, vc
     return out
 
 

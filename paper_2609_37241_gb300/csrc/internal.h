@@ -82,6 +82,13 @@ struct RopeParams {
   int32_t nh_shift;
 };
 
+// RoPE with the block's rows staged by bulk copies (rope_bulk_kernel, calls of many tokens).
+struct RopeBulkParams {
+  RopeParams rp;
+  uint32_t first_wait_polls;  // polls of the wait for the copies (kBulkWaitPolls; 0 under
+                              // TRIDENT_OPT_TEST_WAIT_TIMEOUT)
+};
+
 // out = silu(g) * u over T rows of I elements.
 struct SwigluParams {
   const void* g;
@@ -143,12 +150,13 @@ struct KernelEntry {
   const void* fn_step_role = nullptr;  // chain only: fn_step_inplace, role-major block order
   const void* fn_step = nullptr;          // chain only: several calls per launch (ChainStepParams)
   const void* fn_step_inplace = nullptr;  // ... one block per token for the norms
-  const void* fn_large = nullptr;  // add+RMSNorm: the entry for calls of >= large_rows rows
+  const void* fn_large = nullptr;  // add+RMSNorm / RoPE: the entry for calls of >= large_rows rows
+                                   // (tokens)
   int32_t large_rows = 0;
   int32_t kind = 0;      // which grid rule the host applies (KernelKind)
   int32_t vec = 0;       // elements per vector (VE), or tile width for SwiGLU
   int32_t unroll = 1;    // vectors per thread per tile (SwiGLU, chain)
-  int32_t rows = 1;      // rows per block (KK_NORM_ROWS)
+  int32_t rows = 1;      // rows per block (KK_NORM_ROWS; RoPE's fn_large: tokens per block)
 };
 
 enum KernelKind : int32_t {

@@ -779,6 +779,7 @@ int32_t do_launch(trident_scm* scm, const Version& v, const trident_args* a, con
     RmsNormParams rn;
     PointwiseParams pw;
     RopeParams rp;
+    RopeBulkParams rb;  // rb.rp is rp
     SwigluParams sw;
     ChainParams ch;
   } P;
@@ -800,6 +801,13 @@ int32_t do_launch(trident_scm* scm, const Version& v, const trident_args* a, con
     case TRIDENT_OP_QKNORM_ROPE_KV: {
       pack_rope(a, 0, op == TRIDENT_OP_QKNORM_ROPE_KV ? 6 : -1, v, scm->d_err, &P.rp);
       const int64_t units = P.rp.T * P.rp.NH;
+      if (v.fn_large && s.T >= v.ke.large_rows) {  // bulk-copy kernel: ke.rows tokens per block,
+        const int64_t tpb = v.ke.rows;            // their head-rows staged in shared memory
+        cfg.gridDimX = cap_grid((P.rp.T + tpb - 1) / tpb);
+        cfg.sharedMemBytes = (unsigned)(tpb * P.rp.NH * P.rp.D * 2);
+        P.rb.first_wait_polls = (scm->opt.flags & TRIDENT_OPT_TEST_WAIT_TIMEOUT) ? 0u : kBulkWaitPolls;
+        break;
+      }
       const int64_t upb = v.ke.kind == KK_ROPE_HALFWARP ? rope_units_per_block(P.rp.D, 2) : kThreads / 32;
       cfg.gridDimX = cap_grid((units + upb - 1) / upb);
       break;
@@ -902,7 +910,8 @@ int32_t do_launch(trident_scm* scm, const Version& v, const trident_args* a, con
     fn = wide ? v.fn_wide : v.fn_inplace;
   else if (late && v.fn_late)
     fn = v.fn_late;
-  if (v.fn_large && s.T >= v.ke.large_rows) fn = v.fn_large;  // many rows: the bulk-copy kernel
+  if (v.fn_large && s.T >= v.ke.large_rows) fn = v.fn_large;  // many rows: add+RMSNorm's bulk-copy
+                                                              // kernel, RoPE's several rows per lane
   return launch_on(scm, &cfg, fn, kp);
 }
 
@@ -1301,6 +1310,27 @@ int32_t append_version(trident_scm_t* scm, const trident_spec_desc* desc, int32_
         if (cudaGetFuncBySymbol(&h, v.ke.fn_large) != cudaSuccess || !h)
           return fail(TRIDENT_ERR_CUDA, "cannot resolve the large-call kernel entry");
         v.fn_large = reinterpret_cast<CUfunction>(h);
+        if (v.ke.kind == KK_ROPE_HALFWARP) {
+          // the bulk-copy RoPE kernel stages ke.rows tokens' head-rows in dynamic shared memory:
+          // allow up to what the device gives a block (one setting for every version), or
+          // leave such calls to the vector kernel when a version's rows do not fit
+          const int64_t need = (int64_t)v.ke.rows * (v.d.fixed[0] + 2 * v.d.fixed[1]) * v.d.fixed[2] * 2;
+          int dev = 0, optin = 0;
+          cudaFuncAttributes fa;
+          if (cudaGetDevice(&dev) != cudaSuccess ||
+              cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) != cudaSuccess ||
+              cudaFuncGetAttributes(&fa, v.ke.fn_large) != cudaSuccess)
+            return fail(TRIDENT_ERR_CUDA, "cannot read the shared-memory limits");
+          const int64_t room = (int64_t)optin - (int64_t)fa.sharedSizeBytes;
+          if (need > room) {
+            v.fn_large = nullptr;
+          } else if (cudaFuncSetAttribute(v.ke.fn_large, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)room) !=
+                         cudaSuccess ||
+                     cudaFuncSetAttribute(v.ke.fn_large, cudaFuncAttributePreferredSharedMemoryCarveout,
+                                          (int)cudaSharedmemCarveoutMaxShared) != cudaSuccess) {
+            return fail(TRIDENT_ERR_CUDA, "cannot set the RoPE kernel's shared-memory size");
+          }
+        }
       }
       if (v.ke.fn_inplace) {
         cudaFunction_t g = nullptr;

@@ -315,7 +315,7 @@ def rope_inputs(g, T, Hq, Hkv, D, S_, dtype):
 
 
 def run_rope(S, T, Hq, Hkv, D, S_, theta, qknorm, dtype=BF16, layout="fused", variant=0,
-             pos_override=None, seed=1):
+             pos_override=None, seed=1, flags=0):
     g = np.random.default_rng(seed)
     q, k, v, pos = rope_inputs(g, T, Hq, Hkv, D, S_, dtype)
     if pos_override is not None:
@@ -347,7 +347,7 @@ def run_rope(S, T, Hq, Hkv, D, S_, theta, qknorm, dtype=BF16, layout="fused", va
         ts += [torch.from_numpy(gq).cuda(), torch.from_numpy(gk).cuda()]
     desc = S.make_spec(op, dtype, [Hq, Hkv, D, S_], 1, 1 << 20, layout=lay,
                        align_bytes=2 if variant == 1 else 16, variant=variant, rope_theta=theta)
-    s = one_version_scm(S, desc)
+    s = one_version_scm(S, desc, flags=flags)
     invoke_ok(s, S, S.make_args(op, ts, eps=1e-6, rope_theta=theta))
     st, bits = S.trident_scm_device_status(s.h, stream())
     assert st == S.OK
@@ -384,6 +384,43 @@ def test_rope_bad_positions_flag_and_skip(S):
         ref, got, inp = run_rope(S, 5, 4, 2, 128, 512, 1e4, True, pos_override=pos, variant=variant)
         assert ref["bad"] == 1 and got["status"] == S.DEVERR_POS
         check_rope(ref, got, inp)
+
+
+@pytest.mark.parametrize("T,Hq,Hkv,D,S_,qk,dtype,layout", [
+    (515, 32, 8, 128, 8192, False, BF16, "fused"),     # Llama heads; the last block holds 3 tokens
+    (1024, 32, 8, 128, 8192, True, FP16, "separate"),  # Qwen3-style q/k norm
+    (601, 4, 2, 64, 1024, True, BF16, "fused"),
+    (512, 8, 8, 256, 600, False, FP16, "separate"),
+    (2050, 16, 1, 128, 4096, False, BF16, "fused")])
+def test_rope_kv_many_tokens(S, T, Hq, Hkv, D, S_, qk, dtype, layout):
+    """Calls of at least 512 tokens: the bulk-copy kernel (a few tokens per block, their rows
+    staged in shared memory, each token's angles computed once), ragged last blocks included."""
+    ref, got, inp = run_rope(S, T, Hq, Hkv, D, S_, 5e5, qk, dtype=dtype, layout=layout, seed=T + D)
+    assert got["status"] == 0 and ref["bad"] == 0
+    check_rope(ref, got, inp, dtype)
+
+
+def test_rope_kv_many_tokens_bad_positions(S):
+    T = 603
+    pos = synth.positions(np.random.default_rng(5), T, 8192)
+    pos[100], pos[601] = 8192, -5  # outside [0, 8192): one in a full block, one in the last
+    ref, got, inp = run_rope(S, T, 32, 8, 128, 8192, 5e5, True, pos_override=pos)
+    assert ref["bad"] >= 1 and got["status"] == S.DEVERR_POS
+    check_rope(ref, got, inp)
+
+
+def test_rope_kv_bulk_copy_wait_timeout_path(S):
+    """The bulk-copy RoPE kernel's bounded wait for its row copies, made to run out
+    (TRIDENT_OPT_TEST_WAIT_TIMEOUT: the first wait gives up at once): every block sets the
+    timeout bit, drains its copies with the full bounded wait and returns without writing,
+    so q, k, v and both caches keep their contents."""
+    T, Hq, Hkv, D, S_ = 600, 32, 8, 128, 8192
+    ref, got, inp = run_rope(S, T, Hq, Hkv, D, S_, 5e5, False, flags=S.OPT_TEST_WAIT_TIMEOUT)
+    q, k, v, _ = inp
+    assert got["status"] == S.DEVERR_TIMEOUT
+    assert np.array_equal(got["q"], q) and np.array_equal(got["k"], k) and np.array_equal(got["v"], v)
+    sentinel = synth.cache(Hkv, S_, D)
+    assert np.array_equal(got["k_cache"], sentinel) and np.array_equal(got["v_cache"], sentinel)
 
 
 # ---------------------------------------------------------------------------- SwiGLU
