@@ -338,7 +338,10 @@ typedef int32_t (*trident_compile_hook)(void* user, trident_scm_t* scm, const tr
 
 /* ---------------------------------------------------------------- entry points */
 
-/* Version of this ABI (TRIDENT_ABI_VERSION). */
+/* Version of this ABI (TRIDENT_ABI_VERSION). §3.4: one packed ABI is the common boundary
+ * between the dispatcher and its callers, exposed under one stable entry symbol; a caller
+ * built against another layout of the structs below checks this number before its first
+ * call instead of passing misread arguments. Needs no GPU; never fails. */
 int32_t trident_abi_version(void);
 
 /* Creates an empty SCM (§3.5: an empty SCM takes the miss path first).
@@ -373,7 +376,8 @@ int32_t trident_scm_register_spec(trident_scm_t* scm, const trident_spec_desc* d
 int32_t trident_scm_invoke(trident_scm_t* scm, const trident_args* args, void* stream,
                            int32_t* out_selected);
 
-/* Invokes args[0..n-1] in order with one call (one boundary crossing per decoder step).
+/* Invokes args[0..n-1] in order with one call (one boundary crossing per decoder step;
+ * §3.5: the hit path stays on the compiled side of a single entry call from the caller).
  * Each element behaves as trident_scm_invoke. Stops at the first element that returns
  * an error or MISS and returns that status; the elements after it get TRIDENT_NOT_RUN
  * in out_selected (n entries, may be NULL). Returns OK if all hit, else MISS_HANDLED
@@ -436,7 +440,8 @@ int32_t trident_scm_invoke_tree(trident_scm_t* scm, const trident_node* nodes, i
                                 int32_t nnodes, void* stream, int32_t* out_selected);
 
 /* Installs (or with NULL removes) the compile hook of invoke_tree; same rules as the
- * invoke hook (called only on a miss, never from inside a hook). */
+ * invoke hook (§3.5: the caller's compile path runs only on a miss, never from inside a
+ * hook). Errors: ERR_INVALID (scm NULL). */
 int32_t trident_scm_set_tree_hook(trident_scm_t* scm, trident_tree_hook hook, void* user);
 
 /* Selection only: validation plus Algorithm 1's guard loop, with no launch, no hook
@@ -454,16 +459,25 @@ int32_t trident_scm_select(const trident_scm_t* scm, const trident_args* args,
  * invokers are updating may be a few calls apart. Errors: ERR_INVALID (scm or out NULL). */
 int32_t trident_scm_stats(const trident_scm_t* scm, trident_scm_stats_t* out);
 
-/* Copies per-version hit counts into out[0..cap-1]; *n (may be NULL) gets the count. */
+/* Copies per-version hit counts into out[0..cap-1]; *n (may be NULL) gets the count.
+ * §3.5: versions are tried in creation order and later compatible calls use a newly
+ * installed version; these counts show which version each hit selected (index order is
+ * creation order). Errors: ERR_INVALID (scm NULL, cap < 0, or out NULL with cap > 0). */
 int32_t trident_scm_spec_hits(const trident_scm_t* scm, uint64_t* out, int32_t cap, int32_t* n);
 
-/* With TRIDENT_OPT_TIMING: copies the host nanoseconds of the most recent hits (entry
+/* §4.1 and §2.3: host latency is the time until the call returns to its caller, read on
+ * the warm path over many repeated calls (median and spread).
+ * With TRIDENT_OPT_TIMING: copies the host nanoseconds of the most recent hits (entry
  * of invoke to return, launch included) into out[0..cap-1], oldest first; *n gets the
  * count. Samples are recorded per hit (and per launch of trident_launch_floor), so
- * concurrent invokers may interleave. */
+ * concurrent invokers may interleave. Errors: ERR_INVALID (scm NULL, cap < 0, or out NULL
+ * with cap > 0), ERR_STATE (TRIDENT_OPT_TIMING off). */
 int32_t trident_scm_host_times(const trident_scm_t* scm, uint32_t* out, int32_t cap, int32_t* n);
 
-/* Latency-floor probe (measurement, not part of the dispatch path): launches n empty
+/* Latency-floor probe (measurement, not part of the dispatch path; the paper has no such
+ * probe). §2.3: on short kernels what remains on the warm path is host and launch cost,
+ * and §4.1 reads end-to-end latency until the device finishes; this probe gives the part
+ * of both that no dispatcher can remove, one launch. It launches n empty
  * kernels (one block of 32 threads; the kernel only takes part in programmatic dependent
  * launch) back to back on `stream`, with the SCM's launch configuration (its context, and
  * programmatic stream serialisation when TRIDENT_OPT_PDL is set) through the same driver
@@ -474,7 +488,9 @@ int32_t trident_scm_host_times(const trident_scm_t* scm, uint32_t* out, int32_t 
  * ERR_INVALID (scm NULL or n < 0), ERR_STATE (dry-run SCM), ERR_CUDA. */
 int32_t trident_launch_floor(trident_scm_t* scm, void* stream, int32_t n);
 
-/* Copy-floor probe (measurement, not part of the dispatch path): n launches, back to back on
+/* Copy-floor probe (measurement, not part of the dispatch path; the paper has no such
+ * probe). §4.1 reads end-to-end latency until the device finishes; for a memory-bound
+ * launch that time is bounded below by moving its bytes, which this probe measures: n launches, back to back on
  * `stream` through the same launch code as a hit, of a kernel with a layer chain's traffic
  * and none of its arithmetic. Launch i reads read_bytes at src + (i % sets) * read_bytes and
  * writes write_bytes at dst + (i % sets) * write_bytes with a grid of `blocks` blocks of 256
@@ -490,7 +506,12 @@ int32_t trident_copy_floor(trident_scm_t* scm, void* stream, const void* src, vo
                            int64_t write_bytes, int32_t blocks, int32_t sets, int32_t n);
 
 /* Reads the device status word (TRIDENT_DEVERR_* bits) after synchronising `stream`;
- * clears it when clear != 0. Errors: ERR_STATE in dry-run mode, ERR_CUDA. */
+ * clears it when clear != 0. §3.5: an execution error is a path of its own, never a miss
+ * and never a reason to try another version; an error found inside a kernel (a position
+ * outside the cache, a bounded wait that ran out) cannot return through the launch, so the
+ * kernel sets its bit here and skips the faulty access, and the caller reads it after the
+ * work has finished. Errors: ERR_INVALID (scm or out_bits NULL), ERR_STATE in dry-run mode,
+ * ERR_CUDA. */
 int32_t trident_scm_device_status(trident_scm_t* scm, void* stream, uint32_t* out_bits,
                                   int32_t clear);
 
@@ -530,7 +551,8 @@ void trident_scm_destroy(trident_scm_t* scm);
  * overwritten by that thread's next failing call. */
 const char* trident_scm_last_error(void);
 
-/* Static name of a status code. */
+/* Static name of a status code (§3.4-3.5: a miss and an execution error are distinct
+ * outcomes; the name says which). Unknown codes give "UNKNOWN". Never fails. */
 const char* trident_status_name(int32_t status);
 
 #ifdef __cplusplus

@@ -50,6 +50,24 @@ def test_exports_every_declared_symbol(S):
     assert S.trident_abi_version() == 4
 
 
+def test_every_entry_point_cites_its_passage():
+    """Each prototype's comment block names the paper passage that defines the call (a
+    section or Algorithm 1); the allocation-free entry says instead that the paper has no
+    counterpart."""
+    header = open(os.path.join(ROOT, "include", "trident_scm.h")).read()
+    entries = header.split("/* ---------------------------------------------------------------- entry points */")[1]
+    blocks = re.findall(r"(/\*(?:[^*]|\*(?!/))*\*/)\s*(?:#define[^\n]*\n\s*)?[\w\s\*]+?\b(trident_\w+)\s*\(", entries)
+    names = [n for _, n in blocks]
+    declared = {d for d in re.findall(r"^\s*(?:[\w\s\*]+?)\b(trident_\w+)\s*\(", header, re.M)
+                if not d.endswith("_t")}
+    assert len(names) == len(set(names)) and set(names) == declared
+    for comment, name in blocks:
+        if name == "trident_rope_kv_noalloc":
+            assert "no counterpart" in comment, name
+        else:
+            assert re.search(r"§\d|Algorithm 1", comment), name
+
+
 def test_binding_constants_match_header_defines(S):
     header = open(os.path.join(ROOT, "include", "trident_scm.h")).read()
     defines = dict(re.findall(r"^#define TRIDENT_(\w+) \(?(-?(?:0x)?[0-9a-fA-F]+)u?\)?", header, re.M))
