@@ -1373,15 +1373,15 @@ def run_ours(a):
                     config=dict(workload="llama decode layer non-GEMM chain: 64 tokens, H 4096, 32/8 "
                                          "heads, D 128, I 14336, theta 5e5, KV cache [8,8192,128]",
                                 tokens=HEADLINE_T, path="fused chain, 1 launch per step, PDL",
-                                lead="a 24 us sleep kernel ahead of the first timed step keeps the "
+                                l2="inputs rotated over %d sets (%.0f MB > 2x L2)" % (
+                                    R, R * chain_bytes_per_token(cfg) * HEADLINE_T / 2 ** 20),
+                                parallelism="replicas" if world > 1 else "single GPU"),
+                    timing=dict(lead="a 24 us sleep kernel ahead of the first timed step keeps the "
                                      "device busy while the host issues the first steps (outside "
                                      "the timed window)",
                                 warmup_steps_run=W_run,
                                 warmup_note="max(W, sets): every rotating set is visited once "
-                                            "before timing",
-                                l2="inputs rotated over %d sets (%.0f MB > 2x L2)" % (
-                                    R, R * chain_bytes_per_token(cfg) * HEADLINE_T / 2 ** 20),
-                                parallelism="replicas" if world > 1 else "single GPU"),
+                                            "before timing"),
                     gpu_launches=headline_launches, gpu_launches_whole_run=c.launches,
                     python_binding="fastcall" if c.fc is not None else "ctypes")
         line.update(extra)
@@ -1437,7 +1437,11 @@ def run_reference(a):
                 warmup=a.warmup, ms_per_step=round(us / 1e3, 4), higher_is_better=False,
                 scaling="weak", vs_baseline=None, dtype="f64", data="synthetic", impl="reference",
                 config=dict(workload="llama decode layer non-GEMM chain: 64 tokens, H 4096, 32/8 heads, "
-                                     "D 128, I 14336, theta 5e5, KV cache [8,8192,128]", tokens=HEADLINE_T),
+                                     "D 128, I 14336, theta 5e5, KV cache [8,8192,128]", tokens=HEADLINE_T,
+                            path="CPU oracle (plain C, fp64 arithmetic): the whole chain per step on a "
+                                 "sample of the tokens",
+                            l2="host CPU arm: no GPU cache to flush",
+                            parallelism="single process (rank 0)"),
                 cpu_baseline=dict(value=round(us, 1), unit=UNIT, cores=1, kind="oracle",
                                   sample="each step: the layer chain on %d of the 64 tokens, scaled "
                                          "to 64 (median of %d steps)" % (Ts, a.steps)),
