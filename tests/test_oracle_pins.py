@@ -255,6 +255,38 @@ def test_qknorm_then_rope_keeps_normalised_rms():
         assert np.allclose(got, np.sqrt(ms / (ms + eps)), rtol=1e-12)
 
 
+def test_qknorm_weights_each_head_element_before_the_rotation():
+    """Distinct, non-uniform q and k norm weights. At position 0 (the identity rotation) each
+    head's output divided by its own weights is proportional to the input head with RMS
+    sqrt(ms / (ms + eps)); at any position the rotation keeps the norm of each rotated pair
+    (i, i + D/2) equal to that of the weighted, normalised inputs. Swapped q/k weights,
+    weights applied after the rotation, or weights indexed from the wrong half fail one of
+    these."""
+    g = np.random.default_rng(21)
+    T, Hq, Hkv, D, S, eps = 4, 3, 2, 64, 64, 1e-3
+    q, k, v = (synth.act(g, (T, h, D), BF16) for h in (Hq, Hkv, Hkv))
+    pos = np.array([0, 17, 0, 63], np.int32)
+    gq = (1.0 + 0.3 * g.standard_normal(D)).astype(np.float32)
+    gk = (1.0 - 0.4 * g.standard_normal(D)).astype(np.float32)
+    out = L.rope_kv(q, k, v, pos, synth.cache(Hkv, S, D), synth.cache(Hkv, S, D), 1e6, BF16,
+                    qknorm=True, gamma_q=gq, gamma_k=gk, eps=eps)
+    half = D // 2
+    for src, ref, gam in ((q, out["q_ref"], gq), (k, out["k_ref"], gk)):
+        w = L.widen(src, BF16)
+        gam = gam.astype(np.float64)
+        ms = (w * w).mean(axis=2, keepdims=True)
+        for t in np.flatnonzero(pos == 0):
+            unweighted = ref[t] / gam
+            assert np.allclose(np.sqrt((unweighted ** 2).mean(axis=1)), np.sqrt(ms[t, :, 0] / (ms[t, :, 0] + eps)),
+                               rtol=1e-12)
+            ratio = unweighted / w[t]
+            assert np.allclose(ratio, ratio[:, :1], rtol=1e-12)
+        weighted = w * gam / np.sqrt(ms + eps)
+        pair_in = weighted[..., :half] ** 2 + weighted[..., half:] ** 2
+        pair_out = ref[..., :half] ** 2 + ref[..., half:] ** 2
+        assert np.allclose(pair_out, pair_in, rtol=1e-12)
+
+
 # ---------------------------------------------------------------------------- SwiGLU
 def test_swiglu_closed_forms():
     vals = np.array([0.0, 1.0, -1.0, 20.0, -30.0, 3.0], np.float32)
