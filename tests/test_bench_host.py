@@ -70,3 +70,31 @@ def test_committed_dram_counters_match_the_algorithmic_bytes():
         pytest.skip("chain sources changed since the counters were taken")
     rd, wr = got
     assert abs(rd - r_alg) <= 0.1 * r_alg and abs(wr - w_alg) <= 0.1 * w_alg
+
+
+def _run_reference(env_extra):
+    import subprocess
+    import sys
+    env = dict(os.environ, **env_extra)
+    return subprocess.run([sys.executable, os.path.join(ROOT, "bench.py"), "--impl", "reference",
+                           "--steps", "3", "--warmup", "3", "--quick"],
+                          capture_output=True, text=True, env=env, cwd=ROOT, timeout=600)
+
+
+def test_reference_arm_prints_one_line_on_the_headline_workload(built_lib):
+    """The reference arm (the CPU oracle, as it stands) prints exactly one JSON line with the
+    GPU arm's metric, unit and direction, the headline workload, and its CPU-baseline and
+    end-to-end objects; under a multi-rank launch only rank 0 prints."""
+    r = _run_reference({"RANK": "0", "WORLD_SIZE": "1"})
+    assert r.returncode == 0, r.stderr
+    lines = [ln for ln in r.stdout.splitlines() if ln.startswith("{")]
+    assert len(lines) == 1
+    d = json.loads(lines[0])
+    assert d["impl"] == "reference" and d["metric"] == bench.METRIC and d["unit"] == bench.UNIT
+    assert d["higher_is_better"] is False and d["steps"] == 3 and d["warmup"] == 3
+    assert set(d["config"]) == {"workload", "tokens", "path", "l2", "parallelism"}
+    assert d["config"]["tokens"] == bench.HEADLINE_T
+    assert d["cpu_baseline"]["kind"] == "oracle" and d["cpu_baseline"]["value"] == d["value"] > 0
+    assert d["e2e"] == dict(value=d["value"], unit=d["unit"], h2d_bytes_per_step=0, d2h_bytes_per_step=0)
+    r1 = _run_reference({"RANK": "1", "WORLD_SIZE": "2"})
+    assert r1.returncode == 0 and not [ln for ln in r1.stdout.splitlines() if ln.startswith("{")]
